@@ -1,0 +1,227 @@
+"""Python access to the CPU oracle (liboracle.so).
+
+TEST INFRASTRUCTURE: imported only by tests/, __graft_entry__.smoke() and bench.py's CPU-baseline
+leg.  The GPU library never imports or calls it.
+
+The functions below marshal numpy arrays into the C oracle; the compositions at the bottom
+(`tp_attention`, `tp_ffn`, `tp_layer`) wire the blocks together the way tensor parallelism does
+in Voltron Section 3.2.1: every device gets the same layer input, computes its shard, and the
+shard outputs are summed (with the residual) on the main device.
+"""
+from __future__ import annotations
+
+import ctypes
+from typing import Dict, List, Optional, Sequence, Tuple
+
+import numpy as np
+
+from . import build as _build
+
+_lib = None
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_F64 = ctypes.c_double
+
+
+class OrShapes(ctypes.Structure):
+    _fields_ = [("d_model", _I32), ("n_heads", _I32), ("n_kv_heads", _I32), ("d_head", _I32),
+                ("d_ffn", _I32), ("rms_eps", _F64), ("rope_theta", _F64)]
+
+
+class OrLayer(ctypes.Structure):
+    _fields_ = [(n, _P) for n in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate",
+                                  "w_up", "w_down")]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        L = ctypes.CDLL(str(_build.build()))
+        L.or_num_threads.restype = _I32
+        L.or_set_threads.argtypes = [_I32]
+        L.or_f16_to_f64.argtypes = [ctypes.c_uint16]
+        L.or_f16_to_f64.restype = _F64
+        L.or_f64_to_f16.argtypes = [_F64]
+        L.or_f64_to_f16.restype = ctypes.c_uint16
+        L.or_rmsnorm.argtypes = [_P, _P, _I32, _F64, _P]
+        L.or_rope.argtypes = [_P, _I32, _I64, _F64]
+        L.or_silu.argtypes = [_F64]
+        L.or_silu.restype = _F64
+        L.or_attend.argtypes = [_P, _P, _P, _I64, _I32, _P, _P]
+        L.or_kv_append.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32, _I32,
+                                   _P, _I32, _I64, _P, _P, _I64]
+        L.or_kv_append.restype = _I32
+        L.or_attn_partial.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32,
+                                      _I32, _P, _I32, _P, _P, _P, _I64, _P]
+        L.or_attn_partial.restype = _I32
+        L.or_ffn_partial.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32,
+                                     _I32, _P, _I32, _P]
+        L.or_ffn_partial.restype = _I32
+        L.or_combine.argtypes = [ctypes.POINTER(_P), _I32, _I64, _P, _P]
+        _lib = L
+    return _lib
+
+
+def num_threads() -> int:
+    return int(lib().or_num_threads())
+
+
+def set_threads(n: int) -> None:
+    lib().or_set_threads(int(n))
+
+
+def _f16(a: np.ndarray) -> np.ndarray:
+    a = np.ascontiguousarray(a)
+    if a.dtype != np.float16:
+        raise TypeError(f"expected float16, got {a.dtype}")
+    return a
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def shapes_of(wl) -> OrShapes:
+    return OrShapes(wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, wl.rms_eps,
+                    wl.rope_theta)
+
+
+def layer_of(weights: Dict[str, np.ndarray]) -> Tuple[OrLayer, list]:
+    keep = [_f16(weights[n]) for n, _ in OrLayer._fields_]
+    return OrLayer(*[k.ctypes.data for k in keep]), keep
+
+
+# ------------------------------------------------------------------ building blocks ---------
+
+def f16_to_f64(bits: int) -> float:
+    return float(lib().or_f16_to_f64(int(bits)))
+
+
+def f64_to_f16(x: float) -> int:
+    return int(lib().or_f64_to_f16(float(x)))
+
+
+def rmsnorm(x, gain: np.ndarray, eps: float) -> np.ndarray:
+    x = _f64(x)
+    g = _f16(gain)
+    y = np.empty_like(x)
+    lib().or_rmsnorm(x.ctypes.data, g.ctypes.data, x.size, eps, y.ctypes.data)
+    return y
+
+
+def rope(v, pos: int, theta: float) -> np.ndarray:
+    v = _f64(v).copy()
+    lib().or_rope(v.ctypes.data, v.size, int(pos), float(theta))
+    return v
+
+
+def silu(z: float) -> float:
+    return float(lib().or_silu(float(z)))
+
+
+def attend(q, k: np.ndarray, v: np.ndarray) -> Tuple[np.ndarray, np.ndarray]:
+    """q [dh] (fp64), k/v [n_pos, dh] binary16 -> (weights [n_pos], output [dh])."""
+    q = _f64(q)
+    k, v = _f16(k), _f16(v)
+    n_pos, dh = k.shape
+    w = np.empty(n_pos, np.float64)
+    o = np.empty(dh, np.float64)
+    lib().or_attend(q.ctypes.data, k.ctypes.data, v.ctypes.data, n_pos, dh, w.ctypes.data,
+                    o.ctypes.data)
+    return w, o
+
+
+def kv_append(wl, weights, kv_heads: Tuple[int, int], x: np.ndarray, pos0: int,
+              kcache: np.ndarray, vcache: np.ndarray) -> None:
+    """In-place append into the full-layer caches [Hk, cap, dh] (binary16)."""
+    x = _f16(x).reshape(-1, wl.d_model)
+    assert kcache.flags.c_contiguous and vcache.flags.c_contiguous
+    s = shapes_of(wl)
+    L, keep = layer_of(weights)
+    rc = lib().or_kv_append(ctypes.byref(s), ctypes.byref(L), kv_heads[0], kv_heads[1],
+                            x.ctypes.data, x.shape[0], int(pos0), kcache.ctypes.data,
+                            vcache.ctypes.data, kcache.shape[1])
+    if rc != 0:
+        raise ValueError("or_kv_append rejected its arguments")
+
+
+def attn_partial(wl, weights, heads: Tuple[int, int], x: np.ndarray, pos: Sequence[int],
+                 kcache: np.ndarray, vcache: np.ndarray) -> np.ndarray:
+    x = _f16(x).reshape(-1, wl.d_model)
+    p = np.ascontiguousarray(pos, dtype=np.int64)
+    assert p.size == x.shape[0]
+    out = np.empty((x.shape[0], wl.d_model), np.float64)
+    s = shapes_of(wl)
+    L, keep = layer_of(weights)
+    rc = lib().or_attn_partial(ctypes.byref(s), ctypes.byref(L), heads[0], heads[1],
+                               x.ctypes.data, x.shape[0], p.ctypes.data, _f16(kcache).ctypes.data,
+                               _f16(vcache).ctypes.data, kcache.shape[1], out.ctypes.data)
+    if rc != 0:
+        raise ValueError("or_attn_partial rejected its arguments")
+    return out
+
+
+def ffn_partial(wl, weights, cols: Tuple[int, int], h: np.ndarray) -> np.ndarray:
+    h = _f16(h).reshape(-1, wl.d_model)
+    out = np.empty((h.shape[0], wl.d_model), np.float64)
+    s = shapes_of(wl)
+    L, keep = layer_of(weights)
+    rc = lib().or_ffn_partial(ctypes.byref(s), ctypes.byref(L), cols[0], cols[1], h.ctypes.data,
+                              h.shape[0], out.ctypes.data)
+    if rc != 0:
+        raise ValueError("or_ffn_partial rejected its arguments")
+    return out
+
+
+def combine(partials: Sequence[np.ndarray], residual: Optional[np.ndarray]) -> np.ndarray:
+    parts = [_f64(p) for p in partials]
+    count = parts[0].size if parts else (residual.size if residual is not None else 0)
+    arr = (_P * max(1, len(parts)))(*[p.ctypes.data for p in parts])
+    out = np.empty(count, np.float16)
+    res = _f16(residual).reshape(-1) if residual is not None else None
+    lib().or_combine(arr, len(parts), count, res.ctypes.data if res is not None else None,
+                     out.ctypes.data)
+    shape = parts[0].shape if parts else residual.shape
+    return out.reshape(shape)
+
+
+# ------------------------------------------------------------------ compositions ------------
+
+def kv_heads_of(wl, heads: Tuple[int, int]) -> Tuple[int, int]:
+    g = wl.n_heads // wl.n_kv_heads
+    return heads[0] // g, (heads[1] + g - 1) // g
+
+
+def new_cache(wl, cap: int) -> Tuple[np.ndarray, np.ndarray]:
+    shape = (wl.n_kv_heads, cap, wl.d_head)
+    return np.zeros(shape, np.float16), np.zeros(shape, np.float16)
+
+
+def tp_attention(wl, weights, x: np.ndarray, pos0: int, kcache, vcache,
+                 head_ranges=None) -> Tuple[np.ndarray, List[np.ndarray]]:
+    """One ATTN block under tensor parallelism: every shard appends its KV heads for all rows,
+    then computes its partial; returns (h = binary16(x + sum partials), partials)."""
+    head_ranges = wl.head_ranges if head_ranges is None else head_ranges
+    x = _f16(x).reshape(-1, wl.d_model)
+    rows = x.shape[0]
+    for hr in head_ranges:
+        kv_append(wl, weights, kv_heads_of(wl, hr), x, pos0, kcache, vcache)
+    pos = np.arange(pos0, pos0 + rows)
+    parts = [attn_partial(wl, weights, hr, x, pos, kcache, vcache) for hr in head_ranges]
+    return combine(parts, x), parts
+
+
+def tp_ffn(wl, weights, h: np.ndarray, ffn_ranges=None) -> Tuple[np.ndarray, List[np.ndarray]]:
+    ffn_ranges = wl.ffn_ranges if ffn_ranges is None else ffn_ranges
+    h = _f16(h).reshape(-1, wl.d_model)
+    parts = [ffn_partial(wl, weights, cr, h) for cr in ffn_ranges]
+    return combine(parts, h), parts
+
+
+def tp_layer(wl, weights, x: np.ndarray, pos0: int, kcache, vcache, head_ranges=None,
+             ffn_ranges=None):
+    """Whole decoder layer: returns (h, x_next, attn_partials, ffn_partials)."""
+    h, ap = tp_attention(wl, weights, x, pos0, kcache, vcache, head_ranges)
+    xn, fp = tp_ffn(wl, weights, h, ffn_ranges)
+    return h, xn, ap, fp

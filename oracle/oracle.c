@@ -1,0 +1,280 @@
+/*
+ * CPU oracle for one tensor-parallel shard of a Llama-style decoder layer.
+ *
+ * TEST INFRASTRUCTURE.  Only the tests, the smoke check and the benchmark's CPU-baseline leg
+ * load this library.  It shares no code, header, table or constant with the GPU library.
+ *
+ * Plain loops in fp64.  OpenMP splits only loops whose iterations are independent (output rows
+ * of a matrix-vector product, attention heads); every sum is a sequential accumulation in index
+ * order.  Citations are to the Voltron paper (arXiv 2607.07046):
+ *   - Section 2.1, "LLM Architecture": stacked decoders; attention heads computed independently
+ *     with scaled dot-product of Q, K, V; output linear O; FFN projecting up, applying a
+ *     nonlinearity and projecting back; GQA shares K/V projections across query-head groups.
+ *   - Section 2.1, "LLM Inference": prefill processes the prompt tokens and stores their K and V
+ *     in the KV cache; each decode iteration attends to the cache and appends its own K and V.
+ *   - Section 3.2.1, tensor parallelism: the main device broadcasts the layer input, each device
+ *     computes its shard, and the results are aggregated on the main device.
+ * The Llama-specific forms (RMSNorm, rotate-half RoPE, SwiGLU, no biases) follow the workload
+ * definitions of the target models; the paper names the models but not these formulas.
+ */
+#include "oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* ---------------------------------------------------------------- binary16 ---------------- */
+
+/* binary16: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits.
+ * exponent 0 -> subnormal  (-1)^s * f * 2^-24
+ * exponent 31 -> inf / nan
+ * otherwise   -> (-1)^s * (1024 + f) * 2^(e - 25)                                           */
+double or_f16_to_f64(uint16_t h) {
+    const int s = h >> 15, e = (h >> 10) & 31, f = h & 1023;
+    double mag;
+    if (e == 0)
+        mag = ldexp((double)f, -24);
+    else if (e == 31)
+        mag = f ? NAN : INFINITY;
+    else
+        mag = ldexp((double)(f + 1024), e - 25);
+    return s ? -mag : mag;
+}
+
+/* Round-to-nearest-even encoding.  rint() rounds to even in the default rounding mode, and the
+ * scalings by powers of two are exact, so there is a single rounding. */
+uint16_t or_f64_to_f16(double x) {
+    if (isnan(x)) return 0x7e00;
+    const uint16_t sign = signbit(x) ? 0x8000 : 0;
+    const double a = fabs(x);
+    if (a >= 65520.0) return sign | 0x7c00;            /* halfway above 65504 rounds to inf */
+    if (a < 0x1p-14) {                                  /* subnormal range, quantum 2^-24 */
+        const double q = rint(a * 0x1p24);              /* q == 1024 is the smallest normal */
+        return sign | (uint16_t)q;
+    }
+    int k;
+    frexp(a, &k);                                       /* a = m 2^k, m in [0.5, 1) */
+    int E = k - 1;                                      /* a in [2^E, 2^(E+1)) */
+    double q = rint(ldexp(a, 10 - E));                  /* 11-bit significand in [1024, 2048] */
+    if (q == 2048.0) {
+        q = 1024.0;
+        E += 1;
+    }
+    if (E + 15 >= 31) return sign | 0x7c00;
+    return sign | (uint16_t)(((E + 15) << 10) | ((int)q - 1024));
+}
+
+/* Decoding table, filled from or_f16_to_f64 when the library is loaded. */
+static double g_half[65536];
+
+__attribute__((constructor)) static void or_fill_table(void) {
+    for (int i = 0; i < 65536; ++i) g_half[i] = or_f16_to_f64((uint16_t)i);
+}
+
+#define HALF(b) (g_half[(b)])
+
+int32_t or_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void or_set_threads(int32_t n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
+/* ---------------------------------------------------------------- building blocks --------- */
+
+void or_rmsnorm(const double* x, const uint16_t* gain, int32_t n, double eps, double* y) {
+    double ss = 0.0;
+    for (int32_t i = 0; i < n; ++i) ss += x[i] * x[i];
+    const double r = 1.0 / sqrt(ss / (double)n + eps);
+    for (int32_t i = 0; i < n; ++i) y[i] = x[i] * r * HALF(gain[i]);
+}
+
+void or_rope(double* v, int32_t dh, int64_t pos, double theta) {
+    const int32_t half = dh / 2;
+    for (int32_t i = 0; i < half; ++i) {
+        const double freq = pow(theta, -2.0 * (double)i / (double)dh);
+        const double ang = (double)pos * freq;
+        const double c = cos(ang), s = sin(ang);
+        const double x0 = v[i], x1 = v[i + half];
+        v[i] = x0 * c - x1 * s;
+        v[i + half] = x0 * s + x1 * c;
+    }
+}
+
+double or_silu(double z) { return z / (1.0 + exp(-z)); }
+
+void or_attend(const double* q, const uint16_t* k, const uint16_t* v, int64_t n_pos, int32_t dh,
+               double* w, double* o) {
+    double* s = (double*)malloc(sizeof(double) * (size_t)(n_pos > 0 ? n_pos : 1));
+    const double scale = 1.0 / sqrt((double)dh);
+    double m = -INFINITY;
+    for (int64_t t = 0; t < n_pos; ++t) {
+        double acc = 0.0;
+        for (int32_t c = 0; c < dh; ++c) acc += q[c] * HALF(k[t * dh + c]);
+        s[t] = acc * scale;
+        if (s[t] > m) m = s[t];
+    }
+    double z = 0.0;
+    for (int64_t t = 0; t < n_pos; ++t) {
+        s[t] = exp(s[t] - m);
+        z += s[t];
+    }
+    for (int32_t c = 0; c < dh; ++c) o[c] = 0.0;
+    for (int64_t t = 0; t < n_pos; ++t) {
+        const double wt = s[t] / z;
+        if (w) w[t] = wt;
+        for (int32_t c = 0; c < dh; ++c) o[c] += wt * HALF(v[t * dh + c]);
+    }
+    free(s);
+}
+
+/* y[r] = sum_k W[r * ld + k] * x[k] for r in [0, nrows), k in [0, n). */
+static void matvec(const uint16_t* W, int64_t ld, int64_t nrows, const double* x, int64_t n,
+                   double* y) {
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < nrows; ++r) {
+        const uint16_t* row = W + r * ld;
+        double acc = 0.0;
+        for (int64_t k = 0; k < n; ++k) acc += HALF(row[k]) * x[k];
+        y[r] = acc;
+    }
+}
+
+static void load_row(const uint16_t* src, int32_t n, double* dst) {
+    for (int32_t i = 0; i < n; ++i) dst[i] = HALF(src[i]);
+}
+
+static int shapes_ok(const or_shapes* s) {
+    return s && s->d_model > 0 && s->n_heads > 0 && s->n_kv_heads > 0 && s->d_head > 0 &&
+           (s->d_head % 2) == 0 && s->d_ffn >= 0 && (s->n_heads % s->n_kv_heads) == 0;
+}
+
+/* ---------------------------------------------------------------- attention block --------- */
+
+int32_t or_kv_append(const or_shapes* s, const or_layer* w, int32_t kvh0, int32_t kvh1,
+                     const uint16_t* x, int32_t rows, int64_t pos0, uint16_t* kcache,
+                     uint16_t* vcache, int64_t cap) {
+    if (!shapes_ok(s) || !w || kvh0 < 0 || kvh1 < kvh0 || kvh1 > s->n_kv_heads || rows < 0 ||
+        pos0 < 0 || pos0 + rows > cap)
+        return OR_ERR_ARG;
+    const int32_t D = s->d_model, dh = s->d_head, nk = kvh1 - kvh0;
+    double* xin = (double*)malloc(sizeof(double) * D);
+    double* xh = (double*)malloc(sizeof(double) * D);
+    double* kk = (double*)malloc(sizeof(double) * (size_t)(nk * dh + 1));
+    double* vv = (double*)malloc(sizeof(double) * (size_t)(nk * dh + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        const int64_t p = pos0 + i;
+        load_row(x + (int64_t)i * D, D, xin);
+        or_rmsnorm(xin, w->attn_norm, D, s->rms_eps, xh);
+        matvec(w->wk + (int64_t)kvh0 * dh * D, D, (int64_t)nk * dh, xh, D, kk);
+        matvec(w->wv + (int64_t)kvh0 * dh * D, D, (int64_t)nk * dh, xh, D, vv);
+        for (int32_t j = 0; j < nk; ++j) {
+            or_rope(kk + (int64_t)j * dh, dh, p, s->rope_theta);
+            uint16_t* kd = kcache + ((int64_t)(kvh0 + j) * cap + p) * dh;
+            uint16_t* vd = vcache + ((int64_t)(kvh0 + j) * cap + p) * dh;
+            for (int32_t c = 0; c < dh; ++c) {
+                kd[c] = or_f64_to_f16(kk[(int64_t)j * dh + c]);
+                vd[c] = or_f64_to_f16(vv[(int64_t)j * dh + c]);
+            }
+        }
+    }
+    free(xin);
+    free(xh);
+    free(kk);
+    free(vv);
+    return OR_OK;
+}
+
+int32_t or_attn_partial(const or_shapes* s, const or_layer* w, int32_t h0, int32_t h1,
+                        const uint16_t* x, int32_t rows, const int64_t* pos,
+                        const uint16_t* kcache, const uint16_t* vcache, int64_t cap,
+                        double* partial) {
+    if (!shapes_ok(s) || !w || h0 < 0 || h1 < h0 || h1 > s->n_heads || rows < 0) return OR_ERR_ARG;
+    for (int32_t i = 0; i < rows; ++i)
+        if (pos[i] < 0 || pos[i] >= cap) return OR_ERR_ARG;
+    const int32_t D = s->d_model, dh = s->d_head, H = s->n_heads, nh = h1 - h0;
+    const int32_t group = s->n_heads / s->n_kv_heads;
+    double* xin = (double*)malloc(sizeof(double) * D);
+    double* xh = (double*)malloc(sizeof(double) * D);
+    double* q = (double*)malloc(sizeof(double) * (size_t)(nh * dh + 1));
+    double* o = (double*)malloc(sizeof(double) * (size_t)(nh * dh + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        double* out = partial + (int64_t)i * D;
+        if (nh == 0) {
+            for (int32_t d = 0; d < D; ++d) out[d] = 0.0;
+            continue;
+        }
+        load_row(x + (int64_t)i * D, D, xin);
+        or_rmsnorm(xin, w->attn_norm, D, s->rms_eps, xh);
+        matvec(w->wq + (int64_t)h0 * dh * D, D, (int64_t)nh * dh, xh, D, q);
+        for (int32_t h = 0; h < nh; ++h) or_rope(q + (int64_t)h * dh, dh, pos[i], s->rope_theta);
+#pragma omp parallel for schedule(static)
+        for (int32_t h = 0; h < nh; ++h) {
+            const int32_t j = (h0 + h) / group;
+            or_attend(q + (int64_t)h * dh, kcache + (int64_t)j * cap * dh,
+                      vcache + (int64_t)j * cap * dh, pos[i] + 1, dh, NULL, o + (int64_t)h * dh);
+        }
+        /* partial[d] = sum over the range's columns of Wo[d][h0*dh + k] * o[k] */
+        matvec(w->wo + (int64_t)h0 * dh, (int64_t)H * dh, D, o, (int64_t)nh * dh, out);
+    }
+    free(xin);
+    free(xh);
+    free(q);
+    free(o);
+    return OR_OK;
+}
+
+/* ---------------------------------------------------------------- FFN block --------------- */
+
+int32_t or_ffn_partial(const or_shapes* s, const or_layer* w, int32_t c0, int32_t c1,
+                       const uint16_t* h, int32_t rows, double* partial) {
+    if (!shapes_ok(s) || !w || c0 < 0 || c1 < c0 || c1 > s->d_ffn || rows < 0) return OR_ERR_ARG;
+    const int32_t D = s->d_model, F = s->d_ffn, nc = c1 - c0;
+    double* hin = (double*)malloc(sizeof(double) * D);
+    double* hh = (double*)malloc(sizeof(double) * D);
+    double* g = (double*)malloc(sizeof(double) * (size_t)(nc + 1));
+    double* u = (double*)malloc(sizeof(double) * (size_t)(nc + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        double* out = partial + (int64_t)i * D;
+        if (nc == 0) {
+            for (int32_t d = 0; d < D; ++d) out[d] = 0.0;
+            continue;
+        }
+        load_row(h + (int64_t)i * D, D, hin);
+        or_rmsnorm(hin, w->ffn_norm, D, s->rms_eps, hh);
+        matvec(w->w_gate + (int64_t)c0 * D, D, nc, hh, D, g);
+        matvec(w->w_up + (int64_t)c0 * D, D, nc, hh, D, u);
+        for (int32_t j = 0; j < nc; ++j) g[j] = or_silu(g[j]) * u[j];
+        matvec(w->w_down + c0, F, D, g, nc, out);
+    }
+    free(hin);
+    free(hh);
+    free(g);
+    free(u);
+    return OR_OK;
+}
+
+/* ---------------------------------------------------------------- aggregation ------------- */
+
+void or_combine(const double* const* partials, int32_t n, int64_t count, const uint16_t* residual,
+                uint16_t* out) {
+#pragma omp parallel for schedule(static)
+    for (int64_t e = 0; e < count; ++e) {
+        double acc = residual ? HALF(residual[e]) : 0.0;
+        for (int32_t sidx = 0; sidx < n; ++sidx) acc += partials[sidx][e];
+        out[e] = or_f64_to_f16(acc);
+    }
+}
