@@ -1,0 +1,413 @@
+"""Benchmark: batch-1 decode of the Llama-2-7B-shaped stack, every tensor-parallel shard on one GPU.
+
+One step = one decode token through all 32 layers: for each layer every ATTN shard (4 of them),
+the on-device combine, every FFN shard, the combine; then the KV lengths advance.  The token step
+is one CUDA graph (vt_decode_token captured once) replayed K times; the KV length runs
+1024 -> 1151 and rewinds to 1024 every 128 steps (the 128-step schedule of the workload).
+
+Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs resident in HBM;
+`e2e` is the same metric through the C ABI with host buffers (token id H2D, hidden state D2H,
+synchronised every step); `roofline` is the decode GEMV's achieved HBM bandwidth; `cpu_baseline` is
+the CPU oracle timed on a bounded sample.  `--impl reference` times the CPU oracle alone.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+import numpy as np  # noqa: E402
+
+import synthetic  # noqa: E402
+
+METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def measured_peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return float(d["hbm_gbs"]), float(d.get("bf16_tflops", 1900.0)), \
+            float(d.get("bf16_tflops_sustained", 1700.0)), "measured"
+    return FALLBACK_HBM_GBS, 1900.0, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------------ clocks sampler
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except FileNotFoundError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi"]}
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        load = [r for r in rows if r[2] > 200.0] or rows
+        sm = sorted(r[0] for r in load)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in load for i, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(load), "power_w_max": max(r[2] for r in rows)}
+
+
+# ------------------------------------------------------------------ workload
+
+def shapes_for(vt, wl, max_seq):
+    return vt.make_shapes(wl.n_layers, wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn,
+                          wl.vocab, max_seq, wl.rms_eps, wl.rope_theta)
+
+
+def decode_bytes_per_token(wl, kv_mean):
+    """Algorithmic HBM bytes of one decode token: every shard weight once, the cache read at the
+    mean length (+1 for the new token), the new K/V row written."""
+    D, H, Hk, dh, F, L = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, wl.n_layers
+    w = 2 * (D * (H + 2 * Hk) * dh + D * H * dh + 3 * D * F + 2 * D)
+    kv = 2 * 2 * Hk * dh * (kv_mean + 1)
+    return L * (w + kv)
+
+
+def ffn_gemv_bytes(wl):
+    D, F = wl.d_model, wl.d_ffn
+    return wl.n_layers * 2 * 3 * D * F
+
+
+def kernels_per_token(wl):
+    n = 0
+    g = wl.n_heads // wl.n_kv_heads
+    for (h0, h1), (c0, c1) in zip(wl.head_ranges, wl.ffn_ranges):
+        n += 3 if h1 > h0 else 1
+        n += 2 if c1 > c0 else 1
+    return wl.n_layers * (n + 2) + 1
+
+
+def cpu_baseline_decode(wl, layers=4, tokens=2):
+    """The oracle (as it stands) on `layers` layers x `tokens` decode tokens at KV 1024; tok/s is
+    extrapolated to the full stack by the layer ratio."""
+    import oracle
+    oracle.num_threads()
+    L0 = wl.kv_len
+    ws = [wl.layer_weights(l) for l in range(layers)]
+    caches = [wl.kv_fill(l, L0, L0 + tokens + 1) for l in range(layers)]
+    t0 = time.perf_counter()
+    for t in range(tokens):
+        x = wl.hidden(1, stream=500 + t)
+        for l in range(layers):
+            _, x, _, _ = oracle.tp_layer(wl, ws[l], x, L0 + t, *caches[l])
+    dt = time.perf_counter() - t0
+    per_token = dt / tokens * (wl.n_layers / layers)
+    return {"value": round(1.0 / per_token, 4), "unit": "tok/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"{tokens} decode tokens through layers 0-{layers - 1} of {wl.n_layers} at KV "
+                      f"{L0}, 4-way TP shards; tok/s extrapolated x{wl.n_layers / layers:g} by layers",
+            "seconds": round(dt, 2)}
+
+
+def run_decode(args, rank, world):
+    import torch
+
+    from paper_2607_07046_gb300 import build as vt_build
+    from paper_2607_07046_gb300 import vt
+    from paper_2607_07046_gb300.stack import Stack
+
+    vt_build.build()
+    wl = synthetic.WORKLOADS[2]
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+    sched = wl.decode_steps  # 128-step KV schedule 1024 -> 1151
+    cap = wl.kv_len + sched + 8
+    shapes = shapes_for(vt, wl, cap)
+    stream = torch.cuda.Stream()
+    t_setup = time.perf_counter()
+    with torch.cuda.stream(stream):
+        st = Stack(shapes, wl.layer_weights, wl.head_ranges, wl.ffn_ranges, cap,
+                   embed=wl.embedding(), stream=stream)
+    try:
+        for l in range(wl.n_layers):
+            kc, vc = wl.kv_fill(l, wl.kv_len)
+            for d, (h0, h1) in enumerate(wl.head_ranges):
+                vt.vt_kv_write_raw(st.kv, l, d, kc[h0:h1], vc[h0:h1])
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        setup_s = time.perf_counter() - t_setup
+        D = wl.d_model
+        ids = torch.from_numpy(wl.token_ids(1, stream=1)).cuda()
+        xin = torch.empty(D, dtype=torch.float16, device="cuda")
+        xout = torch.empty(D, dtype=torch.float16, device="cuda")
+        with torch.cuda.stream(stream):
+            vt.vt_embed(st.model, ids, xin, stream)
+        stream.synchronize()
+        # One graph per token: g_tok is one vt_decode_token; g_rew is one vt_decode_token followed
+        # by a rewind of the KV lengths by 128 (the last step of each 128-step schedule).
+        g_tok, g_rew = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(g_tok, stream=stream):
+                vt.vt_decode_token(st.part, st.kv, xin, xout, stream)
+            with torch.cuda.graph(g_rew, stream=stream):
+                vt.vt_decode_token(st.part, st.kv, xin, xout, stream)
+                vt.vt_kv_advance(st.kv, -1, -sched, stream)
+        # the captures moved the host-side length mirror; put device and host back at kv_len
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        pos = 0
+
+        def step():
+            nonlocal pos
+            pos += 1
+            if pos == sched:
+                g_rew.replay()
+                pos = 0
+            else:
+                g_tok.replay()
+
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                step()
+        stream.synchronize()
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        pos = 0
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(torch.cuda.current_device()) as clk:
+            with torch.cuda.stream(stream):
+                e0.record(stream)
+                for _ in range(args.steps):
+                    step()
+                e1.record(stream)
+            e1.synchronize()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        if world > 1:
+            t = torch.tensor([ms], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            ms = float(t.item())
+        ms_per_step = ms / args.steps
+        kv_status = vt.vt_kv_status(st.kv, clear=True)
+        part_status = vt.vt_partition_status(st.part, clear=True)
+
+        # -------------------------------------------------------------- e2e through host buffers
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        pos = 0
+        ids_host = torch.from_numpy(wl.token_ids(max(args.steps, 1), stream=2)).pin_memory()
+        ids_dev = torch.empty(1, dtype=torch.int32, device="cuda")
+        out_host = torch.empty(D, dtype=torch.float16).pin_memory()
+        e2e_steps = max(1, min(args.steps, 256))
+        with torch.cuda.stream(stream):
+            for i in range(min(3, e2e_steps)):
+                ids_dev.copy_(ids_host[i:i + 1], non_blocking=True)
+                vt.vt_embed(st.model, ids_dev, xin, stream)
+                step()
+                out_host.copy_(xout, non_blocking=True)
+                stream.synchronize()
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        pos = 0
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            for i in range(e2e_steps):
+                ids_dev.copy_(ids_host[i:i + 1], non_blocking=True)
+                vt.vt_embed(st.model, ids_dev, xin, stream)
+                step()
+                out_host.copy_(xout, non_blocking=True)
+                stream.synchronize()
+        e2e_s = (time.perf_counter() - t0) / e2e_steps
+        e2e_finite = bool(np.isfinite(out_host.numpy().astype(np.float32)).all())
+
+        # -------------------------------------------------------------- decode GEMV roofline
+        # The FFN shard steps of every layer and shard (gate/up GEMV with SwiGLU + down GEMV) as
+        # one graph: the GEMV kernel family is the dominant cost of the token step.
+        parts = [torch.empty(D, dtype=torch.float32, device="cuda") for _ in range(st.n_devices)]
+        g2 = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(g2, stream=stream):
+                for l in range(wl.n_layers):
+                    for d in range(st.n_devices):
+                        vt.vt_decode_step(st.part, (l, d, 1), xout, None, parts[d], stream)
+            for _ in range(3):
+                g2.replay()
+            reps = max(3, min(20, args.steps // 4 + 3))
+            f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            f0.record(stream)
+            for _ in range(reps):
+                g2.replay()
+            f1.record(stream)
+        f1.synchronize()
+        ffn_ms = f0.elapsed_time(f1) / reps
+        launches_ffn = wl.n_layers * st.n_devices * 2
+    finally:
+        torch.cuda.synchronize()
+        st.close()
+
+    hbm, _, _, peak_kind = measured_peaks()
+    kv_mean = wl.kv_len + (min(args.steps, sched) - 1) / 2.0
+    step_bytes = decode_bytes_per_token(wl, kv_mean)
+    value = world * 1000.0 / ms_per_step
+    ffn_bytes = ffn_gemv_bytes(wl)
+    achieved = ffn_bytes / (ffn_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": "tok/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "fp16",
+        "data": "synthetic (seeded N(0,0.02) fp16 weights, seeded N(0,(0.02*sqrt(D))^2) KV cache)",
+        "config": {
+            "workload": "llama2-7b-shaped batch-1 decode: 32 layers, D 4096, 32 heads x 128 (MHA), "
+                        "FFN 11008 SwiGLU; even 4-way TP (8 heads, 2752 FFN columns per shard), "
+                        "shards run one after another on 1 GPU; KV 1024 -> 1151 (128-step schedule)",
+            "kv_len_start": wl.kv_len,
+            "kv_schedule_steps": sched,
+            "partition": "heads 8/8/8/8, ffn 2752 x 4",
+            "graph": "one CUDA graph per token (vt_decode_token), PDL between kernels",
+            "l2": "no flush: the 13 GB of weights streamed per step exceed the 129 MB L2",
+            "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+            "hbm_bytes_per_step": int(step_bytes),
+        },
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "k_gemv (decode GEMV: gate/up + SwiGLU and down epilogues), FFN shard steps of "
+                      "32 layers x 4 shards replayed as one graph",
+            "achieved": round(achieved, 1),
+            "peak": hbm,
+            "unit": "GB/s",
+            "frac": round(achieved / hbm, 4),
+            "peak_kind": f"{peak_kind} copy bandwidth",
+            "bytes_per_launch": int(ffn_bytes / launches_ffn),
+            "launch_ms": round(ffn_ms / launches_ffn, 6),
+            "traffic": None,
+        },
+        "step_roofline": {
+            "achieved": round(step_bytes / (ms_per_step * 1e-3) / 1e9, 1),
+            "peak": hbm, "unit": "GB/s",
+            "frac": round(step_bytes / (ms_per_step * 1e-3) / 1e9 / hbm, 4),
+            "note": f"whole token step vs {peak_kind} HBM copy bandwidth",
+        },
+        "e2e": {"value": round(world / e2e_s, 3), "unit": "tok/s", "h2d_bytes_per_step": 4,
+                "d2h_bytes_per_step": 2 * D, "finite": e2e_finite},
+        "gpu_launches": kernels_per_token(wl) * args.steps + (args.steps // sched),
+        "device_status": {"kv": kv_status, "partition": part_status},
+        "setup_s": round(setup_s, 1),
+    }
+    return line, clk.summary()
+
+
+# ------------------------------------------------------------------ reference arm (CPU oracle)
+
+def run_reference(args):
+    import oracle
+    wl = synthetic.WORKLOADS[2]
+    w = wl.layer_weights(0)
+    L0 = wl.kv_len
+    kc, vc = wl.kv_fill(0, L0, L0 + args.warmup + args.steps + 1)
+    pos = L0
+    for i in range(args.warmup):
+        oracle.tp_layer(wl, w, wl.hidden(1, stream=600 + i), pos, kc, vc)
+        pos += 1
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.tp_layer(wl, w, wl.hidden(1, stream=700 + i), pos, kc, vc)
+        pos += 1
+    dt = (time.perf_counter() - t0) / max(args.steps, 1)
+    per_token = dt * wl.n_layers
+    value = 1.0 / per_token
+    sample = (f"each step: one decode token through layer 0 of 32 (4-way TP shards, KV from {L0}); "
+              f"tok/s = 1 / (32 x layer time)")
+    return {"metric": METRIC, "value": round(value, 4), "unit": "tok/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(per_token * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": "llama2-7b-shaped batch-1 decode, 4-way TP, KV 1024 (CPU oracle)"},
+            "cpu_baseline": {"value": round(value, 4), "unit": "tok/s", "cores": oracle.num_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": "tok/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=384)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        torch.distributed.init_process_group("nccl")
+    line, clocks = run_decode(args, rank, world)
+    line["clocks"] = clocks
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_decode(synthetic.WORKLOADS[2])
+    if world > 1:
+        import torch
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

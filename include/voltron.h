@@ -1,0 +1,271 @@
+/*
+ * voltron.h - C ABI of the GB300 (sm_103a) library for the per-device tensor-parallel shard of a
+ * Llama-style decoder layer.
+ *
+ * Source of the operation: Voltron (arXiv 2607.07046), Section 3.2.1: under tensor parallelism a
+ * layer is split into shards; the main device broadcasts the layer input, every device computes
+ * its shard with that input, and the shard results are aggregated on the main device, once per
+ * layer.  Section 2.1 fixes what a layer holds: an attention block (independent heads computing
+ * scaled dot-product attention over Q, K, V, then an output linear O; GQA shares K/V heads among
+ * groups of query heads) and a feed-forward block (project up, nonlinearity, project back), and
+ * the two inference phases: prefill (the prompt in parallel, K/V written to the KV cache) and
+ * decode (one token per step, attending to the cache and appending its own K/V).  Section 4.2.1
+ * assigns uneven shares to heterogeneous devices, so partitions are arbitrary contiguous ranges.
+ *
+ * Here every "device" of a partition is a shard executed on the one GPU, one after another; the
+ * broadcast is every shard reading the same device buffer, and the aggregation is vt_combine, an
+ * on-device sum.
+ *
+ * Conventions
+ *  - Dtypes: weights, activations, hidden states and the KV cache are IEEE binary16 ("fp16",
+ *    passed as void*); partial outputs are fp32.  Decode computes in fp32 from fp16 data; prefill
+ *    feeds fp16 operands to the tensor cores with fp32 accumulation.
+ *  - Layouts: row-major.  Linear weights use the nn.Linear layout [out][in].  A hidden-state batch
+ *    is [rows][d_model].
+ *  - Ownership: the library copies weights into its own device buffers, allocated through the
+ *    caller's vt_allocator (or cudaMalloc when it is NULL) and released by the matching destroy
+ *    call.  Every other device pointer is the caller's and must stay valid until the work queued
+ *    on the given stream has finished.
+ *  - Asynchrony: compute calls only enqueue work on `stream` and return.  Host-detectable errors
+ *    (bad arguments, bad shapes or partitions, KV capacity from the host-side length mirror, a
+ *    failed launch) return a nonzero vt_status before anything is enqueued, with a message in
+ *    vt_last_error().  Nothing aborts or traps.  Problems only a kernel can see (a KV length past
+ *    capacity during graph replay, a wait that gave up) set bits in a device status word, read
+ *    with vt_kv_status / vt_partition_status.
+ *  - Threads: objects are not internally locked; use one object from one host thread at a time.
+ *  - Streams and graphs: every compute call can be captured into a CUDA graph; positions come from
+ *    device-resident KV lengths, so a replayed graph appends at the right place.
+ */
+#ifndef VOLTRON_H
+#define VOLTRON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define VT_API __attribute__((visibility("default")))
+#else
+#define VT_API
+#endif
+
+typedef int32_t vt_status;
+#define VT_OK 0
+#define VT_ERR_INVALID_ARG 1      /* null pointer, negative size, unknown enum */
+#define VT_ERR_SHAPE 2            /* vt_shapes not supported (see vt_shapes_validate) */
+#define VT_ERR_PARTITION_OVERLAP 3 /* range d starts before range d-1 ends */
+#define VT_ERR_PARTITION_GAP 4    /* range d starts after range d-1 ends, or the union is short */
+#define VT_ERR_PARTITION_GQA 5    /* a head range does not start and end on a KV-group boundary */
+#define VT_ERR_PARTITION_RANGE 6  /* begin > end, or a bound outside [0, H] / [0, F] */
+#define VT_ERR_KV_CAPACITY 7      /* the call would write past the KV-cache capacity */
+#define VT_ERR_CUDA 8             /* a CUDA runtime call failed (text in vt_last_error) */
+#define VT_ERR_ALLOC 9            /* the allocator returned NULL */
+#define VT_ERR_STATE 10           /* object not ready (e.g. a layer's weights never loaded) */
+
+#define VT_MAX_DEVICES 16
+
+/* Bits of the device status word. */
+#define VT_DEV_KV_OVERFLOW 1u     /* a kernel saw a KV length at or past capacity and skipped */
+#define VT_DEV_WAIT_TIMEOUT 2u    /* a kernel gave up waiting on an asynchronous copy */
+
+typedef void* vt_stream; /* a cudaStream_t; NULL is the legacy default stream */
+
+typedef struct {
+    int32_t n_layers;
+    int32_t d_model;    /* D, multiple of 64 */
+    int32_t n_heads;    /* H, query heads */
+    int32_t n_kv_heads; /* Hk, divides H (H == Hk is MHA) */
+    int32_t d_head;     /* dh, 64 or 128 */
+    int32_t d_ffn;      /* F, SwiGLU intermediate width */
+    int32_t vocab;      /* rows of the embedding table (0: no table) */
+    int32_t max_seq;    /* largest position + 1 that any KV cache may hold */
+    float rms_eps;      /* RMSNorm epsilon (inside the square root) */
+    float rope_theta;   /* RoPE base */
+} vt_shapes;
+
+/* Half-open range [begin, end). */
+typedef struct {
+    int32_t begin, end;
+} vt_range;
+
+/* Device-memory allocator.  alloc(bytes, ctx) returns a device pointer aligned to 256 bytes or
+ * NULL; free(ptr, ctx) releases it.  Both may be called from the thread that calls the library. */
+typedef struct {
+    void* (*alloc)(size_t bytes, void* ctx);
+    void (*free)(void* ptr, void* ctx);
+    void* ctx;
+} vt_allocator;
+
+/* One layer's weights, fp16 host pointers, nn.Linear layout.  Read only during the call. */
+typedef struct {
+    const void* attn_norm; /* [D]        RMSNorm gain of the attention block */
+    const void* wq;        /* [H*dh, D]  */
+    const void* wk;        /* [Hk*dh, D] */
+    const void* wv;        /* [Hk*dh, D] */
+    const void* wo;        /* [D, H*dh]  */
+    const void* ffn_norm;  /* [D]        RMSNorm gain of the FFN block */
+    const void* w_gate;    /* [F, D]     */
+    const void* w_up;      /* [F, D]     */
+    const void* w_down;    /* [D, F]     */
+} vt_layer_weights;
+
+typedef enum { VT_BLOCK_ATTN = 0, VT_BLOCK_FFN = 1 } vt_block;
+
+/* One shard: the `block` of layer `layer` assigned to device `device` of a partition. */
+typedef struct {
+    int32_t layer;
+    int32_t device;
+    int32_t block; /* vt_block */
+} vt_shard;
+
+typedef struct vt_model vt_model;
+typedef struct vt_partition vt_partition;
+typedef struct vt_kv vt_kv;
+
+/* Text of the last error on the calling thread ("" if none).  Valid until the next call. */
+VT_API const char* vt_last_error(void);
+
+/* Library version, "major.minor.patch". */
+VT_API const char* vt_version(void);
+
+/* Host-only checks (no GPU needed).  vt_shapes_validate returns VT_OK or VT_ERR_SHAPE.
+ * vt_partition_validate applies the partition rules of vt_partition below. */
+VT_API vt_status vt_shapes_validate(const vt_shapes* shapes);
+VT_API vt_status vt_partition_validate(const vt_shapes* shapes, int32_t n_devices,
+                                const vt_range* head_ranges, const vt_range* ffn_col_ranges);
+
+/* ---------------------------------------------------------------- model ------------------------
+ * vt_model_create: allocates device storage for every layer in the canonical (unpartitioned)
+ * layout, the RoPE table for positions [0, max_seq) and, if vocab > 0, the embedding table, on
+ * the current CUDA device.  per_layer (nullable) holds n_layers host weight sets, copied now;
+ * embed (nullable) is the host fp16 table [vocab, D].  Layers not given here are loaded later
+ * with vt_model_load_layer.  Synchronizes `stream` before returning (host buffers may be reused).
+ */
+VT_API vt_status vt_model_create(const vt_shapes* shapes, const vt_layer_weights* per_layer,
+                          const void* embed, const vt_allocator* allocator, vt_stream stream,
+                          vt_model** out);
+VT_API vt_status vt_model_load_layer(vt_model* model, int32_t layer, const vt_layer_weights* weights,
+                              vt_stream stream);
+VT_API vt_status vt_model_load_embedding(vt_model* model, const void* embed, vt_stream stream);
+VT_API vt_status vt_model_shapes(const vt_model* model, vt_shapes* out);
+VT_API void vt_model_destroy(vt_model* model);
+
+/* Embedding gather: out[i, :] = E[ids[i], :] for i < n.  ids: device int32 [n] (values outside
+ * [0, vocab) give a zero row and set no error); out: device fp16 [n, D]. */
+VT_API vt_status vt_embed(const vt_model* model, const int32_t* ids, int32_t n, void* out,
+                   vt_stream stream);
+
+/* ---------------------------------------------------------------- partition --------------------
+ * vt_partition: splits every layer among n_devices shards (Section 3.2.1; uneven shares as in
+ * Section 4.2.1).  Device d gets query heads head_ranges[d] of every attention block (and the KV
+ * heads of their groups) and FFN intermediate columns ffn_col_ranges[d] of every FFN block.
+ * Rules: the ranges of each kind are listed in device order, contiguous, disjoint, and cover
+ * [0, H) and [0, F) exactly; empty ranges are allowed (that shard's partial is all zeros); under
+ * GQA every head range starts and ends on a multiple of H/Hk.  Violations return
+ * VT_ERR_PARTITION_* before any device work.  Each (layer, block, device) shard gets its own
+ * allocation holding its weights in the shard-sliced layout, so a shard can be dropped alone.
+ * The model must outlive the partition.  Synchronizes `stream`.
+ */
+VT_API vt_status vt_partition_create(vt_model* model, int32_t n_devices, const vt_range* head_ranges,
+                              const vt_range* ffn_col_ranges, vt_stream stream,
+                              vt_partition** out);
+VT_API int32_t vt_partition_devices(const vt_partition* part);
+/* Reads the device status word (VT_DEV_* bits) of kernels that have no KV cache, synchronizing
+ * the device; clear != 0 resets it. */
+VT_API vt_status vt_partition_status(vt_partition* part, uint32_t* flags, int32_t clear);
+VT_API void vt_partition_destroy(vt_partition* part);
+
+/* Test hook: copies one tensor of a shard's sliced weights to host memory.  which: 0 = attention
+ * RMSNorm gain, 1 = fused QKV rows, 2 = O columns, 3 = FFN RMSNorm gain, 4 = fused gate/up rows,
+ * 5 = down columns.  Copies min(bytes, size) bytes; *size_out (nullable) receives the size.
+ * Layouts are documented beside vt_shard_weight_layout.  Synchronous. */
+VT_API vt_status vt_shard_weights_read(const vt_partition* part, vt_shard shard, int32_t which,
+                                void* host_dst, size_t bytes, size_t* size_out);
+/* Geometry of a shard's sliced tensor: rows and row stride (elements) of tensor `which`.
+ *  which 1 (QKV): rows = (h_s + 2 hk_s) * dh; head block b (q heads, then k heads, then v heads)
+ *    occupies rows [b*dh, (b+1)*dh) and stores, at row b*dh + 2i, the source row of dimension i
+ *    and at row b*dh + 2i + 1 the source row of dimension i + dh/2 (RoPE partners adjacent).
+ *  which 2 (O): rows = D, stride = h_s*dh: columns [h0*dh, h1*dh) of Wo.
+ *  which 4 (gate/up): rows = 2 * c_s: row 2j = gate row c0 + j, row 2j + 1 = up row c0 + j.
+ *  which 5 (down): rows = D, stride = c_s rounded up to 8 (padding zero): columns [c0, c1) of Wd.
+ *  which 0, 3: one row of D. */
+VT_API vt_status vt_shard_weight_layout(const vt_partition* part, vt_shard shard, int32_t which,
+                                 int64_t* rows, int64_t* row_stride);
+
+/* ---------------------------------------------------------------- KV cache ---------------------
+ * vt_kv_create: per (layer, device) fp16 caches K and V, each [hk_s][capacity][dh] for that
+ * device's KV heads (tensor parallelism splits the cache by head), plus one device-resident length
+ * per layer (initially 0) and a host mirror of it.  capacity <= max_seq.  Contents start zeroed.
+ */
+VT_API vt_status vt_kv_create(const vt_partition* part, int32_t capacity, vt_stream stream, vt_kv** out);
+VT_API void vt_kv_destroy(vt_kv* kv);
+VT_API int32_t vt_kv_capacity(const vt_kv* kv);
+/* Adds n to the length of `layer` (or of every layer when layer == -1), on the device (in stream
+ * order) and in the host mirror.  Decode and prefill append at the current length without
+ * advancing it: advance once per layer after all of that layer's attention shards ran. */
+VT_API vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_stream stream);
+/* Sets the length of `layer` (or all when -1) to len, device and host mirror. */
+VT_API vt_status vt_kv_set_length(vt_kv* kv, int32_t layer, int32_t len, vt_stream stream);
+/* Reads the device length of `layer` (synchronizes the stream) and refreshes the host mirror. */
+VT_API vt_status vt_kv_length(vt_kv* kv, int32_t layer, vt_stream stream, int32_t* len);
+/* Reads (and with clear != 0 resets) the device status word of kernels that used this cache. */
+VT_API vt_status vt_kv_status(vt_kv* kv, uint32_t* flags, int32_t clear);
+/* Test hooks, synchronous: copy positions [0, n_pos) of the (layer, device) cache between device
+ * and host.  Host layout [hk_s][n_pos][dh] fp16 for K and for V. */
+VT_API vt_status vt_kv_read(const vt_kv* kv, int32_t layer, int32_t device, int32_t n_pos, void* k_host,
+                     void* v_host);
+VT_API vt_status vt_kv_write_raw(vt_kv* kv, int32_t layer, int32_t device, int32_t n_pos,
+                          const void* k_host, const void* v_host);
+
+/* ---------------------------------------------------------------- shard compute ----------------
+ * vt_decode_step: one decode token through one shard.
+ *   ATTN shard (kv required): x^ = RMSNorm(x); q, k, v of the shard's heads; RoPE on q and k at
+ *   position p = current length of the layer; k, v appended at p; attention of each query head
+ *   over positions 0..p (split-K flash decoding); out_partial = Wo[:, shard cols] . attn.
+ *   FFN shard (kv ignored, may be NULL): x^ = RMSNorm(x); u = silu(Wg x^) * (Wu x^) over the shard's
+ *   columns; out_partial = Wd[:, shard cols] . u.
+ *   x: device fp16 [D] (the block input, identical for every shard); out_partial: device fp32 [D],
+ *   excluding the residual.  Does not advance the KV length.
+ */
+VT_API vt_status vt_decode_step(const vt_partition* part, vt_shard shard, const void* x, vt_kv* kv,
+                         float* out_partial, vt_stream stream);
+
+/* vt_prefill: n prompt rows through one shard (n >= 1).
+ *   ATTN shard: rows sit at positions p0..p0+n-1 with p0 = current length of the layer; row i
+ *   attends causally to positions 0..p0+i (earlier turns' cache included).  K and V of all rows
+ *   are appended.  FFN shard: as decode, row by row.
+ *   x: device fp16 [n, D]; out_partial: device fp32 [n, D]; n <= max_seq.  Does not advance.
+ */
+VT_API vt_status vt_prefill(const vt_partition* part, vt_shard shard, const void* x, int32_t n,
+                     vt_kv* kv, float* out_partial, vt_stream stream);
+
+/* vt_combine: the aggregation on the main device.
+ *   out[e] = fp16(residual[e] + sum_{s=0}^{n-1} partials[s][e]), e < rows*d, summed in fp32 in
+ *   the order s = 0..n-1.  partials: host array of n device pointers to fp32 [rows, d];
+ *   residual: device fp16 [rows, d] or NULL; out: device fp16 [rows, d] (may alias residual).
+ *   1 <= n <= VT_MAX_DEVICES. */
+VT_API vt_status vt_combine(const float* const* partials, int32_t n, int32_t rows, int32_t d,
+                     const void* residual, void* out, vt_stream stream);
+
+/* ---------------------------------------------------------------- whole stack ------------------
+ * vt_decode_token: one decode token through every layer, shards one after another:
+ *   for each layer: every ATTN shard (vt_decode_step), vt_combine with the residual; every FFN
+ *   shard, vt_combine; then every layer's KV length advances by one.
+ *   x_in, x_out: device fp16 [D]; they may be the same buffer.  Uses buffers owned by the
+ *   partition, so one partition runs one vt_decode_token / vt_prefill_tokens at a time.
+ */
+VT_API vt_status vt_decode_token(const vt_partition* part, vt_kv* kv, const void* x_in, void* x_out,
+                          vt_stream stream);
+/* vt_prefill_tokens: n prompt rows through every layer (same order as vt_decode_token), then
+ * every layer's KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same. */
+VT_API vt_status vt_prefill_tokens(const vt_partition* part, vt_kv* kv, const void* x_in, int32_t n,
+                            void* x_out, vt_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VOLTRON_H */

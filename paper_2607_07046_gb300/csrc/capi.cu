@@ -1,0 +1,1128 @@
+// C ABI of the library: validation, object lifetime, the shard-sliced weight layout, the KV-cache
+// geometry, and the orchestration of the decode and prefill kernels for one shard or the whole
+// stack.  Host code only; kernels live in decode.cu and prefill.cu.
+//
+// The operation follows Voltron (arXiv 2607.07046) Section 3.2.1: tensor parallelism splits each
+// layer into shards (attention heads for ATTN, intermediate columns for FFN), every device
+// computes its shard from the same broadcast input, and the shard results are aggregated on the
+// main device.  Section 4.2.1 allows uneven shares.  Section 4.3.1 ("Pruning") motivates one
+// allocation per shard, so one shard's weights can be dropped without touching the others.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+
+using namespace vt;
+
+// ================================================================== errors
+
+namespace {
+
+thread_local std::string t_err;
+
+vt_status fail(vt_status st, const char* fmt, ...) {
+    char buf[1024];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_err = buf;
+    return st;
+}
+
+vt_status ok() {
+    t_err.clear();
+    return VT_OK;
+}
+
+#define VT_CUDA(expr)                                                                        \
+    do {                                                                                     \
+        cudaError_t e_ = (expr);                                                             \
+        if (e_ != cudaSuccess)                                                               \
+            return fail(VT_ERR_CUDA, "%s failed: %s (%s:%d)", #expr, cudaGetErrorString(e_), \
+                        __FILE__, __LINE__);                                                 \
+    } while (0)
+
+#define VT_TRY(expr)                     \
+    do {                                 \
+        vt_status s_ = (expr);           \
+        if (s_ != VT_OK) return s_;      \
+    } while (0)
+
+inline size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+inline int round_up8(int k) { return (k + 7) & ~7; }
+
+// ------------------------------------------------------------------ allocator
+struct Allocator {
+    vt_allocator a{};
+    bool custom = false;
+    void* get(size_t bytes) {
+        if (bytes == 0) bytes = 256;
+        if (custom) return a.alloc(bytes, a.ctx);
+        void* p = nullptr;
+        if (cudaMalloc(&p, bytes) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        return p;
+    }
+    void put(void* p) {
+        if (!p) return;
+        if (custom)
+            a.free(p, a.ctx);
+        else
+            cudaFree(p);
+    }
+};
+
+std::once_flag g_init_once;
+cudaError_t g_init_err = cudaSuccess;
+
+cudaError_t init_library() {
+    std::call_once(g_init_once, [] {
+        const char* e = getenv("VT_NO_PDL");
+        g_use_pdl = !(e && e[0] && e[0] != '0');
+        int dev = 0;
+        g_init_err = cudaGetDevice(&dev);
+        if (g_init_err != cudaSuccess) return;
+        g_init_err = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_init_err != cudaSuccess) return;
+        g_init_err = init_decode_kernels();
+        if (g_init_err != cudaSuccess) return;
+        g_init_err = init_prefill_kernels();
+    });
+    return g_init_err;
+}
+
+}  // namespace
+
+// ================================================================== objects
+
+struct LayerPtrs {
+    __half *attn_norm = nullptr, *wq = nullptr, *wk = nullptr, *wv = nullptr, *wo = nullptr,
+           *ffn_norm = nullptr, *w_gate = nullptr, *w_up = nullptr, *w_down = nullptr;
+};
+
+struct vt_model {
+    vt_shapes s{};
+    Allocator alloc;
+    std::vector<void*> layer_base;
+    std::vector<LayerPtrs> layer;
+    std::vector<char> loaded;
+    __half* embed = nullptr;
+    bool embed_loaded = false;
+    float2* rope = nullptr;
+};
+
+struct AttnShard {
+    void* base = nullptr;
+    __half* norm = nullptr;
+    __half* wqkv = nullptr;  // [(hq + 2 hk) dh][D]
+    __half* wo = nullptr;    // [D][hq dh]
+    int h0 = 0, h1 = 0, kv0 = 0, kv1 = 0;
+};
+
+struct FfnShard {
+    void* base = nullptr;
+    __half* norm = nullptr;
+    __half* wgu = nullptr;  // [2c][D]
+    __half* wd = nullptr;   // [D][ld]
+    int c0 = 0, c1 = 0, ld = 0;
+};
+
+struct DecodeScratch {  // per device of the partition
+    float* q = nullptr;
+    float* attn = nullptr;
+    float* part_ml = nullptr;
+    float* part_o = nullptr;
+    int32_t* tickets = nullptr;
+    float* u = nullptr;
+    int nsplit = 1;
+};
+
+constexpr int kPrefillChunk = 1024;  // rows per prefill pass (longer prompts run in chunks)
+
+struct vt_partition {
+    vt_model* m = nullptr;
+    int n_dev = 0;
+    std::vector<vt_range> heads, cols;
+    std::vector<AttnShard> attn;  // [layer * n_dev + dev]
+    std::vector<FfnShard> ffn;
+    std::vector<DecodeScratch> dec;
+    std::vector<void*> owned;  // every allocation besides the shard bases
+    uint32_t* status = nullptr;
+    // whole-stack buffers
+    float* partials = nullptr;  // [n_dev][kPrefillChunk][D]
+    __half* hbuf = nullptr;     // [kPrefillChunk][D]
+    __half* xbuf = nullptr;     // [kPrefillChunk][D]
+    // prefill scratch
+    __half* p_xhat = nullptr;   // [kPrefillChunk][D]
+    __half* p_q = nullptr;      // [kPrefillChunk][max_hq][dh]
+    __half* p_attn = nullptr;   // [kPrefillChunk][max_hq dh]
+    __half* p_u = nullptr;      // [kPrefillChunk][max_ld]
+    int max_hq = 0, max_ld = 0;
+
+    const AttnShard& a(int l, int d) const { return attn[(size_t)l * n_dev + d]; }
+    const FfnShard& f(int l, int d) const { return ffn[(size_t)l * n_dev + d]; }
+};
+
+struct vt_kv {
+    const vt_partition* p = nullptr;
+    int cap = 0;
+    std::vector<void*> buf;  // [layer * n_dev + dev]: K then V, each [hk][cap][dh]
+    int32_t* len = nullptr;  // device [n_layers]
+    std::vector<int32_t> h_len;
+    uint32_t* status = nullptr;
+    Allocator* alloc() const { return &p->m->alloc; }
+    __half* k(int l, int d) const { return static_cast<__half*>(buf[(size_t)l * p->n_dev + d]); }
+    __half* v(int l, int d) const {
+        const AttnShard& s = p->a(l, d);
+        return k(l, d) + (size_t)(s.kv1 - s.kv0) * cap * p->m->s.d_head;
+    }
+};
+
+// ================================================================== validation
+
+extern "C" const char* vt_last_error(void) { return t_err.c_str(); }
+extern "C" const char* vt_version(void) { return "0.1.0"; }
+
+extern "C" vt_status vt_shapes_validate(const vt_shapes* s) {
+    if (!s) return fail(VT_ERR_INVALID_ARG, "shapes is NULL");
+    if (s->n_layers < 1) return fail(VT_ERR_SHAPE, "n_layers must be >= 1");
+    if (s->d_model < 64 || s->d_model % 64 != 0 || s->d_model > 16384)
+        return fail(VT_ERR_SHAPE, "d_model must be a multiple of 64 in [64, 16384]");
+    if (s->n_heads < 1 || s->n_kv_heads < 1 || s->n_heads % s->n_kv_heads != 0)
+        return fail(VT_ERR_SHAPE, "n_heads must be a positive multiple of n_kv_heads");
+    {
+        const int g = s->n_heads / s->n_kv_heads;
+        if (g != 1 && g != 2 && g != 4 && g != 8)
+            return fail(VT_ERR_SHAPE, "query heads per KV head must be 1, 2, 4 or 8 (got %d)", g);
+    }
+    if (s->d_head != 64 && s->d_head != 128) return fail(VT_ERR_SHAPE, "d_head must be 64 or 128");
+    if ((int64_t)s->n_heads * s->d_head > 16384)
+        return fail(VT_ERR_SHAPE, "n_heads * d_head must be <= 16384");
+    if (s->d_ffn < 1 || s->d_ffn > 32768) return fail(VT_ERR_SHAPE, "d_ffn must be in [1, 32768]");
+    if (s->vocab < 0) return fail(VT_ERR_SHAPE, "vocab must be >= 0");
+    if (s->max_seq < 1 || s->max_seq > (1 << 20))
+        return fail(VT_ERR_SHAPE, "max_seq must be in [1, 2^20]");
+    if (!(s->rms_eps >= 0.f) || !(s->rope_theta > 0.f))
+        return fail(VT_ERR_SHAPE, "rms_eps must be >= 0 and rope_theta > 0");
+    return ok();
+}
+
+static vt_status check_ranges(const vt_range* r, int n, int total, int align, const char* what) {
+    int expect = 0;
+    for (int d = 0; d < n; ++d) {
+        if (r[d].begin < 0 || r[d].end > total || r[d].begin > r[d].end)
+            return fail(VT_ERR_PARTITION_RANGE, "%s range %d [%d, %d) is not inside [0, %d)", what, d,
+                        r[d].begin, r[d].end, total);
+        if (r[d].begin < expect)
+            return fail(VT_ERR_PARTITION_OVERLAP, "%s range %d starts at %d, before %d", what, d,
+                        r[d].begin, expect);
+        if (r[d].begin > expect)
+            return fail(VT_ERR_PARTITION_GAP, "%s range %d starts at %d, leaving [%d, %d) unassigned",
+                        what, d, r[d].begin, expect, r[d].begin);
+        if (align > 1 && (r[d].begin % align != 0 || r[d].end % align != 0))
+            return fail(VT_ERR_PARTITION_GQA,
+                        "%s range %d [%d, %d) does not align to KV groups of %d heads", what, d,
+                        r[d].begin, r[d].end, align);
+        expect = r[d].end;
+    }
+    if (expect != total)
+        return fail(VT_ERR_PARTITION_GAP, "%s ranges cover [0, %d) of [0, %d)", what, expect, total);
+    return VT_OK;
+}
+
+extern "C" vt_status vt_partition_validate(const vt_shapes* s, int32_t n, const vt_range* heads,
+                                           const vt_range* cols) {
+    VT_TRY(vt_shapes_validate(s));
+    if (n < 1 || n > VT_MAX_DEVICES)
+        return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
+    if (!heads || !cols) return fail(VT_ERR_INVALID_ARG, "range arrays must not be NULL");
+    VT_TRY(check_ranges(heads, n, s->n_heads, s->n_heads / s->n_kv_heads, "head"));
+    VT_TRY(check_ranges(cols, n, s->d_ffn, 1, "ffn column"));
+    return ok();
+}
+
+// ================================================================== model
+
+static vt_status upload(void* dst, const void* src, size_t bytes, cudaStream_t st) {
+    if (!src) return fail(VT_ERR_INVALID_ARG, "a weight pointer is NULL");
+    VT_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st));
+    return VT_OK;
+}
+
+extern "C" vt_status vt_model_load_layer(vt_model* m, int32_t l, const vt_layer_weights* w,
+                                         vt_stream stream) {
+    if (!m || !w) return fail(VT_ERR_INVALID_ARG, "model and weights must not be NULL");
+    if (l < 0 || l >= m->s.n_layers) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", l);
+    cudaStream_t st = (cudaStream_t)stream;
+    const vt_shapes& s = m->s;
+    const size_t D = s.d_model, Q = (size_t)s.n_heads * s.d_head, KV = (size_t)s.n_kv_heads * s.d_head,
+                 F = s.d_ffn;
+    LayerPtrs& L = m->layer[l];
+    VT_TRY(upload(L.attn_norm, w->attn_norm, D * 2, st));
+    VT_TRY(upload(L.wq, w->wq, Q * D * 2, st));
+    VT_TRY(upload(L.wk, w->wk, KV * D * 2, st));
+    VT_TRY(upload(L.wv, w->wv, KV * D * 2, st));
+    VT_TRY(upload(L.wo, w->wo, D * Q * 2, st));
+    VT_TRY(upload(L.ffn_norm, w->ffn_norm, D * 2, st));
+    VT_TRY(upload(L.w_gate, w->w_gate, F * D * 2, st));
+    VT_TRY(upload(L.w_up, w->w_up, F * D * 2, st));
+    VT_TRY(upload(L.w_down, w->w_down, D * F * 2, st));
+    VT_CUDA(cudaStreamSynchronize(st));
+    m->loaded[l] = 1;
+    return ok();
+}
+
+extern "C" vt_status vt_model_load_embedding(vt_model* m, const void* embed, vt_stream stream) {
+    if (!m || !embed) return fail(VT_ERR_INVALID_ARG, "model and embed must not be NULL");
+    if (!m->embed) return fail(VT_ERR_STATE, "the model has no embedding table (vocab == 0)");
+    cudaStream_t st = (cudaStream_t)stream;
+    VT_TRY(upload(m->embed, embed, (size_t)m->s.vocab * m->s.d_model * 2, st));
+    VT_CUDA(cudaStreamSynchronize(st));
+    m->embed_loaded = true;
+    return ok();
+}
+
+extern "C" void vt_model_destroy(vt_model* m) {
+    if (!m) return;
+    cudaDeviceSynchronize();
+    for (void* p : m->layer_base) m->alloc.put(p);
+    m->alloc.put(m->embed);
+    m->alloc.put(m->rope);
+    delete m;
+}
+
+extern "C" vt_status vt_model_create(const vt_shapes* shapes, const vt_layer_weights* per_layer,
+                                     const void* embed, const vt_allocator* allocator,
+                                     vt_stream stream, vt_model** out) {
+    if (!out) return fail(VT_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    VT_TRY(vt_shapes_validate(shapes));
+    if (allocator && (!allocator->alloc || !allocator->free))
+        return fail(VT_ERR_INVALID_ARG, "allocator callbacks must not be NULL");
+    VT_CUDA(init_library());
+    cudaStream_t st = (cudaStream_t)stream;
+    vt_model* m = new vt_model();
+    m->s = *shapes;
+    if (allocator) {
+        m->alloc.a = *allocator;
+        m->alloc.custom = true;
+    }
+    const vt_shapes& s = m->s;
+    const size_t D = s.d_model, Q = (size_t)s.n_heads * s.d_head, KV = (size_t)s.n_kv_heads * s.d_head,
+                 F = s.d_ffn;
+    const size_t sizes[9] = {D * 2, Q * D * 2, KV * D * 2, KV * D * 2, D * Q * 2,
+                             D * 2, F * D * 2, F * D * 2, D * F * 2};
+    size_t total = 0;
+    for (size_t b : sizes) total += align256(b);
+    m->layer.resize(s.n_layers);
+    m->loaded.assign(s.n_layers, 0);
+    for (int l = 0; l < s.n_layers; ++l) {
+        uint8_t* base = static_cast<uint8_t*>(m->alloc.get(total));
+        if (!base) {
+            vt_model_destroy(m);
+            return fail(VT_ERR_ALLOC, "allocating %zu bytes for layer %d failed", total, l);
+        }
+        m->layer_base.push_back(base);
+        __half** slots[9] = {&m->layer[l].attn_norm, &m->layer[l].wq, &m->layer[l].wk,
+                             &m->layer[l].wv, &m->layer[l].wo, &m->layer[l].ffn_norm,
+                             &m->layer[l].w_gate, &m->layer[l].w_up, &m->layer[l].w_down};
+        size_t off = 0;
+        for (int t = 0; t < 9; ++t) {
+            *slots[t] = reinterpret_cast<__half*>(base + off);
+            off += align256(sizes[t]);
+        }
+    }
+    if (s.vocab > 0) {
+        m->embed = static_cast<__half*>(m->alloc.get((size_t)s.vocab * D * 2));
+        if (!m->embed) {
+            vt_model_destroy(m);
+            return fail(VT_ERR_ALLOC, "allocating the embedding table failed");
+        }
+    }
+    const size_t rope_bytes = (size_t)s.max_seq * (s.d_head / 2) * sizeof(float2);
+    m->rope = static_cast<float2*>(m->alloc.get(rope_bytes));
+    if (!m->rope) {
+        vt_model_destroy(m);
+        return fail(VT_ERR_ALLOC, "allocating the RoPE table failed");
+    }
+    cudaError_t e = launch_rope_table(m->rope, s.max_seq, s.d_head, (double)s.rope_theta, st);
+    if (e != cudaSuccess) {
+        vt_model_destroy(m);
+        return fail(VT_ERR_CUDA, "RoPE table launch failed: %s", cudaGetErrorString(e));
+    }
+    if (per_layer) {
+        for (int l = 0; l < s.n_layers; ++l) {
+            vt_status r = vt_model_load_layer(m, l, &per_layer[l], stream);
+            if (r != VT_OK) {
+                std::string keep = t_err;
+                vt_model_destroy(m);
+                t_err = keep;
+                return r;
+            }
+        }
+    }
+    if (embed && m->embed) {
+        vt_status r = vt_model_load_embedding(m, embed, stream);
+        if (r != VT_OK) {
+            std::string keep = t_err;
+            vt_model_destroy(m);
+            t_err = keep;
+            return r;
+        }
+    }
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        vt_model_destroy(m);
+        return fail(VT_ERR_CUDA, "model setup failed: %s", cudaGetErrorString(e));
+    }
+    *out = m;
+    return ok();
+}
+
+extern "C" vt_status vt_model_shapes(const vt_model* m, vt_shapes* out) {
+    if (!m || !out) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    *out = m->s;
+    return ok();
+}
+
+extern "C" vt_status vt_embed(const vt_model* m, const int32_t* ids, int32_t n, void* out,
+                              vt_stream stream) {
+    if (!m || (!ids && n > 0) || (!out && n > 0) || n < 0)
+        return fail(VT_ERR_INVALID_ARG, "bad vt_embed arguments");
+    if (!m->embed || !m->embed_loaded) return fail(VT_ERR_STATE, "no embedding table loaded");
+    VT_CUDA(launch_embed(m->embed, ids, n, m->s.d_model, m->s.vocab, static_cast<__half*>(out),
+                         (cudaStream_t)stream));
+    return ok();
+}
+
+// ================================================================== partition
+
+extern "C" void vt_partition_destroy(vt_partition* p) {
+    if (!p) return;
+    cudaDeviceSynchronize();
+    Allocator& A = p->m->alloc;
+    for (auto& s : p->attn) A.put(s.base);
+    for (auto& s : p->ffn) A.put(s.base);
+    for (void* q : p->owned) A.put(q);
+    delete p;
+}
+
+namespace {
+
+struct Bump {  // carves one allocation into 256-byte aligned pieces
+    uint8_t* base;
+    size_t off = 0;
+    template <typename T>
+    T* take(size_t count) {
+        T* r = reinterpret_cast<T*>(base + off);
+        off += align256(count * sizeof(T));
+        return r;
+    }
+};
+
+vt_status owned_alloc(vt_partition* p, size_t bytes, void** out) {
+    void* q = p->m->alloc.get(bytes);
+    if (!q) return fail(VT_ERR_ALLOC, "allocating %zu bytes failed", bytes);
+    p->owned.push_back(q);
+    *out = q;
+    return VT_OK;
+}
+
+}  // namespace
+
+extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range* heads,
+                                         const vt_range* cols, vt_stream stream,
+                                         vt_partition** out) {
+    if (!out || !m) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    *out = nullptr;
+    VT_TRY(vt_partition_validate(&m->s, n, heads, cols));
+    for (int l = 0; l < m->s.n_layers; ++l)
+        if (!m->loaded[l]) return fail(VT_ERR_STATE, "layer %d weights were never loaded", l);
+    cudaStream_t st = (cudaStream_t)stream;
+    const vt_shapes& s = m->s;
+    const int D = s.d_model, dh = s.d_head, H = s.n_heads, F = s.d_ffn;
+    const int g = s.n_heads / s.n_kv_heads;
+    vt_partition* p = new vt_partition();
+    p->m = m;
+    p->n_dev = n;
+    p->heads.assign(heads, heads + n);
+    p->cols.assign(cols, cols + n);
+    p->attn.resize((size_t)s.n_layers * n);
+    p->ffn.resize((size_t)s.n_layers * n);
+    Allocator& A = m->alloc;
+
+    auto bail = [&](vt_status r) {
+        std::string keep = t_err;
+        vt_partition_destroy(p);
+        t_err = keep;
+        return r;
+    };
+
+    // host staging of row-pointer tables for the gather kernel (per layer)
+    std::vector<const __half*> rows_host;
+    const __half** rows_dev = nullptr;
+    size_t rows_cap = (size_t)(H + 2 * s.n_kv_heads) * dh;
+    if ((size_t)2 * F > rows_cap) rows_cap = (size_t)2 * F;
+    rows_dev = static_cast<const __half**>(A.get(rows_cap * sizeof(void*)));
+    if (!rows_dev) return bail(fail(VT_ERR_ALLOC, "allocating the gather table failed"));
+
+    vt_status r = VT_OK;
+    for (int l = 0; l < s.n_layers && r == VT_OK; ++l) {
+        const LayerPtrs& L = m->layer[l];
+        for (int d = 0; d < n; ++d) {
+            // ---------------------------------------------------------- ATTN shard
+            AttnShard& as = p->attn[(size_t)l * n + d];
+            as.h0 = heads[d].begin;
+            as.h1 = heads[d].end;
+            as.kv0 = as.h0 / g;
+            as.kv1 = as.h1 / g;
+            const int hq = as.h1 - as.h0, hk = as.kv1 - as.kv0;
+            const int qkv_rows = (hq + 2 * hk) * dh;
+            if (hq > 0) {
+                const size_t bytes = align256((size_t)D * 2) + align256((size_t)qkv_rows * D * 2) +
+                                     align256((size_t)D * hq * dh * 2);
+                as.base = A.get(bytes);
+                if (!as.base) return bail(fail(VT_ERR_ALLOC, "shard allocation failed"));
+                Bump b{static_cast<uint8_t*>(as.base)};
+                as.norm = b.take<__half>(D);
+                as.wqkv = b.take<__half>((size_t)qkv_rows * D);
+                as.wo = b.take<__half>((size_t)D * hq * dh);
+                VT_CUDA(cudaMemcpyAsync(as.norm, L.attn_norm, (size_t)D * 2,
+                                        cudaMemcpyDeviceToDevice, st));
+                rows_host.clear();
+                for (int blk = 0; blk < hq + 2 * hk; ++blk) {
+                    const __half* src;
+                    int head;
+                    if (blk < hq) {
+                        src = L.wq;
+                        head = as.h0 + blk;
+                    } else if (blk < hq + hk) {
+                        src = L.wk;
+                        head = as.kv0 + blk - hq;
+                    } else {
+                        src = L.wv;
+                        head = as.kv0 + blk - hq - hk;
+                    }
+                    for (int i = 0; i < dh / 2; ++i) {
+                        rows_host.push_back(src + ((size_t)head * dh + i) * D);
+                        rows_host.push_back(src + ((size_t)head * dh + i + dh / 2) * D);
+                    }
+                }
+                VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*),
+                                        cudaMemcpyHostToDevice, st));
+                VT_CUDA(launch_gather_rows(rows_dev, as.wqkv, (int)rows_host.size(), D, D, st));
+                VT_CUDA(cudaStreamSynchronize(st));  // rows_host / rows_dev are reused
+                VT_CUDA(cudaMemcpy2DAsync(as.wo, (size_t)hq * dh * 2, L.wo + (size_t)as.h0 * dh,
+                                          (size_t)H * dh * 2, (size_t)hq * dh * 2, D,
+                                          cudaMemcpyDeviceToDevice, st));
+            }
+            // ---------------------------------------------------------- FFN shard
+            FfnShard& fs = p->ffn[(size_t)l * n + d];
+            fs.c0 = cols[d].begin;
+            fs.c1 = cols[d].end;
+            const int c = fs.c1 - fs.c0;
+            fs.ld = round_up8(c);
+            if (c > 0) {
+                const size_t bytes = align256((size_t)D * 2) + align256((size_t)2 * c * D * 2) +
+                                     align256((size_t)D * fs.ld * 2);
+                fs.base = A.get(bytes);
+                if (!fs.base) return bail(fail(VT_ERR_ALLOC, "shard allocation failed"));
+                Bump b{static_cast<uint8_t*>(fs.base)};
+                fs.norm = b.take<__half>(D);
+                fs.wgu = b.take<__half>((size_t)2 * c * D);
+                fs.wd = b.take<__half>((size_t)D * fs.ld);
+                VT_CUDA(cudaMemcpyAsync(fs.norm, L.ffn_norm, (size_t)D * 2,
+                                        cudaMemcpyDeviceToDevice, st));
+                rows_host.clear();
+                for (int j = 0; j < c; ++j) {
+                    rows_host.push_back(L.w_gate + (size_t)(fs.c0 + j) * D);
+                    rows_host.push_back(L.w_up + (size_t)(fs.c0 + j) * D);
+                }
+                VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*),
+                                        cudaMemcpyHostToDevice, st));
+                VT_CUDA(launch_gather_rows(rows_dev, fs.wgu, (int)rows_host.size(), D, D, st));
+                VT_CUDA(cudaStreamSynchronize(st));
+                VT_CUDA(cudaMemsetAsync(fs.wd, 0, (size_t)D * fs.ld * 2, st));
+                VT_CUDA(cudaMemcpy2DAsync(fs.wd, (size_t)fs.ld * 2, L.w_down + fs.c0, (size_t)F * 2,
+                                          (size_t)c * 2, D, cudaMemcpyDeviceToDevice, st));
+            }
+        }
+    }
+    A.put(rows_dev);
+
+    // ------------------------------------------------------------------ decode scratch
+    p->dec.resize(n);
+    for (int d = 0; d < n; ++d) {
+        const int hq = heads[d].end - heads[d].begin, hk = hq / g, c = cols[d].end - cols[d].begin;
+        DecodeScratch& ds = p->dec[d];
+        const int target = 2 * (g_num_sms > 0 ? g_num_sms : 148);
+        int ns = hk > 0 ? (target + hk - 1) / hk : 1;
+        const int ns_max = std::max(1, s.max_seq / 16);
+        ns = std::max(1, std::min(std::min(ns, ns_max), 1024));
+        ds.nsplit = ns;
+        const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2 +
+                             align256((size_t)std::max(hq, 1) * ns * 2 * 4) +
+                             align256((size_t)std::max(hq, 1) * ns * dh * 4) +
+                             align256((size_t)std::max(hk, 1) * 4) + align256((size_t)std::max(c, 1) * 4);
+        void* q;
+        if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
+        Bump b{static_cast<uint8_t*>(q)};
+        ds.q = b.take<float>((size_t)std::max(hq, 1) * dh);
+        ds.attn = b.take<float>((size_t)std::max(hq, 1) * dh);
+        ds.part_ml = b.take<float>((size_t)std::max(hq, 1) * ns * 2);
+        ds.part_o = b.take<float>((size_t)std::max(hq, 1) * ns * dh);
+        ds.tickets = b.take<int32_t>(std::max(hk, 1));
+        ds.u = b.take<float>(std::max(c, 1));
+        VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
+        p->max_hq = std::max(p->max_hq, hq);
+        p->max_ld = std::max(p->max_ld, round_up8(c));
+    }
+    // ------------------------------------------------------------------ stack + prefill scratch
+    {
+        const size_t R = kPrefillChunk;
+        const size_t bytes = align256(4) + align256((size_t)n * R * D * 4) + 2 * align256(R * D * 2) +
+                             align256(R * D * 2) + 2 * align256(R * std::max(p->max_hq, 1) * dh * 2) +
+                             align256(R * std::max(p->max_ld, 8) * 2);
+        void* q;
+        if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
+        Bump b{static_cast<uint8_t*>(q)};
+        p->status = b.take<uint32_t>(1);
+        p->partials = b.take<float>((size_t)n * R * D);
+        p->hbuf = b.take<__half>(R * D);
+        p->xbuf = b.take<__half>(R * D);
+        p->p_xhat = b.take<__half>(R * D);
+        p->p_q = b.take<__half>(R * std::max(p->max_hq, 1) * dh);
+        p->p_attn = b.take<__half>(R * std::max(p->max_hq, 1) * dh);
+        p->p_u = b.take<__half>(R * std::max(p->max_ld, 8));
+        VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
+    }
+    VT_CUDA(cudaStreamSynchronize(st));
+    *out = p;
+    return ok();
+}
+
+extern "C" int32_t vt_partition_devices(const vt_partition* p) { return p ? p->n_dev : 0; }
+
+static vt_status read_status(uint32_t* dev, uint32_t* flags, int32_t clear) {
+    if (!flags) return fail(VT_ERR_INVALID_ARG, "flags is NULL");
+    VT_CUDA(cudaDeviceSynchronize());
+    VT_CUDA(cudaMemcpy(flags, dev, 4, cudaMemcpyDeviceToHost));
+    if (clear) VT_CUDA(cudaMemset(dev, 0, 4));
+    return ok();
+}
+
+extern "C" vt_status vt_partition_status(vt_partition* p, uint32_t* flags, int32_t clear) {
+    if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
+    return read_status(p->status, flags, clear);
+}
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
+
+static vt_status check_shard(const vt_partition* p, vt_shard sh) {
+    if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
+    if (sh.layer < 0 || sh.layer >= p->m->s.n_layers || sh.device < 0 || sh.device >= p->n_dev ||
+        (sh.block != VT_BLOCK_ATTN && sh.block != VT_BLOCK_FFN))
+        return fail(VT_ERR_INVALID_ARG, "shard (layer %d, device %d, block %d) out of range",
+                    sh.layer, sh.device, sh.block);
+    return VT_OK;
+}
+
+extern "C" vt_status vt_shard_weight_layout(const vt_partition* p, vt_shard sh, int32_t which,
+                                            int64_t* rows, int64_t* stride) {
+    VT_TRY(check_shard(p, sh));
+    if (!rows || !stride) return fail(VT_ERR_INVALID_ARG, "NULL output");
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(sh.layer, sh.device);
+    const FfnShard& f = p->f(sh.layer, sh.device);
+    const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, c = f.c1 - f.c0;
+    switch (which) {
+        case 0: *rows = hq > 0; *stride = s.d_model; break;
+        case 1: *rows = (int64_t)(hq + 2 * hk) * s.d_head; *stride = s.d_model; break;
+        case 2: *rows = hq > 0 ? s.d_model : 0; *stride = (int64_t)hq * s.d_head; break;
+        case 3: *rows = c > 0; *stride = s.d_model; break;
+        case 4: *rows = 2 * (int64_t)c; *stride = s.d_model; break;
+        case 5: *rows = c > 0 ? s.d_model : 0; *stride = f.ld; break;
+        default: return fail(VT_ERR_INVALID_ARG, "unknown tensor %d", which);
+    }
+    return ok();
+}
+
+extern "C" vt_status vt_shard_weights_read(const vt_partition* p, vt_shard sh, int32_t which,
+                                           void* dst, size_t bytes, size_t* size_out) {
+    int64_t rows = 0, stride = 0;
+    VT_TRY(vt_shard_weight_layout(p, sh, which, &rows, &stride));
+    const AttnShard& a = p->a(sh.layer, sh.device);
+    const FfnShard& f = p->f(sh.layer, sh.device);
+    const __half* src = nullptr;
+    switch (which) {
+        case 0: src = a.norm; break;
+        case 1: src = a.wqkv; break;
+        case 2: src = a.wo; break;
+        case 3: src = f.norm; break;
+        case 4: src = f.wgu; break;
+        default: src = f.wd; break;
+    }
+    const size_t size = (size_t)rows * stride * 2;
+    if (size_out) *size_out = size;
+    const size_t nb = std::min(bytes, size);
+    if (nb > 0) {
+        if (!dst) return fail(VT_ERR_INVALID_ARG, "dst is NULL");
+        VT_CUDA(cudaDeviceSynchronize());
+        VT_CUDA(cudaMemcpy(dst, src, nb, cudaMemcpyDeviceToHost));
+    }
+    return ok();
+}
+
+// ================================================================== KV cache
+
+extern "C" void vt_kv_destroy(vt_kv* kv) {
+    if (!kv) return;
+    cudaDeviceSynchronize();
+    Allocator* A = kv->alloc();
+    for (void* b : kv->buf) A->put(b);
+    A->put(kv->len);
+    delete kv;
+}
+
+extern "C" vt_status vt_kv_create(const vt_partition* p, int32_t cap, vt_stream stream, vt_kv** out) {
+    if (!p || !out) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    *out = nullptr;
+    const vt_shapes& s = p->m->s;
+    if (cap < 1 || cap > s.max_seq)
+        return fail(VT_ERR_INVALID_ARG, "capacity %d must be in [1, max_seq = %d]", cap, s.max_seq);
+    cudaStream_t st = (cudaStream_t)stream;
+    vt_kv* kv = new vt_kv();
+    kv->p = p;
+    kv->cap = cap;
+    kv->buf.assign((size_t)s.n_layers * p->n_dev, nullptr);
+    Allocator* A = kv->alloc();
+    for (int l = 0; l < s.n_layers; ++l)
+        for (int d = 0; d < p->n_dev; ++d) {
+            const AttnShard& a = p->a(l, d);
+            const int hk = a.kv1 - a.kv0;
+            if (hk == 0) continue;
+            const size_t bytes = (size_t)2 * hk * cap * s.d_head * 2;
+            void* b = A->get(bytes);
+            if (!b) {
+                vt_kv_destroy(kv);
+                return fail(VT_ERR_ALLOC, "allocating the KV cache of layer %d device %d failed", l, d);
+            }
+            kv->buf[(size_t)l * p->n_dev + d] = b;
+            cudaError_t e = cudaMemsetAsync(b, 0, bytes, st);
+            if (e != cudaSuccess) {
+                vt_kv_destroy(kv);
+                return fail(VT_ERR_CUDA, "cudaMemsetAsync failed: %s", cudaGetErrorString(e));
+            }
+        }
+    const size_t meta = align256((size_t)s.n_layers * 4) + 256;
+    uint8_t* mb = static_cast<uint8_t*>(A->get(meta));
+    if (!mb) {
+        vt_kv_destroy(kv);
+        return fail(VT_ERR_ALLOC, "allocating KV lengths failed");
+    }
+    kv->len = reinterpret_cast<int32_t*>(mb);
+    kv->status = reinterpret_cast<uint32_t*>(mb + align256((size_t)s.n_layers * 4));
+    kv->h_len.assign(s.n_layers, 0);
+    cudaError_t e = cudaMemsetAsync(mb, 0, meta, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        vt_kv_destroy(kv);
+        return fail(VT_ERR_CUDA, "KV setup failed: %s", cudaGetErrorString(e));
+    }
+    *out = kv;
+    return ok();
+}
+
+extern "C" int32_t vt_kv_capacity(const vt_kv* kv) { return kv ? kv->cap : 0; }
+
+extern "C" vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_stream stream) {
+    if (!kv) return fail(VT_ERR_INVALID_ARG, "kv is NULL");
+    const int L = kv->p->m->s.n_layers;
+    if (layer < -1 || layer >= L) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
+    const int first = layer < 0 ? 0 : layer, count = layer < 0 ? L : 1;
+    for (int l = first; l < first + count; ++l)
+        if ((int64_t)kv->h_len[l] + n > kv->cap || (int64_t)kv->h_len[l] + n < 0)
+            return fail(VT_ERR_KV_CAPACITY, "advancing layer %d from %d by %d leaves [0, %d]", l,
+                        kv->h_len[l], n, kv->cap);
+    VT_CUDA(launch_kv_advance(kv->len, first, count, n, (cudaStream_t)stream));
+    for (int l = first; l < first + count; ++l) kv->h_len[l] += n;
+    return ok();
+}
+
+extern "C" vt_status vt_kv_set_length(vt_kv* kv, int32_t layer, int32_t len, vt_stream stream) {
+    if (!kv) return fail(VT_ERR_INVALID_ARG, "kv is NULL");
+    const int L = kv->p->m->s.n_layers;
+    if (layer < -1 || layer >= L) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
+    if (len < 0 || len > kv->cap) return fail(VT_ERR_KV_CAPACITY, "length %d outside [0, %d]", len, kv->cap);
+    const int first = layer < 0 ? 0 : layer, count = layer < 0 ? L : 1;
+    cudaStream_t st = (cudaStream_t)stream;
+    std::vector<int32_t> v(count, len);
+    VT_CUDA(cudaMemcpyAsync(kv->len + first, v.data(), count * 4, cudaMemcpyHostToDevice, st));
+    VT_CUDA(cudaStreamSynchronize(st));
+    for (int l = first; l < first + count; ++l) kv->h_len[l] = len;
+    return ok();
+}
+
+extern "C" vt_status vt_kv_length(vt_kv* kv, int32_t layer, vt_stream stream, int32_t* out) {
+    if (!kv || !out) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    if (layer < 0 || layer >= kv->p->m->s.n_layers)
+        return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
+    cudaStream_t st = (cudaStream_t)stream;
+    VT_CUDA(cudaMemcpyAsync(out, kv->len + layer, 4, cudaMemcpyDeviceToHost, st));
+    VT_CUDA(cudaStreamSynchronize(st));
+    kv->h_len[layer] = *out;
+    return ok();
+}
+
+extern "C" vt_status vt_kv_status(vt_kv* kv, uint32_t* flags, int32_t clear) {
+    if (!kv) return fail(VT_ERR_INVALID_ARG, "kv is NULL");
+    return read_status(kv->status, flags, clear);
+}
+
+static vt_status kv_copy(const vt_kv* kv, int32_t l, int32_t d, int32_t n_pos, void* kh,
+                         const void* kh_in, void* vh, const void* vh_in) {
+    if (!kv) return fail(VT_ERR_INVALID_ARG, "kv is NULL");
+    const vt_partition* p = kv->p;
+    if (l < 0 || l >= p->m->s.n_layers || d < 0 || d >= p->n_dev)
+        return fail(VT_ERR_INVALID_ARG, "(layer %d, device %d) out of range", l, d);
+    if (n_pos < 0 || n_pos > kv->cap) return fail(VT_ERR_KV_CAPACITY, "n_pos %d outside [0, %d]", n_pos, kv->cap);
+    const AttnShard& a = p->a(l, d);
+    const int hk = a.kv1 - a.kv0, dh = p->m->s.d_head;
+    if (hk == 0 || n_pos == 0) return ok();
+    VT_CUDA(cudaDeviceSynchronize());
+    const size_t row = (size_t)n_pos * dh * 2, pitch = (size_t)kv->cap * dh * 2;
+    if (kh_in) {
+        VT_CUDA(cudaMemcpy2D(kv->k(l, d), pitch, kh_in, row, row, hk, cudaMemcpyHostToDevice));
+        VT_CUDA(cudaMemcpy2D(kv->v(l, d), pitch, vh_in, row, row, hk, cudaMemcpyHostToDevice));
+    } else {
+        VT_CUDA(cudaMemcpy2D(kh, row, kv->k(l, d), pitch, row, hk, cudaMemcpyDeviceToHost));
+        VT_CUDA(cudaMemcpy2D(vh, row, kv->v(l, d), pitch, row, hk, cudaMemcpyDeviceToHost));
+    }
+    return ok();
+}
+
+extern "C" vt_status vt_kv_read(const vt_kv* kv, int32_t l, int32_t d, int32_t n_pos, void* kh,
+                                void* vh) {
+    if (!kh || !vh) return fail(VT_ERR_INVALID_ARG, "NULL host buffer");
+    return kv_copy(kv, l, d, n_pos, kh, nullptr, vh, nullptr);
+}
+
+extern "C" vt_status vt_kv_write_raw(vt_kv* kv, int32_t l, int32_t d, int32_t n_pos,
+                                     const void* kh, const void* vh) {
+    if (!kh || !vh) return fail(VT_ERR_INVALID_ARG, "NULL host buffer");
+    return kv_copy(kv, l, d, n_pos, nullptr, kh, nullptr, vh);
+}
+
+// ================================================================== shard compute
+
+static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* x, vt_kv* kv,
+                             float* out, cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(l, d);
+    const DecodeScratch& ds = p->dec[d];
+    const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, dh = s.d_head, D = s.d_model;
+    if (hq == 0) {
+        VT_CUDA(launch_fill_zero_f32(out, D, st));
+        return VT_OK;
+    }
+    GemvArgs g{};
+    g.w = a.wqkv;
+    g.row_stride = D;
+    g.rows = (hq + 2 * hk) * dh;
+    g.k = D;
+    g.x = x;
+    g.gain = a.norm;
+    g.eps = s.rms_eps;
+    g.out = ds.q;
+    g.kcache = kv->k(l, d);
+    g.vcache = kv->v(l, d);
+    g.cap = kv->cap;
+    g.len = kv->len + l;
+    g.rope = p->m->rope;
+    g.dh = dh;
+    g.hq = hq;
+    g.hk = hk;
+    g.status = kv->status;
+    VT_CUDA(launch_gemv(kEpiQkvRope, g, st));
+
+    AttnDecodeArgs t{};
+    t.q = ds.q;
+    t.kcache = kv->k(l, d);
+    t.vcache = kv->v(l, d);
+    t.len = kv->len + l;
+    t.cap = kv->cap;
+    t.hk = hk;
+    t.group = s.n_heads / s.n_kv_heads;
+    t.dh = dh;
+    t.nsplit = ds.nsplit;
+    t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    t.part_ml = ds.part_ml;
+    t.part_o = ds.part_o;
+    t.tickets = ds.tickets;
+    t.out = ds.attn;
+    t.status = kv->status;
+    VT_CUDA(launch_attn_decode(t, st));
+
+    GemvArgs o{};
+    o.w = a.wo;
+    o.row_stride = (int64_t)hq * dh;
+    o.rows = D;
+    o.k = hq * dh;
+    o.vin = ds.attn;
+    o.out = out;
+    o.status = kv->status;
+    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    return VT_OK;
+}
+
+static vt_status decode_ffn(const vt_partition* p, int l, int d, const __half* x, float* out,
+                            cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const FfnShard& f = p->f(l, d);
+    const DecodeScratch& ds = p->dec[d];
+    const int c = f.c1 - f.c0, D = s.d_model;
+    if (c == 0) {
+        VT_CUDA(launch_fill_zero_f32(out, D, st));
+        return VT_OK;
+    }
+    GemvArgs g{};
+    g.w = f.wgu;
+    g.row_stride = D;
+    g.rows = 2 * c;
+    g.k = D;
+    g.x = x;
+    g.gain = f.norm;
+    g.eps = s.rms_eps;
+    g.out = ds.u;
+    g.status = p->status;
+    VT_CUDA(launch_gemv(kEpiSwiglu, g, st));
+    GemvArgs o{};
+    o.w = f.wd;
+    o.row_stride = f.ld;
+    o.rows = D;
+    o.k = c;
+    o.vin = ds.u;
+    o.out = out;
+    o.status = p->status;
+    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    return VT_OK;
+}
+
+extern "C" vt_status vt_decode_step(const vt_partition* p, vt_shard sh, const void* x, vt_kv* kv,
+                                    float* out, vt_stream stream) {
+    VT_TRY(check_shard(p, sh));
+    if (!x || !out) return fail(VT_ERR_INVALID_ARG, "x and out_partial must not be NULL");
+    if (!aligned16(x)) return fail(VT_ERR_INVALID_ARG, "x must be 16-byte aligned");
+    cudaStream_t st = (cudaStream_t)stream;
+    if (sh.block == VT_BLOCK_ATTN) {
+        if (!kv || kv->p != p) return fail(VT_ERR_INVALID_ARG, "an ATTN shard needs this partition's KV cache");
+        if (kv->h_len[sh.layer] + 1 > kv->cap)
+            return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions", sh.layer,
+                        kv->h_len[sh.layer], kv->cap);
+        VT_TRY(decode_attn(p, sh.layer, sh.device, static_cast<const __half*>(x), kv, out, st));
+    } else {
+        VT_TRY(decode_ffn(p, sh.layer, sh.device, static_cast<const __half*>(x), out, st));
+    }
+    return ok();
+}
+
+extern "C" vt_status vt_combine(const float* const* partials, int32_t n, int32_t rows, int32_t d,
+                                const void* residual, void* out, vt_stream stream) {
+    if (!partials || !out || n < 1 || n > VT_MAX_DEVICES || rows < 0 || d < 0)
+        return fail(VT_ERR_INVALID_ARG, "bad vt_combine arguments");
+    CombineArgs c{};
+    for (int s = 0; s < n; ++s) {
+        if (!partials[s]) return fail(VT_ERR_INVALID_ARG, "partial %d is NULL", s);
+        c.parts[s] = partials[s];
+    }
+    c.n = n;
+    c.count = (int64_t)rows * d;
+    c.residual = static_cast<const __half*>(residual);
+    c.out = static_cast<__half*>(out);
+    VT_CUDA(launch_combine(c, (cudaStream_t)stream));
+    return ok();
+}
+
+// ------------------------------------------------------------------ prefill
+
+static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half* x, int n, vt_kv* kv,
+                               float* out, int row_offset, cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const int D = s.d_model;
+    std::string err;
+    if (sh.block == VT_BLOCK_ATTN) {
+        const AttnShard& a = p->a(sh.layer, sh.device);
+        const int hq = a.h1 - a.h0;
+        if (hq == 0) {
+            VT_CUDA(launch_fill_zero_f32(out, (int64_t)n * D, st));
+            return VT_OK;
+        }
+        PrefillAttnArgs t{};
+        t.n = n;
+        t.d = D;
+        t.dh = s.d_head;
+        t.hq = hq;
+        t.hk = a.kv1 - a.kv0;
+        t.eps = s.rms_eps;
+        t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)s.d_head));
+        t.x = x;
+        t.gain = a.norm;
+        t.wqkv = a.wqkv;
+        t.wo = a.wo;
+        t.kcache = kv->k(sh.layer, sh.device);
+        t.vcache = kv->v(sh.layer, sh.device);
+        t.cap = kv->cap;
+        t.len = kv->len + sh.layer;
+        t.row_offset = row_offset;
+        t.rope = p->m->rope;
+        t.xhat = p->p_xhat;
+        t.q = p->p_q;
+        t.attn = p->p_attn;
+        t.out = out;
+        t.status = kv->status;
+        vt_status r = prefill_attn_shard(t, st, &err);
+        if (r != VT_OK) return fail(r, "%s", err.c_str());
+    } else {
+        const FfnShard& f = p->f(sh.layer, sh.device);
+        const int c = f.c1 - f.c0;
+        if (c == 0) {
+            VT_CUDA(launch_fill_zero_f32(out, (int64_t)n * D, st));
+            return VT_OK;
+        }
+        PrefillFfnArgs t{};
+        t.n = n;
+        t.d = D;
+        t.c = c;
+        t.ld_down = f.ld;
+        t.eps = s.rms_eps;
+        t.x = x;
+        t.gain = f.norm;
+        t.wgu = f.wgu;
+        t.wd = f.wd;
+        t.xhat = p->p_xhat;
+        t.u = p->p_u;
+        t.out = out;
+        t.status = p->status;
+        vt_status r = prefill_ffn_shard(t, st, &err);
+        if (r != VT_OK) return fail(r, "%s", err.c_str());
+    }
+    return VT_OK;
+}
+
+extern "C" vt_status vt_prefill(const vt_partition* p, vt_shard sh, const void* x, int32_t n,
+                                vt_kv* kv, float* out, vt_stream stream) {
+    VT_TRY(check_shard(p, sh));
+    if (!x || !out || n < 1) return fail(VT_ERR_INVALID_ARG, "x, out_partial must be set and n >= 1");
+    if (!aligned16(x) || !aligned16(out)) return fail(VT_ERR_INVALID_ARG, "x and out_partial must be 16-byte aligned");
+    if (n > p->m->s.max_seq) return fail(VT_ERR_INVALID_ARG, "n %d exceeds max_seq", n);
+    cudaStream_t st = (cudaStream_t)stream;
+    if (sh.block == VT_BLOCK_ATTN) {
+        if (!kv || kv->p != p) return fail(VT_ERR_INVALID_ARG, "an ATTN shard needs this partition's KV cache");
+        if ((int64_t)kv->h_len[sh.layer] + n > kv->cap)
+            return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions; %d more do not fit",
+                        sh.layer, kv->h_len[sh.layer], kv->cap, n);
+    }
+    const int D = p->m->s.d_model;
+    for (int r0 = 0; r0 < n; r0 += kPrefillChunk) {
+        const int rows = std::min(kPrefillChunk, n - r0);
+        VT_TRY(prefill_shard(p, sh, static_cast<const __half*>(x) + (size_t)r0 * D, rows, kv,
+                             out + (size_t)r0 * D, r0, st));
+    }
+    return ok();
+}
+
+// ------------------------------------------------------------------ whole stack
+
+extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
+                                     vt_stream stream) {
+    if (!p || !kv || kv->p != p || !x_in || !x_out)
+        return fail(VT_ERR_INVALID_ARG, "bad vt_decode_token arguments");
+    if (!aligned16(x_in)) return fail(VT_ERR_INVALID_ARG, "x_in must be 16-byte aligned");
+    const vt_shapes& s = p->m->s;
+    for (int l = 0; l < s.n_layers; ++l)
+        if (kv->h_len[l] + 1 > kv->cap)
+            return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions", l, kv->h_len[l], kv->cap);
+    cudaStream_t st = (cudaStream_t)stream;
+    const int D = s.d_model, n = p->n_dev;
+    CombineArgs c{};
+    c.n = n;
+    c.count = D;
+    for (int d = 0; d < n; ++d) c.parts[d] = p->partials + (size_t)d * D;
+    const __half* cur = static_cast<const __half*>(x_in);
+    for (int l = 0; l < s.n_layers; ++l) {
+        for (int d = 0; d < n; ++d)
+            VT_TRY(decode_attn(p, l, d, cur, kv, p->partials + (size_t)d * D, st));
+        c.residual = cur;
+        c.out = p->hbuf;
+        VT_CUDA(launch_combine(c, st));
+        for (int d = 0; d < n; ++d)
+            VT_TRY(decode_ffn(p, l, d, p->hbuf, p->partials + (size_t)d * D, st));
+        __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) : p->xbuf;
+        c.residual = p->hbuf;
+        c.out = dst;
+        VT_CUDA(launch_combine(c, st));
+        cur = dst;
+    }
+    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, 1, st));
+    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
+    return ok();
+}
+
+extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const void* x_in, int32_t n,
+                                       void* x_out, vt_stream stream) {
+    if (!p || !kv || kv->p != p || !x_in || !x_out || n < 1)
+        return fail(VT_ERR_INVALID_ARG, "bad vt_prefill_tokens arguments");
+    if (!aligned16(x_in) || !aligned16(x_out))
+        return fail(VT_ERR_INVALID_ARG, "x_in and x_out must be 16-byte aligned");
+    const vt_shapes& s = p->m->s;
+    for (int l = 0; l < s.n_layers; ++l)
+        if ((int64_t)kv->h_len[l] + n > kv->cap)
+            return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions; %d more do not fit", l,
+                        kv->h_len[l], kv->cap, n);
+    cudaStream_t st = (cudaStream_t)stream;
+    const int D = s.d_model, nd = p->n_dev;
+    for (int r0 = 0; r0 < n; r0 += kPrefillChunk) {
+        const int rows = std::min(kPrefillChunk, n - r0);
+        CombineArgs c{};
+        c.n = nd;
+        c.count = (int64_t)rows * D;
+        for (int d = 0; d < nd; ++d) c.parts[d] = p->partials + (size_t)d * kPrefillChunk * D;
+        const __half* cur = static_cast<const __half*>(x_in) + (size_t)r0 * D;
+        for (int l = 0; l < s.n_layers; ++l) {
+            for (int d = 0; d < nd; ++d) {
+                vt_shard sh{l, d, VT_BLOCK_ATTN};
+                VT_TRY(prefill_shard(p, sh, cur, rows, kv, p->partials + (size_t)d * kPrefillChunk * D,
+                                     r0, st));
+            }
+            c.residual = cur;
+            c.out = p->hbuf;
+            VT_CUDA(launch_combine(c, st));
+            for (int d = 0; d < nd; ++d) {
+                vt_shard sh{l, d, VT_BLOCK_FFN};
+                VT_TRY(prefill_shard(p, sh, p->hbuf, rows, kv,
+                                     p->partials + (size_t)d * kPrefillChunk * D, r0, st));
+            }
+            __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) + (size_t)r0 * D : p->xbuf;
+            c.residual = p->hbuf;
+            c.out = dst;
+            VT_CUDA(launch_combine(c, st));
+            cur = dst;
+        }
+    }
+    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, n, st));
+    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += n;
+    return ok();
+}

@@ -1,0 +1,150 @@
+// Internal declarations shared by the library's translation units (host bookkeeping and kernel
+// launchers).  Not part of the C ABI.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/voltron.h"
+
+namespace vt {
+
+// ------------------------------------------------------------------ decode GEMV geometry
+constexpr int kGemvConsumerWarps = 8;
+constexpr int kGemvThreads = (kGemvConsumerWarps + 1) * 32;  // + one producer warp
+constexpr int kGemvStages = 4;
+constexpr int kGemvStageBytes = 16384;
+constexpr int kGemvMaxSlabRows = 128;  // rows per CTA (slot array bound)
+constexpr int kGemvMaxTileRows = 8;    // rows of one pipeline stage
+
+// ------------------------------------------------------------------ decode attention geometry
+constexpr int kAttnWarps = 4;
+constexpr int kAttnThreads = (kAttnWarps + 1) * 32;  // + one producer warp
+constexpr int kAttnTilePos = 32;                     // cached positions per pipeline stage
+constexpr int kAttnStages = 3;
+constexpr int kAttnMaxGroup = 8;  // query heads per KV head supported by the decode kernel
+
+enum GemvEpilogue : int {
+    kEpiPlain = 0,   // out[r] = y[r] (fp32)
+    kEpiQkvRope = 1, // rows in RoPE-pair order: rotate q/k, append k/v to the cache
+    kEpiSwiglu = 2,  // rows (gate, up) interleaved: u[j] = silu(gate) * up
+};
+
+struct GemvArgs {
+    const __half* w;     // [rows][row_stride]
+    int64_t row_stride;  // elements, multiple of 8
+    int rows;
+    int k;               // used columns (<= row_stride); columns beyond k are never multiplied
+    // input: either RMSNorm(x) with gain, or an fp32 vector
+    const __half* x;     // fp16 [k] (norm prologue) or nullptr
+    const __half* gain;  // fp16 [k]
+    float eps;
+    const float* vin;    // fp32 [k] when x == nullptr
+    // epilogue
+    float* out;          // plain: [rows]; swiglu: [rows/2]; qkv: q [h_s*dh]
+    // qkv epilogue
+    __half* kcache;      // [hk_s][cap][dh]
+    __half* vcache;
+    int cap;
+    const int32_t* len;  // device length of this layer (position of the new token)
+    const float2* rope;  // [max_seq][dh/2] (cos, sin)
+    int dh;
+    int hq;              // query heads of the shard
+    int hk;              // KV heads of the shard
+    uint32_t* status;
+};
+
+struct AttnDecodeArgs {
+    const float* q;        // [h_s][dh] rotated queries
+    const __half* kcache;  // [hk_s][cap][dh]
+    const __half* vcache;
+    const int32_t* len;
+    int cap;
+    int hk;                // KV heads of the shard
+    int group;             // query heads per KV head
+    int dh;
+    int nsplit;
+    float scale_log2;      // log2(e) / sqrt(dh)
+    float* part_ml;        // [h_s][nsplit][2]  (running max in log2 units, sum)
+    float* part_o;         // [h_s][nsplit][dh]
+    int32_t* tickets;      // [hk_s], zero between calls
+    float* out;            // [h_s][dh]
+    uint32_t* status;
+};
+
+struct CombineArgs {
+    const float* parts[VT_MAX_DEVICES];
+    int n;
+    int64_t count;
+    const __half* residual;
+    __half* out;
+};
+
+// ------------------------------------------------------------------ launchers (stream-ordered)
+extern bool g_use_pdl;  // programmatic dependent launch between the library's kernels
+extern int g_num_sms;
+
+cudaError_t launch_gemv(int epi, const GemvArgs& a, cudaStream_t st);
+int gemv_grid(int rows, int unit);
+size_t gemv_smem_bytes(int k);
+cudaError_t launch_attn_decode(const AttnDecodeArgs& a, cudaStream_t st);
+size_t attn_decode_smem_bytes(int dh);
+cudaError_t launch_combine(const CombineArgs& a, cudaStream_t st);
+cudaError_t launch_fill_zero_f32(float* p, int64_t n, cudaStream_t st);
+cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, cudaStream_t st);
+cudaError_t launch_rope_table(float2* tab, int max_seq, int dh, double theta, cudaStream_t st);
+cudaError_t launch_embed(const __half* table, const int32_t* ids, int n, int d, int vocab,
+                         __half* out, cudaStream_t st);
+cudaError_t launch_gather_rows(const __half* const* src_rows, __half* dst, int n_rows,
+                               int64_t row_len, int64_t dst_stride, cudaStream_t st);
+
+// One-time per-process setup of kernel attributes (dynamic shared-memory limits).
+cudaError_t init_decode_kernels();
+cudaError_t init_prefill_kernels();
+
+// ------------------------------------------------------------------ prefill path (prefill.cu)
+struct PrefillAttnArgs {
+    // shard geometry
+    int n;                  // rows (tokens) of this call
+    int d;                  // d_model
+    int dh, hq, hk;         // head dim, query heads and KV heads of the shard
+    float eps;
+    float scale_log2;       // log2(e) / sqrt(dh)
+    const __half* x;        // [n][d] layer input
+    const __half* gain;     // [d]
+    const __half* wqkv;     // [(hq + 2 hk) * dh][d], RoPE-pair row order
+    const __half* wo;       // [d][hq * dh]
+    __half* kcache;         // [hk][cap][dh]
+    __half* vcache;
+    int cap;
+    const int32_t* len;     // device length: rows sit at positions len + row_offset + i
+    int row_offset;         // rows already processed by earlier chunks of the same call
+    const float2* rope;     // [max_seq][dh/2]
+    // scratch
+    __half* xhat;           // [n][d]
+    __half* q;              // [n][hq][dh]
+    __half* attn;           // [n][hq * dh]
+    float* out;             // [n][d] partial
+    uint32_t* status;
+};
+struct PrefillFfnArgs {
+    int n, d, c;            // rows, d_model, shard columns
+    int ld_down;            // row stride of the down slice (c rounded up to 8)
+    float eps;
+    const __half* x;        // [n][d]
+    const __half* gain;
+    const __half* wgu;      // [2c][d], gate/up rows interleaved
+    const __half* wd;       // [d][ld_down]
+    __half* xhat;           // [n][d]
+    __half* u;              // [n][ld_down]
+    float* out;             // [n][d]
+    uint32_t* status;
+};
+vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err);
+vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err);
+
+}  // namespace vt

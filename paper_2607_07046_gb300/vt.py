@@ -1,0 +1,386 @@
+"""ctypes binding of libvoltron.so, with the C ABI's names (include/voltron.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA kernels.  Device
+buffers are torch CUDA tensors (their data_ptr() is passed through); the library allocates its own
+buffers through torch's caching allocator, so PyTorch owns device memory.  Streams default to
+torch's current stream.  There is no fallback: without the built library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+from typing import Iterable, List, Optional, Sequence, Tuple
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+LIB_PATH = _HERE / "libvoltron.so"
+
+VT_OK = 0
+VT_ERR_INVALID_ARG = 1
+VT_ERR_SHAPE = 2
+VT_ERR_PARTITION_OVERLAP = 3
+VT_ERR_PARTITION_GAP = 4
+VT_ERR_PARTITION_GQA = 5
+VT_ERR_PARTITION_RANGE = 6
+VT_ERR_KV_CAPACITY = 7
+VT_ERR_CUDA = 8
+VT_ERR_ALLOC = 9
+VT_ERR_STATE = 10
+VT_MAX_DEVICES = 16
+VT_DEV_KV_OVERFLOW = 1
+VT_DEV_WAIT_TIMEOUT = 2
+VT_BLOCK_ATTN = 0
+VT_BLOCK_FFN = 1
+
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+
+
+class VtError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"vt status {status}: {message}")
+        self.status = status
+
+
+class vt_shapes(ctypes.Structure):
+    _fields_ = [("n_layers", _I32), ("d_model", _I32), ("n_heads", _I32), ("n_kv_heads", _I32),
+                ("d_head", _I32), ("d_ffn", _I32), ("vocab", _I32), ("max_seq", _I32),
+                ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+
+
+class vt_range(ctypes.Structure):
+    _fields_ = [("begin", _I32), ("end", _I32)]
+
+
+ALLOC_FN = ctypes.CFUNCTYPE(_P, ctypes.c_size_t, _P)
+FREE_FN = ctypes.CFUNCTYPE(None, _P, _P)
+
+
+class vt_allocator(ctypes.Structure):
+    _fields_ = [("alloc", ALLOC_FN), ("free", FREE_FN), ("ctx", _P)]
+
+
+class vt_layer_weights(ctypes.Structure):
+    _fields_ = [(n, _P) for n in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate",
+                                  "w_up", "w_down")]
+
+
+class vt_shard(ctypes.Structure):
+    _fields_ = [("layer", _I32), ("device", _I32), ("block", _I32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library; raises if it has not been built (no CPU fallback exists)."""
+    global _lib
+    if _lib is None:
+        if not LIB_PATH.exists():
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "paper_2607_07046_gb300.build.build()")
+        L = ctypes.CDLL(str(LIB_PATH))
+        S = vt_status_t = _I32
+        sig = {
+            "vt_last_error": (ctypes.c_char_p, []),
+            "vt_version": (ctypes.c_char_p, []),
+            "vt_shapes_validate": (S, [ctypes.POINTER(vt_shapes)]),
+            "vt_partition_validate": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(vt_range),
+                                          ctypes.POINTER(vt_range)]),
+            "vt_model_create": (S, [ctypes.POINTER(vt_shapes), ctypes.POINTER(vt_layer_weights), _P,
+                                    ctypes.POINTER(vt_allocator), _P, ctypes.POINTER(_P)]),
+            "vt_model_load_layer": (S, [_P, _I32, ctypes.POINTER(vt_layer_weights), _P]),
+            "vt_model_load_embedding": (S, [_P, _P, _P]),
+            "vt_model_shapes": (S, [_P, ctypes.POINTER(vt_shapes)]),
+            "vt_model_destroy": (None, [_P]),
+            "vt_embed": (S, [_P, _P, _I32, _P, _P]),
+            "vt_partition_create": (S, [_P, _I32, ctypes.POINTER(vt_range), ctypes.POINTER(vt_range),
+                                        _P, ctypes.POINTER(_P)]),
+            "vt_partition_devices": (_I32, [_P]),
+            "vt_partition_status": (S, [_P, ctypes.POINTER(ctypes.c_uint32), _I32]),
+            "vt_partition_destroy": (None, [_P]),
+            "vt_shard_weights_read": (S, [_P, vt_shard, _I32, _P, ctypes.c_size_t,
+                                          ctypes.POINTER(ctypes.c_size_t)]),
+            "vt_shard_weight_layout": (S, [_P, vt_shard, _I32, ctypes.POINTER(ctypes.c_int64),
+                                           ctypes.POINTER(ctypes.c_int64)]),
+            "vt_kv_create": (S, [_P, _I32, _P, ctypes.POINTER(_P)]),
+            "vt_kv_destroy": (None, [_P]),
+            "vt_kv_capacity": (_I32, [_P]),
+            "vt_kv_advance": (S, [_P, _I32, _I32, _P]),
+            "vt_kv_set_length": (S, [_P, _I32, _I32, _P]),
+            "vt_kv_length": (S, [_P, _I32, _P, ctypes.POINTER(_I32)]),
+            "vt_kv_status": (S, [_P, ctypes.POINTER(ctypes.c_uint32), _I32]),
+            "vt_kv_read": (S, [_P, _I32, _I32, _I32, _P, _P]),
+            "vt_kv_write_raw": (S, [_P, _I32, _I32, _I32, _P, _P]),
+            "vt_decode_step": (S, [_P, vt_shard, _P, _P, _P, _P]),
+            "vt_prefill": (S, [_P, vt_shard, _P, _I32, _P, _P, _P]),
+            "vt_combine": (S, [ctypes.POINTER(_P), _I32, _I32, _I32, _P, _P, _P]),
+            "vt_decode_token": (S, [_P, _P, _P, _P, _P]),
+            "vt_prefill_tokens": (S, [_P, _P, _P, _I32, _P, _P]),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def vt_last_error() -> str:
+    return lib().vt_last_error().decode()
+
+
+def vt_version() -> str:
+    return lib().vt_version().decode()
+
+
+def _check(status: int) -> None:
+    if status != VT_OK:
+        raise VtError(status, vt_last_error())
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if hasattr(stream, "cuda_stream"):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _ptr(t, dtype=None) -> int:
+    """data_ptr of a contiguous CUDA tensor (checked), or 0 for None."""
+    if t is None:
+        return 0
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch tensor")
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("expected a contiguous CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"expected {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def make_shapes(n_layers, d_model, n_heads, n_kv_heads, d_head, d_ffn, vocab, max_seq,
+                rms_eps=1e-5, rope_theta=1e4) -> vt_shapes:
+    return vt_shapes(n_layers, d_model, n_heads, n_kv_heads, d_head, d_ffn, vocab, max_seq,
+                     rms_eps, rope_theta)
+
+
+def _ranges(rs: Sequence[Tuple[int, int]]):
+    arr = (vt_range * max(1, len(rs)))(*[vt_range(a, b) for a, b in rs])
+    return arr
+
+
+# ------------------------------------------------------------------ allocator (torch-backed)
+
+def _torch_alloc(nbytes, ctx):
+    import torch
+    try:
+        return torch.cuda.caching_allocator_alloc(int(nbytes), torch.cuda.current_device())
+    except Exception:  # out of memory: the library reports VT_ERR_ALLOC
+        return None
+
+
+def _torch_free(ptr, ctx):
+    import torch
+    torch.cuda.caching_allocator_delete(ptr)
+
+
+_TORCH_ALLOCATOR = vt_allocator(ALLOC_FN(_torch_alloc), FREE_FN(_torch_free), None)
+
+
+# ------------------------------------------------------------------ validation (host only)
+
+def vt_shapes_validate(shapes: vt_shapes) -> int:
+    return int(lib().vt_shapes_validate(ctypes.byref(shapes)))
+
+
+def vt_partition_validate(shapes: vt_shapes, head_ranges, ffn_col_ranges) -> int:
+    n = len(head_ranges)
+    if len(ffn_col_ranges) != n:
+        raise ValueError("one head range and one FFN range per device")
+    return int(lib().vt_partition_validate(ctypes.byref(shapes), n, _ranges(head_ranges),
+                                           _ranges(ffn_col_ranges)))
+
+
+# ------------------------------------------------------------------ model
+
+_WEIGHT_NAMES = ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down")
+
+
+def _layer_struct(w) -> Tuple[vt_layer_weights, list]:
+    keep = [np.ascontiguousarray(w[n], dtype=np.float16) for n in _WEIGHT_NAMES]
+    return vt_layer_weights(*[k.ctypes.data for k in keep]), keep
+
+
+def vt_model_create(shapes: vt_shapes, per_layer=None, embed: Optional[np.ndarray] = None,
+                    stream=None, allocator: str = "torch") -> int:
+    """per_layer: list of dicts of host fp16 arrays (nn.Linear layout), or None."""
+    keep = []
+    arr = None
+    if per_layer is not None:
+        structs = []
+        for w in per_layer:
+            s, k = _layer_struct(w)
+            structs.append(s)
+            keep.append(k)
+        arr = (vt_layer_weights * len(structs))(*structs)
+    emb = None if embed is None else np.ascontiguousarray(embed, dtype=np.float16)
+    out = _P()
+    alloc = ctypes.byref(_TORCH_ALLOCATOR) if allocator == "torch" else None
+    _check(lib().vt_model_create(ctypes.byref(shapes), arr, emb.ctypes.data if emb is not None else None,
+                                 alloc, _stream(stream), ctypes.byref(out)))
+    return out.value
+
+
+def vt_model_load_layer(model: int, layer: int, weights, stream=None) -> None:
+    s, keep = _layer_struct(weights)
+    _check(lib().vt_model_load_layer(model, layer, ctypes.byref(s), _stream(stream)))
+
+
+def vt_model_load_embedding(model: int, embed: np.ndarray, stream=None) -> None:
+    e = np.ascontiguousarray(embed, dtype=np.float16)
+    _check(lib().vt_model_load_embedding(model, e.ctypes.data, _stream(stream)))
+
+
+def vt_model_destroy(model: int) -> None:
+    if model:
+        lib().vt_model_destroy(model)
+
+
+def vt_embed(model: int, ids, out, stream=None) -> None:
+    import torch
+    _check(lib().vt_embed(model, _ptr(ids, torch.int32), ids.numel(), _ptr(out, torch.float16),
+                          _stream(stream)))
+
+
+# ------------------------------------------------------------------ partition
+
+def vt_partition_create(model: int, head_ranges, ffn_col_ranges, stream=None) -> int:
+    n = len(head_ranges)
+    out = _P()
+    _check(lib().vt_partition_create(model, n, _ranges(head_ranges), _ranges(ffn_col_ranges),
+                                     _stream(stream), ctypes.byref(out)))
+    return out.value
+
+
+def vt_partition_devices(part: int) -> int:
+    return int(lib().vt_partition_devices(part))
+
+
+def vt_partition_status(part: int, clear: bool = False) -> int:
+    f = ctypes.c_uint32()
+    _check(lib().vt_partition_status(part, ctypes.byref(f), int(clear)))
+    return int(f.value)
+
+
+def vt_partition_destroy(part: int) -> None:
+    if part:
+        lib().vt_partition_destroy(part)
+
+
+def vt_shard_weight_layout(part: int, shard: Tuple[int, int, int], which: int) -> Tuple[int, int]:
+    rows, stride = ctypes.c_int64(), ctypes.c_int64()
+    _check(lib().vt_shard_weight_layout(part, vt_shard(*shard), which, ctypes.byref(rows),
+                                        ctypes.byref(stride)))
+    return int(rows.value), int(stride.value)
+
+
+def vt_shard_weights_read(part: int, shard: Tuple[int, int, int], which: int) -> np.ndarray:
+    rows, stride = vt_shard_weight_layout(part, shard, which)
+    out = np.empty((rows, stride), np.float16)
+    size = ctypes.c_size_t()
+    _check(lib().vt_shard_weights_read(part, vt_shard(*shard), which, out.ctypes.data, out.nbytes,
+                                       ctypes.byref(size)))
+    assert size.value == out.nbytes
+    return out
+
+
+# ------------------------------------------------------------------ KV cache
+
+def vt_kv_create(part: int, capacity: int, stream=None) -> int:
+    out = _P()
+    _check(lib().vt_kv_create(part, capacity, _stream(stream), ctypes.byref(out)))
+    return out.value
+
+
+def vt_kv_destroy(kv: int) -> None:
+    if kv:
+        lib().vt_kv_destroy(kv)
+
+
+def vt_kv_capacity(kv: int) -> int:
+    return int(lib().vt_kv_capacity(kv))
+
+
+def vt_kv_advance(kv: int, layer: int, n: int, stream=None) -> None:
+    _check(lib().vt_kv_advance(kv, layer, n, _stream(stream)))
+
+
+def vt_kv_set_length(kv: int, layer: int, length: int, stream=None) -> None:
+    _check(lib().vt_kv_set_length(kv, layer, length, _stream(stream)))
+
+
+def vt_kv_length(kv: int, layer: int, stream=None) -> int:
+    v = _I32()
+    _check(lib().vt_kv_length(kv, layer, _stream(stream), ctypes.byref(v)))
+    return int(v.value)
+
+
+def vt_kv_status(kv: int, clear: bool = False) -> int:
+    f = ctypes.c_uint32()
+    _check(lib().vt_kv_status(kv, ctypes.byref(f), int(clear)))
+    return int(f.value)
+
+
+def vt_kv_read(kv: int, layer: int, device: int, n_pos: int, hk: int, d_head: int):
+    k = np.empty((hk, n_pos, d_head), np.float16)
+    v = np.empty_like(k)
+    _check(lib().vt_kv_read(kv, layer, device, n_pos, k.ctypes.data, v.ctypes.data))
+    return k, v
+
+
+def vt_kv_write_raw(kv: int, layer: int, device: int, k: np.ndarray, v: np.ndarray) -> None:
+    k = np.ascontiguousarray(k, dtype=np.float16)
+    v = np.ascontiguousarray(v, dtype=np.float16)
+    assert k.shape == v.shape and k.ndim == 3
+    _check(lib().vt_kv_write_raw(kv, layer, device, k.shape[1], k.ctypes.data, v.ctypes.data))
+
+
+# ------------------------------------------------------------------ shard compute
+
+def vt_decode_step(part: int, shard: Tuple[int, int, int], x, kv: Optional[int], out_partial,
+                   stream=None) -> None:
+    import torch
+    _check(lib().vt_decode_step(part, vt_shard(*shard), _ptr(x, torch.float16), kv or None,
+                                _ptr(out_partial, torch.float32), _stream(stream)))
+
+
+def vt_prefill(part: int, shard: Tuple[int, int, int], x, n: int, kv: Optional[int], out_partial,
+               stream=None) -> None:
+    import torch
+    _check(lib().vt_prefill(part, vt_shard(*shard), _ptr(x, torch.float16), n, kv or None,
+                            _ptr(out_partial, torch.float32), _stream(stream)))
+
+
+def vt_combine(partials: Sequence, residual, out, rows: int, d: int, stream=None) -> None:
+    import torch
+    arr = (_P * len(partials))(*[_ptr(p, torch.float32) for p in partials])
+    _check(lib().vt_combine(arr, len(partials), rows, d,
+                            _ptr(residual, torch.float16) if residual is not None else None,
+                            _ptr(out, torch.float16), _stream(stream)))
+
+
+def vt_decode_token(part: int, kv: int, x_in, x_out, stream=None) -> None:
+    import torch
+    _check(lib().vt_decode_token(part, kv, _ptr(x_in, torch.float16), _ptr(x_out, torch.float16),
+                                 _stream(stream)))
+
+
+def vt_prefill_tokens(part: int, kv: int, x_in, n: int, x_out, stream=None) -> None:
+    import torch
+    _check(lib().vt_prefill_tokens(part, kv, _ptr(x_in, torch.float16), n,
+                                   _ptr(x_out, torch.float16), _stream(stream)))

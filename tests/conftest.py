@@ -26,3 +26,12 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def vtlib():
+    """The built CUDA library (compiled here with nvcc if missing or stale)."""
+    from paper_2607_07046_gb300 import build as vt_build
+    from paper_2607_07046_gb300 import vt
+    vt_build.build()
+    return vt
