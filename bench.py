@@ -162,6 +162,9 @@ def run_decode(args, rank, world):
 
     vt_build.build()
     wl = synthetic.WORKLOADS[2]
+    if args.layers:
+        import dataclasses
+        wl = dataclasses.replace(wl, n_layers=args.layers)
     torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
     sched = wl.decode_steps  # 128-step KV schedule 1024 -> 1151
     cap = wl.kv_len + sched + 8
@@ -385,6 +388,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="small case for profiling: only the first N layers of the stack")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world = int(os.environ.get("WORLD_SIZE", "1"))

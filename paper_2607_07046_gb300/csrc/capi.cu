@@ -211,7 +211,8 @@ extern "C" vt_status vt_shapes_validate(const vt_shapes* s) {
     if (s->d_head != 64 && s->d_head != 128) return fail(VT_ERR_SHAPE, "d_head must be 64 or 128");
     if ((int64_t)s->n_heads * s->d_head > 16384)
         return fail(VT_ERR_SHAPE, "n_heads * d_head must be <= 16384");
-    if (s->d_ffn < 1 || s->d_ffn > 32768) return fail(VT_ERR_SHAPE, "d_ffn must be in [1, 32768]");
+    if (s->d_ffn < 1 || s->d_ffn > kGemvMaxK)
+        return fail(VT_ERR_SHAPE, "d_ffn must be in [1, %d]", kGemvMaxK);
     if (s->vocab < 0) return fail(VT_ERR_SHAPE, "vocab must be >= 0");
     if (s->max_seq < 1 || s->max_seq > (1 << 20))
         return fail(VT_ERR_SHAPE, "max_seq must be in [1, 2^20]");
@@ -571,7 +572,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         const int target = 2 * (g_num_sms > 0 ? g_num_sms : 148);
         int ns = hk > 0 ? (target + hk - 1) / hk : 1;
         const int ns_max = std::max(1, s.max_seq / 16);
-        ns = std::max(1, std::min(std::min(ns, ns_max), 1024));
+        ns = std::max(1, std::min(std::min(ns, ns_max), kAttnMaxSplit));
         ds.nsplit = ns;
         const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2 +
                              align256((size_t)std::max(hq, 1) * ns * 2 * 4) +
@@ -828,8 +829,10 @@ extern "C" vt_status vt_kv_write_raw(vt_kv* kv, int32_t l, int32_t d, int32_t n_
 
 // ================================================================== shard compute
 
+// indep: the caller guarantees that `x` was written at least two kernel launches before this
+// shard's first kernel, so that kernel may read it before griddepcontrol.wait (see k_gemv).
 static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* x, vt_kv* kv,
-                             float* out, cudaStream_t st) {
+                             float* out, cudaStream_t st, int indep = 0) {
     const vt_shapes& s = p->m->s;
     const AttnShard& a = p->a(l, d);
     const DecodeScratch& ds = p->dec[d];
@@ -856,6 +859,7 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
     g.hq = hq;
     g.hk = hk;
     g.status = kv->status;
+    g.indep = indep;
     VT_CUDA(launch_gemv(kEpiQkvRope, g, st));
 
     AttnDecodeArgs t{};
@@ -889,7 +893,7 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
 }
 
 static vt_status decode_ffn(const vt_partition* p, int l, int d, const __half* x, float* out,
-                            cudaStream_t st) {
+                            cudaStream_t st, int indep = 0) {
     const vt_shapes& s = p->m->s;
     const FfnShard& f = p->f(l, d);
     const DecodeScratch& ds = p->dec[d];
@@ -908,6 +912,7 @@ static vt_status decode_ffn(const vt_partition* p, int l, int d, const __half* x
     g.eps = s.rms_eps;
     g.out = ds.u;
     g.status = p->status;
+    g.indep = indep;
     VT_CUDA(launch_gemv(kEpiSwiglu, g, st));
     GemvArgs o{};
     o.w = f.wd;
@@ -1063,13 +1068,14 @@ extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const voi
     for (int d = 0; d < n; ++d) c.parts[d] = p->partials + (size_t)d * D;
     const __half* cur = static_cast<const __half*>(x_in);
     for (int l = 0; l < s.n_layers; ++l) {
+        // Shard d >= 1 reads the layer input written by the combine several launches earlier.
         for (int d = 0; d < n; ++d)
-            VT_TRY(decode_attn(p, l, d, cur, kv, p->partials + (size_t)d * D, st));
+            VT_TRY(decode_attn(p, l, d, cur, kv, p->partials + (size_t)d * D, st, d > 0));
         c.residual = cur;
         c.out = p->hbuf;
         VT_CUDA(launch_combine(c, st));
         for (int d = 0; d < n; ++d)
-            VT_TRY(decode_ffn(p, l, d, p->hbuf, p->partials + (size_t)d * D, st));
+            VT_TRY(decode_ffn(p, l, d, p->hbuf, p->partials + (size_t)d * D, st, d > 0));
         __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) : p->xbuf;
         c.residual = p->hbuf;
         c.out = dst;

@@ -11,13 +11,7 @@
 //                 and the last CTA of the head merges the slices with log-sum-exp weights.
 //   k_combine     the aggregation on the main device: residual + sum of partials, in shard order.
 //
-// The GEMV is HBM-bound (one fp16 weight read per two flops).  Its data path: one producer thread
-// streams the CTA's contiguous slab of weight rows into a 4-stage shared-memory ring with bulk
-// asynchronous copies (cp.async.bulk, tracked by mbarriers), so each SM keeps up to 64 KB of
-// loads in flight with a single thread; eight consumer warps each own a fixed column slice of
-// every row, so the per-row reduction (lane partials -> warp shuffle -> slot per warp -> fixed
-// order sum) is deterministic.  The producer starts before griddepcontrol.wait: weights are
-// constant, so a kernel streams its first 64 KB while the previous kernel is still finishing.
+// The GEMV is HBM-bound (one fp16 weight read per two flops); its design notes are at k_gemv.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -54,31 +48,82 @@ __device__ __forceinline__ void consumer_bar(int id, int nthreads) {
 }
 
 // ============================================================== GEMV
+//
+// Geometry.  A CTA of 8 warps owns a contiguous slab of rows (pairs of rows for the paired
+// epilogues).  The row length k is cut into 16-byte chunks; each lane owns CPL chunks of a row
+// (chunk (slice * CPL + q) * 32 + lane), WPR = ceil(chunks / (32 CPL)) warps cover one row, and
+// the 8 warps form RG = 8 / WPR row groups that walk the slab's rows in lockstep.  A lane's input
+// values (x^ or v) are therefore fixed for the whole slab and stay in registers.
+//
+// Pipeline.  Weights move with 16-byte LDG.128 loads straight into registers, two batches of R
+// rows (R * CPL chunks per lane) in flight.  Both batches are issued before griddepcontrol.wait:
+// they do not depend on the previous kernel, so a kernel streams its first 64 KB per SM while
+// the previous kernel finishes.  After a batch is consumed, its R row partials per lane are
+// reduced across the warp with a multi-row butterfly (R rows in 9 shuffles for R = 8 rather than
+// 5 per row), and each (row, slice) total goes to a shared-memory slot; the epilogue sums the
+// WPR slots of a row in slice order, so results are deterministic.
 
 static __host__ __device__ __forceinline__ int round_up8(int k) { return (k + 7) & ~7; }
 
-struct GemvTiling {
-    int kpad;   // columns rounded up to 16 bytes
-    int cb;     // column-block width (elements)
-    int ncb;    // column blocks per row
-    int tr;     // rows per tile
-};
-
-static __host__ __device__ __forceinline__ GemvTiling gemv_tiling(int k) {
-    GemvTiling t;
-    t.kpad = round_up8(k);
-    const int cbmax = kGemvStageBytes / 2;
-    t.cb = t.kpad < cbmax ? t.kpad : cbmax;
-    t.ncb = (t.kpad + t.cb - 1) / t.cb;
-    int tr = kGemvStageBytes / (t.cb * 2);
-    t.tr = tr < 1 ? 1 : (tr > kGemvMaxTileRows ? kGemvMaxTileRows : tr);
-    return t;
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
 }
 
-size_t gemv_smem_bytes(int k) {
-    const GemvTiling t = gemv_tiling(k);
-    return (size_t)kGemvStages * kGemvStageBytes + (size_t)t.kpad * 4 +
-           (size_t)kGemvMaxSlabRows * kGemvConsumerWarps * 4 + 64 * 4 + 2 * kGemvStages * 8 + 128;
+// R row partials per lane -> lane l with l % (32 / R) == 0 returns the warp total of row
+// l / (32 / R).  Each level halves the values a lane carries: lanes whose bit `o` is set keep the
+// upper half and send the lower half to their partner, and vice versa.
+template <int R>
+__device__ __forceinline__ float multi_row_sum(float (&v)[8], int lane) {
+    if constexpr (R == 8) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const bool hi = lane & 16;
+            const float send = hi ? v[i] : v[i + 4];
+            v[i] = (hi ? v[i + 4] : v[i]) + __shfl_xor_sync(0xffffffffu, send, 16);
+        }
+    }
+    if constexpr (R >= 4) {
+        constexpr int o = R == 8 ? 8 : 16;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const bool hi = lane & o;
+            const float send = hi ? v[i] : v[i + 2];
+            v[i] = (hi ? v[i + 2] : v[i]) + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    if constexpr (R >= 2) {
+        constexpr int o = R == 8 ? 4 : (R == 4 ? 8 : 16);
+        const bool hi = lane & o;
+        const float send = hi ? v[0] : v[1];
+        v[0] = (hi ? v[1] : v[0]) + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+    constexpr int first = R == 8 ? 2 : (R == 4 ? 4 : (R == 2 ? 8 : 16));
+#pragma unroll
+    for (int o = first; o >= 1; o >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    return v[0];
+}
+
+// Chunks per lane for a row of `k` columns: the choice with the best use of the 8 warps' lanes.
+int gemv_cpl(int k) {
+    const int nch = round_up8(k) / 8;
+    static const int cand[] = {1, 2, 3, 4, 8};
+    int best = 8;
+    double bs = -1.0;
+    for (int c : cand) {
+        const int wpr = (nch + 32 * c - 1) / (32 * c);
+        if (wpr > kGemvWarps) continue;
+        const int rg = kGemvWarps / wpr;
+        const double score = (double)(rg * wpr) / kGemvWarps * (double)nch / (double)(wpr * 32 * c);
+        if (score > bs + 1e-9) {
+            bs = score;
+            best = c;
+        }
+    }
+    return best;
 }
 
 int gemv_grid(int rows, int unit) {
@@ -92,168 +137,130 @@ int gemv_grid(int rows, int unit) {
     return g;
 }
 
-template <int EPI>
-__global__ void __launch_bounds__(kGemvThreads, 1) k_gemv(const __grid_constant__ GemvArgs a) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    const GemvTiling tl = gemv_tiling(a.k);
-    uint8_t* ring = smem;
-    float* xs = reinterpret_cast<float*>(smem + kGemvStages * kGemvStageBytes);
-    float* slots = xs + tl.kpad;
-    float* red = slots + kGemvMaxSlabRows * kGemvConsumerWarps;
-    uint64_t* full = reinterpret_cast<uint64_t*>(red + 64);
-    uint64_t* empty = full + kGemvStages;
-    __shared__ int s_abort;
-
+template <int EPI, int CPL, int R>
+__global__ void __launch_bounds__(kGemvThreads, (CPL <= 4 ? 2 : 1))
+    k_gemv(const __grid_constant__ GemvArgs a) {
+    constexpr int NB = R * CPL;  // chunks per lane per batch
+    __shared__ float slots[kGemvMaxSlabRows * kGemvWarps];
+    __shared__ float red[kGemvWarps + 1];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     constexpr int unit = (EPI == kEpiPlain) ? 1 : 2;
     const int units = a.rows / unit;
     const int r0 = (int)(((int64_t)blockIdx.x * units) / gridDim.x) * unit;
     const int r1 = (int)(((int64_t)(blockIdx.x + 1) * units) / gridDim.x) * unit;
     const int nrows = r1 - r0;
-    const int nrb = (nrows + tl.tr - 1) / tl.tr;
-    const int ntiles = nrb * tl.ncb;
+    const int nch = round_up8(a.k) >> 3;
+    const int wpr = (nch + 32 * CPL - 1) / (32 * CPL);
+    const int rg = kGemvWarps / wpr;
+    const int slice = warp % wpr, grp = warp / wpr;
+    const bool active = grp < rg;
+    const int n_my = active ? max(0, (nrows - grp + rg - 1) / rg) : 0;
+    const __half* wbase = a.w + (int64_t)(r0 + grp) * a.row_stride;
+    const int64_t rstep = (int64_t)rg * a.row_stride;
 
-    if (tid == 0) {
-        for (int s = 0; s < kGemvStages; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], kGemvConsumerWarps);
-        }
-        s_abort = 0;
-        fence_mbar_init();
-    }
-    __syncthreads();
-
-    if (warp == kGemvConsumerWarps) {
-        // ---------------------------------------------------------- producer (one thread)
-        if (lane == 0) {
-            int last_issued[kGemvStages];
-            for (int s = 0; s < kGemvStages; ++s) last_issued[s] = -1;
-            for (int t = 0; t < ntiles; ++t) {
-                const int s = t % kGemvStages;
-                if (t >= kGemvStages) {
-                    if (!mbar_wait(&empty[s], ((t / kGemvStages) - 1) & 1)) {
-                        s_abort = 1;
-                        set_status(a.status, VT_DEV_WAIT_TIMEOUT);
-                        break;
-                    }
-                }
-                if (*(volatile int*)&s_abort) break;
-                const int rb = t / tl.ncb, cbi = t - rb * tl.ncb;
-                const int rows_t = min(tl.tr, nrows - rb * tl.tr);
-                const int width = min(tl.cb, tl.kpad - cbi * tl.cb);
-                const uint32_t bytes = (uint32_t)rows_t * width * 2;
-                mbar_arrive_expect_tx(&full[s], bytes);
-                uint8_t* dst = ring + s * kGemvStageBytes;
-                const __half* src = a.w + (int64_t)(r0 + rb * tl.tr) * a.row_stride + cbi * tl.cb;
-                for (int i = 0; i < rows_t; ++i)
-                    bulk_g2s(dst + i * width * 2, src + (int64_t)i * a.row_stride, width * 2,
-                             &full[s]);
-                last_issued[s] = t;
+    auto load = [&](uint4 (&b)[NB], int i0) {
+#pragma unroll
+        for (int j = 0; j < R; ++j)
+#pragma unroll
+            for (int q = 0; q < CPL; ++q) {
+                const int i = i0 + j, ch = (slice * CPL + q) * 32 + lane;
+                b[j * CPL + q] = (i < n_my && ch < nch) ? ldg_stream(wbase + i * rstep + ch * 8)
+                                                        : make_uint4(0u, 0u, 0u, 0u);
             }
-            // never leave with copies in flight
-            for (int s = 0; s < kGemvStages; ++s)
-                if (last_issued[s] >= 0 && !mbar_wait(&full[s], (last_issued[s] / kGemvStages) & 1))
-                    set_status(a.status, VT_DEV_WAIT_TIMEOUT);
-        }
-        return;
-    }
+    };
+    uint4 b0[NB], b1[NB];
+    load(b0, 0);  // weights are constant: stream them before waiting on the previous kernel
+    load(b1, R);
+    if (!a.indep) pdl_wait();
 
-    // -------------------------------------------------------------- consumers (8 warps)
-    constexpr int NC = kGemvConsumerWarps * 32;
-    pdl_wait();
+    // this lane's input values
+    float xr[CPL][8];
     if (a.x != nullptr) {
         float ss = 0.f;
-        for (int i = tid * 8; i < a.k; i += NC * 8) {
+        for (int i = tid * 8; i < a.k; i += kGemvThreads * 8) {
             const uint4 u = *reinterpret_cast<const uint4*>(a.x + i);
-            const float2 p0 = h2_to_f2(u.x), p1 = h2_to_f2(u.y), p2 = h2_to_f2(u.z),
-                         p3 = h2_to_f2(u.w);
-            ss += p0.x * p0.x + p0.y * p0.y + p1.x * p1.x + p1.y * p1.y + p2.x * p2.x +
-                  p2.y * p2.y + p3.x * p3.x + p3.y * p3.y;
+            const float2 p0 = h2_to_f2(u.x), p1 = h2_to_f2(u.y), p2 = h2_to_f2(u.z), p3 = h2_to_f2(u.w);
+            ss += p0.x * p0.x + p0.y * p0.y + p1.x * p1.x + p1.y * p1.y + p2.x * p2.x + p2.y * p2.y +
+                  p3.x * p3.x + p3.y * p3.y;
         }
         ss = warp_sum(ss);
         if (lane == 0) red[warp] = ss;
-        consumer_bar(1, NC);
+        __syncthreads();
         if (tid == 0) {
             float tot = 0.f;
-            for (int w = 0; w < kGemvConsumerWarps; ++w) tot += red[w];
-            red[32] = 1.0f / sqrtf(tot / (float)a.k + a.eps);
+            for (int w = 0; w < kGemvWarps; ++w) tot += red[w];
+            red[kGemvWarps] = 1.0f / sqrtf(tot / (float)a.k + a.eps);
         }
-        consumer_bar(1, NC);
-        const float r = red[32];
-        for (int i = tid * 8; i < a.k; i += NC * 8) {
-            const uint4 u = *reinterpret_cast<const uint4*>(a.x + i);
-            const uint4 g = *reinterpret_cast<const uint4*>(a.gain + i);
-            const uint32_t uu[4] = {u.x, u.y, u.z, u.w}, gg[4] = {g.x, g.y, g.z, g.w};
+        __syncthreads();
+        const float rinv = red[kGemvWarps];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const float2 xv = h2_to_f2(uu[q]), gv = h2_to_f2(gg[q]);
-                xs[i + 2 * q] = xv.x * r * gv.x;
-                xs[i + 2 * q + 1] = xv.y * r * gv.y;
-            }
-        }
-        for (int i = a.k + tid; i < tl.kpad; i += NC) xs[i] = 0.f;
-    } else {
-        for (int i = tid; i < tl.kpad; i += NC) xs[i] = i < a.k ? a.vin[i] : 0.f;
-    }
-    consumer_bar(1, NC);
-    pdl_launch_dependents();
-
-    float part[kGemvMaxTileRows];
+        for (int q = 0; q < CPL; ++q) {
+            const int ch = (slice * CPL + q) * 32 + lane;
+            if (ch < nch) {
+                const uint4 u = *reinterpret_cast<const uint4*>(a.x + ch * 8);
+                const uint4 g = *reinterpret_cast<const uint4*>(a.gain + ch * 8);
+                const uint32_t uu[4] = {u.x, u.y, u.z, u.w}, gg[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
-    for (int i = 0; i < kGemvMaxTileRows; ++i) part[i] = 0.f;
-
-    for (int t = 0; t < ntiles; ++t) {
-        const int s = t % kGemvStages;
-        if (!mbar_wait(&full[s], (t / kGemvStages) & 1)) {
-            s_abort = 1;
-            set_status(a.status, VT_DEV_WAIT_TIMEOUT);
-            break;
-        }
-        const int rb = t / tl.ncb, cbi = t - rb * tl.ncb;
-        const int rows_t = min(tl.tr, nrows - rb * tl.tr);
-        const int width = min(tl.cb, tl.kpad - cbi * tl.cb);
-        const int nch = width >> 3;
-        const int cpw = (nch + kGemvConsumerWarps - 1) / kGemvConsumerWarps;
-        const int c_lo = warp * cpw, c_hi = min(c_lo + cpw, nch);
-        const uint8_t* tile = ring + s * kGemvStageBytes;
-        const float* xcol = xs + cbi * tl.cb;
-#pragma unroll
-        for (int i = 0; i < kGemvMaxTileRows; ++i) {
-            if (i < rows_t) {
-                float acc = 0.f;
-                const uint8_t* rowp = tile + i * width * 2;
-                for (int j = c_lo + lane; j < c_hi; j += 32)
-                    acc += dot8(lds128(rowp + j * 16), xcol + j * 8);
-                part[i] += acc;
-            }
-        }
-        if (cbi == tl.ncb - 1) {
-#pragma unroll
-            for (int i = 0; i < kGemvMaxTileRows; ++i) {
-                if (i < rows_t) {
-                    const float v = warp_sum(part[i]);
-                    if (lane == 0) slots[(rb * tl.tr + i) * kGemvConsumerWarps + warp] = v;
+                for (int e = 0; e < 4; ++e) {
+                    const float2 xv = h2_to_f2(uu[e]), gv = h2_to_f2(gg[e]);
+                    xr[q][2 * e] = xv.x * rinv * gv.x;
+                    xr[q][2 * e + 1] = xv.y * rinv * gv.y;
                 }
-                part[i] = 0.f;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) xr[q][e] = 0.f;
             }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[s]);
+    } else {
+#pragma unroll
+        for (int q = 0; q < CPL; ++q) {
+            const int ch = (slice * CPL + q) * 32 + lane;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int idx = ch * 8 + e;
+                xr[q][e] = (ch < nch && idx < a.k) ? __ldcg(a.vin + idx) : 0.f;
+            }
+        }
     }
-    consumer_bar(1, NC);
-    if (s_abort) return;
+    if (!a.indep) pdl_launch_dependents();
+
+    constexpr int per = 32 / R;
+    auto consume = [&](uint4 (&b)[NB], int i0) {
+        float v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = 0.f;
+#pragma unroll
+        for (int j = 0; j < R; ++j) {
+            float acc = 0.f;
+#pragma unroll
+            for (int q = 0; q < CPL; ++q) acc += dot8(b[j * CPL + q], xr[q]);
+            v[j] = acc;
+        }
+        load(b, i0 + 2 * R);
+        const float t = multi_row_sum<R>(v, lane);
+        const int i = i0 + lane / per;
+        if ((lane % per) == 0 && i < n_my) slots[(grp + rg * i) * kGemvWarps + slice] = t;
+    };
+    for (int i = 0; i < n_my; i += 2 * R) {
+        consume(b0, i);
+        if (i + R < n_my) consume(b1, i + R);
+    }
+    if (a.indep) {  // all reads done; complete only after the previous kernel, then publish
+        pdl_wait();
+        pdl_launch_dependents();
+    }
+    __syncthreads();
 
     // -------------------------------------------------------------- epilogues
     auto row_value = [&](int r) {
         float y = 0.f;
-#pragma unroll
-        for (int w = 0; w < kGemvConsumerWarps; ++w) y += slots[r * kGemvConsumerWarps + w];
+        for (int w = 0; w < wpr; ++w) y += slots[r * kGemvWarps + w];
         return y;
     };
     if constexpr (EPI == kEpiPlain) {
-        for (int r = tid; r < nrows; r += NC) a.out[r0 + r] = row_value(r);
+        for (int r = tid; r < nrows; r += kGemvThreads) a.out[r0 + r] = row_value(r);
     } else if constexpr (EPI == kEpiSwiglu) {
-        for (int t = tid; t < nrows / 2; t += NC) {
+        for (int t = tid; t < nrows / 2; t += kGemvThreads) {
             const float g = row_value(2 * t), u = row_value(2 * t + 1);
             a.out[r0 / 2 + t] = silu(g) * u;
         }
@@ -262,7 +269,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) k_gemv(const __grid_constant_
         const bool ok = p >= 0 && p < a.cap;
         if (!ok && tid == 0) set_status(a.status, VT_DEV_KV_OVERFLOW);
         const int half = a.dh >> 1;
-        for (int t = tid; t < nrows / 2; t += NC) {
+        for (int t = tid; t < nrows / 2; t += kGemvThreads) {
             const float ye = row_value(2 * t), yo = row_value(2 * t + 1);
             const int gr = r0 + 2 * t;
             const int b = gr / a.dh;
@@ -288,18 +295,26 @@ __global__ void __launch_bounds__(kGemvThreads, 1) k_gemv(const __grid_constant_
     }
 }
 
+template <int EPI>
+static cudaError_t launch_gemv_epi(const GemvArgs& a, int grid, cudaStream_t st) {
+    const dim3 g(grid), b(kGemvThreads);
+    switch (gemv_cpl(a.k)) {
+        case 1: return launch_k(k_gemv<EPI, 1, 8>, g, b, 0, st, a);
+        case 2: return launch_k(k_gemv<EPI, 2, 4>, g, b, 0, st, a);
+        case 3: return launch_k(k_gemv<EPI, 3, 2>, g, b, 0, st, a);
+        case 4: return launch_k(k_gemv<EPI, 4, 2>, g, b, 0, st, a);
+        default: return launch_k(k_gemv<EPI, 8, 1>, g, b, 0, st, a);
+    }
+}
+
 cudaError_t launch_gemv(int epi, const GemvArgs& a, cudaStream_t st) {
     const int unit = epi == kEpiPlain ? 1 : 2;
     const int grid = gemv_grid(a.rows, unit);
     if (grid == 0) return cudaSuccess;
-    const size_t smem = gemv_smem_bytes(a.k);
     switch (epi) {
-        case kEpiPlain:
-            return launch_k(k_gemv<kEpiPlain>, dim3(grid), dim3(kGemvThreads), smem, st, a);
-        case kEpiQkvRope:
-            return launch_k(k_gemv<kEpiQkvRope>, dim3(grid), dim3(kGemvThreads), smem, st, a);
-        default:
-            return launch_k(k_gemv<kEpiSwiglu>, dim3(grid), dim3(kGemvThreads), smem, st, a);
+        case kEpiPlain: return launch_gemv_epi<kEpiPlain>(a, grid, st);
+        case kEpiQkvRope: return launch_gemv_epi<kEpiQkvRope>(a, grid, st);
+        default: return launch_gemv_epi<kEpiSwiglu>(a, grid, st);
     }
 }
 
@@ -496,21 +511,43 @@ __global__ void __launch_bounds__(kAttnThreads) k_attn_decode(const __grid_const
     consumer_bar(1, NC);
     if (!s_last) return;
     __threadfence();
+    // Merge the nsplit slices of the group's heads.  Slice weights exp2(m_c - M) / L are computed
+    // once per (head, slice) into shared memory (the tile ring is free by now), then every
+    // (head, dim) output is a weighted sum over the slices.
+    float* wts = reinterpret_cast<float*>(ring);  // [G][nsplit]
+    for (int h = warp; h < G; h += kAttnWarps) {
+        const float* ml = a.part_ml + (int64_t)(j * G + h) * a.nsplit * 2;
+        float M = -INFINITY;
+        for (int cc = lane; cc < a.nsplit; cc += 32) M = fmaxf(M, __ldcg(ml + 2 * cc));
+        M = warp_max(M);
+        float L = 0.f;
+        for (int cc = lane; cc < a.nsplit; cc += 32) {
+            const float mc = __ldcg(ml + 2 * cc);
+            const float f = mc == -INFINITY ? 0.f : exp2f(mc - M);
+            wts[h * a.nsplit + cc] = f;
+            L += __ldcg(ml + 2 * cc + 1) * f;
+        }
+        L = warp_sum(L);
+        const float inv = L > 0.f ? 1.0f / L : 0.f;
+        __syncwarp();
+        for (int cc = lane; cc < a.nsplit; cc += 32) wts[h * a.nsplit + cc] *= inv;
+    }
+    consumer_bar(1, NC);
     for (int idx = tid; idx < G * DH; idx += NC) {
         const int h = idx / DH, d = idx - h * DH;
         const int hl = j * G + h;
-        const float* ml = a.part_ml + (int64_t)hl * a.nsplit * 2;
-        float M = -INFINITY;
-        for (int cc = 0; cc < a.nsplit; ++cc) M = fmaxf(M, __ldcg(ml + 2 * cc));
-        float L = 0.f, O = 0.f;
-        for (int cc = 0; cc < a.nsplit; ++cc) {
-            const float mc = __ldcg(ml + 2 * cc);
-            if (mc == -INFINITY) continue;
-            const float f = exp2f(mc - M);
-            L += __ldcg(ml + 2 * cc + 1) * f;
-            O += __ldcg(a.part_o + ((int64_t)hl * a.nsplit + cc) * DH + d) * f;
+        const float* po = a.part_o + (int64_t)hl * a.nsplit * DH + d;
+        const float* w = wts + h * a.nsplit;
+        float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+        int cc = 0;
+        for (; cc + 4 <= a.nsplit; cc += 4) {
+            O0 += w[cc] * __ldcg(po + (int64_t)cc * DH);
+            O1 += w[cc + 1] * __ldcg(po + (int64_t)(cc + 1) * DH);
+            O2 += w[cc + 2] * __ldcg(po + (int64_t)(cc + 2) * DH);
+            O3 += w[cc + 3] * __ldcg(po + (int64_t)(cc + 3) * DH);
         }
-        a.out[hl * DH + d] = L > 0.f ? O / L : 0.f;
+        for (; cc < a.nsplit; ++cc) O0 += w[cc] * __ldcg(po + (int64_t)cc * DH);
+        a.out[hl * DH + d] = (O0 + O1) + (O2 + O3);
     }
     if (tid == 0) a.tickets[j] = 0;
 }
@@ -661,11 +698,7 @@ static cudaError_t allow_smem(K kern, size_t want) {
 }
 
 cudaError_t init_decode_kernels() {
-    const size_t gemv_max = 232448;  // the largest request is capped by allow_smem
     cudaError_t e;
-    if ((e = allow_smem(k_gemv<kEpiPlain>, gemv_max)) != cudaSuccess) return e;
-    if ((e = allow_smem(k_gemv<kEpiQkvRope>, gemv_max)) != cudaSuccess) return e;
-    if ((e = allow_smem(k_gemv<kEpiSwiglu>, gemv_max)) != cudaSuccess) return e;
 #define VT_ATTN_ATTR(DH, G) \
     if ((e = allow_smem(k_attn_decode<DH, G>, attn_decode_smem_bytes(DH))) != cudaSuccess) return e;
     VT_ATTN_ATTR(64, 1) VT_ATTN_ATTR(64, 2) VT_ATTN_ATTR(64, 4) VT_ATTN_ATTR(64, 8)

@@ -14,12 +14,10 @@
 namespace vt {
 
 // ------------------------------------------------------------------ decode GEMV geometry
-constexpr int kGemvConsumerWarps = 8;
-constexpr int kGemvThreads = (kGemvConsumerWarps + 1) * 32;  // + one producer warp
-constexpr int kGemvStages = 4;
-constexpr int kGemvStageBytes = 16384;
+constexpr int kGemvWarps = 8;
+constexpr int kGemvThreads = kGemvWarps * 32;
 constexpr int kGemvMaxSlabRows = 128;  // rows per CTA (slot array bound)
-constexpr int kGemvMaxTileRows = 8;    // rows of one pipeline stage
+constexpr int kGemvMaxK = 16384;       // longest row: 8 warps x 32 lanes x 8 chunks x 8 halves
 
 // ------------------------------------------------------------------ decode attention geometry
 constexpr int kAttnWarps = 4;
@@ -27,6 +25,7 @@ constexpr int kAttnThreads = (kAttnWarps + 1) * 32;  // + one producer warp
 constexpr int kAttnTilePos = 32;                     // cached positions per pipeline stage
 constexpr int kAttnStages = 3;
 constexpr int kAttnMaxGroup = 8;  // query heads per KV head supported by the decode kernel
+constexpr int kAttnMaxSplit = 256; // KV slices per head (the merge stages G x nsplit weights in smem)
 
 enum GemvEpilogue : int {
     kEpiPlain = 0,   // out[r] = y[r] (fp32)
@@ -56,6 +55,9 @@ struct GemvArgs {
     int hq;              // query heads of the shard
     int hk;              // KV heads of the shard
     uint32_t* status;
+    // 1: the input vector was written at least two launches earlier, so the kernel may read it
+    // before griddepcontrol.wait and stream its whole slab while the previous kernel runs
+    int indep;
 };
 
 struct AttnDecodeArgs {
@@ -90,7 +92,7 @@ extern int g_num_sms;
 
 cudaError_t launch_gemv(int epi, const GemvArgs& a, cudaStream_t st);
 int gemv_grid(int rows, int unit);
-size_t gemv_smem_bytes(int k);
+int gemv_cpl(int k);
 cudaError_t launch_attn_decode(const AttnDecodeArgs& a, cudaStream_t st);
 size_t attn_decode_smem_bytes(int dh);
 cudaError_t launch_combine(const CombineArgs& a, cudaStream_t st);
