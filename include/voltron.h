@@ -190,7 +190,7 @@ VT_API vt_status vt_shard_weights_read(const vt_partition* part, vt_shard shard,
  *    and at row b*dh + 2i + 1 the source row of dimension i + dh/2 (RoPE partners adjacent).
  *  which 2 (O): rows = D, stride = h_s*dh: columns [h0*dh, h1*dh) of Wo.
  *  which 4 (gate/up): rows = 2 * c_s: row 2j = gate row c0 + j, row 2j + 1 = up row c0 + j.
- *  which 5 (down): rows = D, stride = c_s rounded up to 8 (padding zero): columns [c0, c1) of Wd.
+ *  which 5 (down, transposed): rows = c_s, stride = D: row j = column c0 + j of Wd.
  *  which 0, 3: one row of D. */
 VT_API vt_status vt_shard_weight_layout(const vt_partition* part, vt_shard shard, int32_t which,
                                  int64_t* rows, int64_t* row_stride);

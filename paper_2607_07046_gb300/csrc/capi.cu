@@ -92,6 +92,8 @@ cudaError_t init_library() {
     std::call_once(g_init_once, [] {
         const char* e = getenv("VT_NO_PDL");
         g_use_pdl = !(e && e[0] && e[0] != '0');
+        const char* gm = getenv("VT_GRID_MULT");
+        if (gm && gm[0] >= '1' && gm[0] <= '4') g_grid_mult = gm[0] - '0';
         int dev = 0;
         g_init_err = cudaGetDevice(&dev);
         if (g_init_err != cudaSuccess) return;
@@ -135,19 +137,15 @@ struct AttnShard {
 struct FfnShard {
     void* base = nullptr;
     __half* norm = nullptr;
-    __half* wgu = nullptr;  // [2c][D]
-    __half* wd = nullptr;   // [D][ld]
-    int c0 = 0, c1 = 0, ld = 0;
+    __half* wgu = nullptr;  // [2c][D], gate/up rows interleaved
+    __half* wdt = nullptr;  // [c][D], row j = column c0 + j of Wd
+    int c0 = 0, c1 = 0;
 };
 
 struct DecodeScratch {  // per device of the partition
-    float* q = nullptr;
-    float* attn = nullptr;
-    float* part_ml = nullptr;
-    float* part_o = nullptr;
-    int32_t* tickets = nullptr;
-    float* u = nullptr;
-    int nsplit = 1;
+    float* q = nullptr;     // [hq][dh] rotated queries of the token
+    float* attn = nullptr;  // [hq][dh] attention output (input of the O projection)
+    int ffn_grid = 0;       // CTAs of the fused FFN kernel
 };
 
 constexpr int kPrefillChunk = 1024;  // rows per prefill pass (longer prompts run in chunks)
@@ -162,6 +160,7 @@ struct vt_partition {
     std::vector<void*> owned;  // every allocation besides the shard bases
     uint32_t* status = nullptr;
     // whole-stack buffers
+    float* dpart = nullptr;     // [n_dev][D] decode partials (kept zero between blocks)
     float* partials = nullptr;  // [n_dev][kPrefillChunk][D]
     __half* hbuf = nullptr;     // [kPrefillChunk][D]
     __half* xbuf = nullptr;     // [kPrefillChunk][D]
@@ -535,16 +534,15 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
             fs.c0 = cols[d].begin;
             fs.c1 = cols[d].end;
             const int c = fs.c1 - fs.c0;
-            fs.ld = round_up8(c);
             if (c > 0) {
                 const size_t bytes = align256((size_t)D * 2) + align256((size_t)2 * c * D * 2) +
-                                     align256((size_t)D * fs.ld * 2);
+                                     align256((size_t)c * D * 2);
                 fs.base = A.get(bytes);
                 if (!fs.base) return bail(fail(VT_ERR_ALLOC, "shard allocation failed"));
                 Bump b{static_cast<uint8_t*>(fs.base)};
                 fs.norm = b.take<__half>(D);
                 fs.wgu = b.take<__half>((size_t)2 * c * D);
-                fs.wd = b.take<__half>((size_t)D * fs.ld);
+                fs.wdt = b.take<__half>((size_t)c * D);
                 VT_CUDA(cudaMemcpyAsync(fs.norm, L.ffn_norm, (size_t)D * 2,
                                         cudaMemcpyDeviceToDevice, st));
                 rows_host.clear();
@@ -556,9 +554,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
                                         cudaMemcpyHostToDevice, st));
                 VT_CUDA(launch_gather_rows(rows_dev, fs.wgu, (int)rows_host.size(), D, D, st));
                 VT_CUDA(cudaStreamSynchronize(st));
-                VT_CUDA(cudaMemsetAsync(fs.wd, 0, (size_t)D * fs.ld * 2, st));
-                VT_CUDA(cudaMemcpy2DAsync(fs.wd, (size_t)fs.ld * 2, L.w_down + fs.c0, (size_t)F * 2,
-                                          (size_t)c * 2, D, cudaMemcpyDeviceToDevice, st));
+                VT_CUDA(launch_transpose_f16(L.w_down + fs.c0, F, D, c, fs.wdt, D, st));
             }
         }
     }
@@ -569,38 +565,29 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     for (int d = 0; d < n; ++d) {
         const int hq = heads[d].end - heads[d].begin, hk = hq / g, c = cols[d].end - cols[d].begin;
         DecodeScratch& ds = p->dec[d];
-        const int target = 2 * (g_num_sms > 0 ? g_num_sms : 148);
-        int ns = hk > 0 ? (target + hk - 1) / hk : 1;
-        const int ns_max = std::max(1, s.max_seq / 16);
-        ns = std::max(1, std::min(std::min(ns, ns_max), kAttnMaxSplit));
-        ds.nsplit = ns;
-        const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2 +
-                             align256((size_t)std::max(hq, 1) * ns * 2 * 4) +
-                             align256((size_t)std::max(hq, 1) * ns * dh * 4) +
-                             align256((size_t)std::max(hk, 1) * 4) + align256((size_t)std::max(c, 1) * 4);
+        ds.ffn_grid = ffn_grid(c);
+        const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2;
         void* q;
         if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
         Bump b{static_cast<uint8_t*>(q)};
         ds.q = b.take<float>((size_t)std::max(hq, 1) * dh);
         ds.attn = b.take<float>((size_t)std::max(hq, 1) * dh);
-        ds.part_ml = b.take<float>((size_t)std::max(hq, 1) * ns * 2);
-        ds.part_o = b.take<float>((size_t)std::max(hq, 1) * ns * dh);
-        ds.tickets = b.take<int32_t>(std::max(hk, 1));
-        ds.u = b.take<float>(std::max(c, 1));
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
         p->max_hq = std::max(p->max_hq, hq);
         p->max_ld = std::max(p->max_ld, round_up8(c));
+        (void)hk;
     }
     // ------------------------------------------------------------------ stack + prefill scratch
     {
         const size_t R = kPrefillChunk;
-        const size_t bytes = align256(4) + align256((size_t)n * R * D * 4) + 2 * align256(R * D * 2) +
+        const size_t bytes = align256(4) + align256((size_t)n * D * 4) + align256((size_t)n * R * D * 4) + 2 * align256(R * D * 2) +
                              align256(R * D * 2) + 2 * align256(R * std::max(p->max_hq, 1) * dh * 2) +
                              align256(R * std::max(p->max_ld, 8) * 2);
         void* q;
         if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
         Bump b{static_cast<uint8_t*>(q)};
         p->status = b.take<uint32_t>(1);
+        p->dpart = b.take<float>((size_t)n * D);
         p->partials = b.take<float>((size_t)n * R * D);
         p->hbuf = b.take<__half>(R * D);
         p->xbuf = b.take<__half>(R * D);
@@ -655,7 +642,7 @@ extern "C" vt_status vt_shard_weight_layout(const vt_partition* p, vt_shard sh, 
         case 2: *rows = hq > 0 ? s.d_model : 0; *stride = (int64_t)hq * s.d_head; break;
         case 3: *rows = c > 0; *stride = s.d_model; break;
         case 4: *rows = 2 * (int64_t)c; *stride = s.d_model; break;
-        case 5: *rows = c > 0 ? s.d_model : 0; *stride = f.ld; break;
+        case 5: *rows = c; *stride = s.d_model; break;
         default: return fail(VT_ERR_INVALID_ARG, "unknown tensor %d", which);
     }
     return ok();
@@ -674,7 +661,7 @@ extern "C" vt_status vt_shard_weights_read(const vt_partition* p, vt_shard sh, i
         case 2: src = a.wo; break;
         case 3: src = f.norm; break;
         case 4: src = f.wgu; break;
-        default: src = f.wd; break;
+        default: src = f.wdt; break;
     }
     const size_t size = (size_t)rows * stride * 2;
     if (size_out) *size_out = size;
@@ -871,11 +858,8 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
     t.hk = hk;
     t.group = s.n_heads / s.n_kv_heads;
     t.dh = dh;
-    t.nsplit = ds.nsplit;
+    t.stages = attn_stages(kv->cap, attn_cluster_size(hk));
     t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
-    t.part_ml = ds.part_ml;
-    t.part_o = ds.part_o;
-    t.tickets = ds.tickets;
     t.out = ds.attn;
     t.status = kv->status;
     VT_CUDA(launch_attn_decode(t, st));
@@ -892,37 +876,27 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
     return VT_OK;
 }
 
+// FFN shard decode: the fused column-split kernel adds every CTA's partial into `out`, which
+// must hold zeros; `zero_first` clears it in stream order before the kernel runs.
 static vt_status decode_ffn(const vt_partition* p, int l, int d, const __half* x, float* out,
-                            cudaStream_t st, int indep = 0) {
+                            cudaStream_t st, int indep = 0, bool zero_first = true) {
     const vt_shapes& s = p->m->s;
     const FfnShard& f = p->f(l, d);
     const DecodeScratch& ds = p->dec[d];
     const int c = f.c1 - f.c0, D = s.d_model;
-    if (c == 0) {
-        VT_CUDA(launch_fill_zero_f32(out, D, st));
-        return VT_OK;
-    }
-    GemvArgs g{};
-    g.w = f.wgu;
-    g.row_stride = D;
-    g.rows = 2 * c;
-    g.k = D;
+    if (zero_first) VT_CUDA(launch_fill_zero_f32(out, D, st));
+    if (c == 0) return VT_OK;
+    FfnDecodeArgs g{};
     g.x = x;
     g.gain = f.norm;
     g.eps = s.rms_eps;
-    g.out = ds.u;
-    g.status = p->status;
+    g.wgu = f.wgu;
+    g.wdt = f.wdt;
+    g.d = D;
+    g.cols = c;
+    g.out = out;
     g.indep = indep;
-    VT_CUDA(launch_gemv(kEpiSwiglu, g, st));
-    GemvArgs o{};
-    o.w = f.wd;
-    o.row_stride = f.ld;
-    o.rows = D;
-    o.k = c;
-    o.vin = ds.u;
-    o.out = out;
-    o.status = p->status;
-    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    VT_CUDA(launch_ffn_decode(g, ds.ffn_grid, st));
     return VT_OK;
 }
 
@@ -951,7 +925,7 @@ extern "C" vt_status vt_combine(const float* const* partials, int32_t n, int32_t
     CombineArgs c{};
     for (int s = 0; s < n; ++s) {
         if (!partials[s]) return fail(VT_ERR_INVALID_ARG, "partial %d is NULL", s);
-        c.parts[s] = partials[s];
+        c.parts[s] = const_cast<float*>(partials[s]);
     }
     c.n = n;
     c.count = (int64_t)rows * d;
@@ -1011,12 +985,12 @@ static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half*
         t.n = n;
         t.d = D;
         t.c = c;
-        t.ld_down = f.ld;
+        t.ld_down = s.d_model;
         t.eps = s.rms_eps;
         t.x = x;
         t.gain = f.norm;
         t.wgu = f.wgu;
-        t.wd = f.wd;
+        t.wd = f.wdt;
         t.xhat = p->p_xhat;
         t.u = p->p_u;
         t.out = out;
@@ -1062,20 +1036,35 @@ extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const voi
             return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions", l, kv->h_len[l], kv->cap);
     cudaStream_t st = (cudaStream_t)stream;
     const int D = s.d_model, n = p->n_dev;
+    // One fp32 partial buffer per shard serves both blocks: the O projection stores the ATTN
+    // partial; the ATTN combine reads and clears it; the FFN kernels add into it; the FFN combine
+    // reads and clears it again (buffers start zeroed, so empty shards contribute zeros).
     CombineArgs c{};
     c.n = n;
     c.count = D;
-    for (int d = 0; d < n; ++d) c.parts[d] = p->partials + (size_t)d * D;
+    c.clear = 1;
+    for (int d = 0; d < n; ++d) c.parts[d] = p->dpart + (size_t)d * D;
     const __half* cur = static_cast<const __half*>(x_in);
     for (int l = 0; l < s.n_layers; ++l) {
-        // Shard d >= 1 reads the layer input written by the combine several launches earlier.
-        for (int d = 0; d < n; ++d)
-            VT_TRY(decode_attn(p, l, d, cur, kv, p->partials + (size_t)d * D, st, d > 0));
+        // After the first launched shard of a block, a shard's input was written by the combine
+        // at least two launches earlier, so its first kernel may read it before waiting.
+        bool launched = false;
+        for (int d = 0; d < n; ++d) {
+            const AttnShard& as = p->a(l, d);
+            if (as.h1 == as.h0) continue;
+            VT_TRY(decode_attn(p, l, d, cur, kv, p->dpart + (size_t)d * D, st, launched));
+            launched = true;
+        }
         c.residual = cur;
         c.out = p->hbuf;
         VT_CUDA(launch_combine(c, st));
-        for (int d = 0; d < n; ++d)
-            VT_TRY(decode_ffn(p, l, d, p->hbuf, p->partials + (size_t)d * D, st, d > 0));
+        launched = false;
+        for (int d = 0; d < n; ++d) {
+            const FfnShard& fs = p->f(l, d);
+            if (fs.c1 == fs.c0) continue;
+            VT_TRY(decode_ffn(p, l, d, p->hbuf, p->dpart + (size_t)d * D, st, launched, false));
+            launched = true;
+        }
         __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) : p->xbuf;
         c.residual = p->hbuf;
         c.out = dst;

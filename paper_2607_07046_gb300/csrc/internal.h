@@ -19,13 +19,17 @@ constexpr int kGemvThreads = kGemvWarps * 32;
 constexpr int kGemvMaxSlabRows = 128;  // rows per CTA (slot array bound)
 constexpr int kGemvMaxK = 16384;       // longest row: 8 warps x 32 lanes x 8 chunks x 8 halves
 
+
 // ------------------------------------------------------------------ decode attention geometry
-constexpr int kAttnWarps = 4;
+constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = (kAttnWarps + 1) * 32;  // + one producer warp
-constexpr int kAttnTilePos = 32;                     // cached positions per pipeline stage
-constexpr int kAttnStages = 3;
+// cached positions per pipeline stage: K and V of a stage are two bulk copies of 64 rows; a
+// bulk copy carries a fixed engine cost, so copies of 16 KB or more are needed to stream at full
+// rate (8 KB copies reach about half of it).
+constexpr int kAttnTilePos = 64;
+constexpr int kAttnMaxStages = 3;                    // tiles of K and V in flight per CTA
+constexpr int kAttnMaxCluster = 16;                  // CTAs per KV head (thread-block cluster)
 constexpr int kAttnMaxGroup = 8;  // query heads per KV head supported by the decode kernel
-constexpr int kAttnMaxSplit = 256; // KV slices per head (the merge stages G x nsplit weights in smem)
 
 enum GemvEpilogue : int {
     kEpiPlain = 0,   // out[r] = y[r] (fp32)
@@ -56,7 +60,9 @@ struct GemvArgs {
     int hk;              // KV heads of the shard
     uint32_t* status;
     // 1: the input vector was written at least two launches earlier, so the kernel may read it
-    // before griddepcontrol.wait and stream its whole slab while the previous kernel runs
+    // before griddepcontrol.wait and stream its whole slab while the previous kernel runs.  Such
+    // a kernel releases its dependents at once: they may only read, before their own wait, data
+    // that was complete when this kernel started (weights, earlier tokens' KV entries, lengths).
     int indep;
 };
 
@@ -69,33 +75,51 @@ struct AttnDecodeArgs {
     int hk;                // KV heads of the shard
     int group;             // query heads per KV head
     int dh;
-    int nsplit;
+    int stages;            // K/V tiles in flight per CTA (attn_stages)
     float scale_log2;      // log2(e) / sqrt(dh)
-    float* part_ml;        // [h_s][nsplit][2]  (running max in log2 units, sum)
-    float* part_o;         // [h_s][nsplit][dh]
-    int32_t* tickets;      // [hk_s], zero between calls
-    float* out;            // [h_s][dh]
+    float* out;            // [h_s][dh] attention output of the shard's query heads
     uint32_t* status;
 };
 
 struct CombineArgs {
-    const float* parts[VT_MAX_DEVICES];
+    float* parts[VT_MAX_DEVICES];  // shard s: one partial of `count` floats (nullptr: none)
     int n;
     int64_t count;
-    const __half* residual;
+    const __half* residual;  // nullable
     __half* out;
+    int clear;               // 1: zero every partial after reading it (consume and clear)
+};
+
+constexpr int kFfnMaxCols = 64;  // intermediate columns per CTA of the fused FFN kernel
+
+struct FfnDecodeArgs {
+    const __half* x;     // [d] block input (h)
+    const __half* gain;  // [d]
+    float eps;
+    const __half* wgu;   // [2 cols][d] gate/up rows interleaved
+    const __half* wdt;   // [cols][d] transposed down slice
+    int d, cols;
+    float* out;          // [d] shard partial; the kernel adds into it (must start at zero)
+    int indep;           // as GemvArgs::indep
 };
 
 // ------------------------------------------------------------------ launchers (stream-ordered)
 extern bool g_use_pdl;  // programmatic dependent launch between the library's kernels
+extern int g_grid_mult; // CTAs per SM of the streaming kernels
 extern int g_num_sms;
 
 cudaError_t launch_gemv(int epi, const GemvArgs& a, cudaStream_t st);
 int gemv_grid(int rows, int unit);
 int gemv_cpl(int k);
 cudaError_t launch_attn_decode(const AttnDecodeArgs& a, cudaStream_t st);
-size_t attn_decode_smem_bytes(int dh);
+size_t attn_decode_smem_bytes(int dh, int group, int stages);
+int attn_cluster_size(int hk);
+int attn_stages(int cap, int csize);
 cudaError_t launch_combine(const CombineArgs& a, cudaStream_t st);
+int ffn_grid(int cols);
+cudaError_t launch_ffn_decode(const FfnDecodeArgs& a, int grid, cudaStream_t st);
+cudaError_t launch_transpose_f16(const __half* src, int64_t src_ld, int rows, int cols, __half* dst,
+                                 int64_t dst_ld, cudaStream_t st);
 cudaError_t launch_fill_zero_f32(float* p, int64_t n, cudaStream_t st);
 cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, cudaStream_t st);
 cudaError_t launch_rope_table(float2* tab, int max_seq, int dh, double theta, cudaStream_t st);

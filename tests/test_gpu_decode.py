@@ -174,10 +174,8 @@ def test_shard_weights_are_exact_slices(vtlib):
                 c0, c1 = cr
                 gu = np.stack([w["w_gate"][c0:c1], w["w_up"][c0:c1]], 1).reshape(2 * (c1 - c0), -1)
                 assert np.array_equal(vtlib.vt_shard_weights_read(st.part, (l, d, 1), 4), gu)
-                down = vtlib.vt_shard_weights_read(st.part, (l, d, 1), 5)
-                assert down.shape[1] == (c1 - c0 + 7) // 8 * 8
-                assert np.array_equal(down[:, :c1 - c0], w["w_down"][:, c0:c1])
-                assert not down[:, c1 - c0:].any()
+                down_t = vtlib.vt_shard_weights_read(st.part, (l, d, 1), 5)
+                assert np.array_equal(down_t, w["w_down"][:, c0:c1].T)
                 assert np.array_equal(vtlib.vt_shard_weights_read(st.part, (l, d, 1), 3)[0],
                                       w["ffn_norm"])
 
@@ -224,7 +222,9 @@ def test_kv_tagged_round_trip_and_append_position(vtlib):
         assert [vtlib.vt_kv_length(st.kv, l) for l in range(2)] == [3, L + 3]
 
 
-def test_decode_is_bit_reproducible(vtlib):
+def test_decode_is_reproducible(vtlib):
+    """ATTN partials repeat bit for bit; FFN partials are added into the output by bulk
+    reductions whose order across CTAs varies, so they repeat to fp32 rounding."""
     wl = synthetic.WORKLOADS[1]
     kc, vc = wl.kv_fill(0, 128, 136)
     with build(vtlib, wl, capacity=136) as st:
@@ -237,8 +237,11 @@ def test_decode_is_bit_reproducible(vtlib):
             for d in range(2):
                 vtlib.vt_decode_step(st.part, (0, d, ATTN), x, st.kv, o[d])
                 vtlib.vt_decode_step(st.part, (0, d, FFN), x, None, o[2 + d])
-            outs.append([host(t).tobytes() for t in o])
-        assert outs[0] == outs[1]
+            outs.append([host(t) for t in o])
+        for d in range(2):
+            assert outs[0][d].tobytes() == outs[1][d].tobytes()
+            ffn_a, ffn_b = outs[0][2 + d].astype(np.float64), outs[1][2 + d].astype(np.float64)
+            assert np.max(np.abs(ffn_a - ffn_b)) <= 1e-6 * max(1.0, np.max(np.abs(ffn_a)))
 
 
 # ------------------------------------------------------------------ whole stack + graphs
