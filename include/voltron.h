@@ -33,8 +33,9 @@
  *    capacity during graph replay, a wait that gave up) set bits in a device status word, read
  *    with vt_kv_status / vt_partition_status.
  *  - Threads: objects are not internally locked; use one object from one host thread at a time.
- *  - Streams and graphs: every compute call can be captured into a CUDA graph; positions come from
- *    device-resident KV lengths, so a replayed graph appends at the right place.
+ *  - Streams and graphs: every compute call except vt_decode_step_static can be captured into a
+ *    CUDA graph; positions come from device-resident KV lengths, so a replayed graph appends at
+ *    the right place.  (No claim is made for vt_decode_step_static.)
  */
 #ifndef VOLTRON_H
 #define VOLTRON_H
@@ -232,6 +233,33 @@ VT_API vt_status vt_kv_write_raw(vt_kv* kv, int32_t layer, int32_t device, int32
  */
 VT_API vt_status vt_decode_step(const vt_partition* part, vt_shard shard, const void* x, vt_kv* kv,
                          float* out_partial, vt_stream stream);
+
+/* vt_decode_step_static: vt_decode_step for an ATTN shard with no allocation and no allocated
+ * scratch.  The paper has no counterpart; it is a library convenience.
+ *   Who needs it: callers that cannot allocate device memory when they run decoding.  For
+ *   example, a host whose memory plan has given all of HBM to the weights and the KV cache, or
+ *   one whose allocator cannot be entered from the thread that drives decoding.  The step keeps
+ *   every intermediate in one file-scope __device__ array of 1 MiB (1048576 bytes) that is part
+ *   of the library's device image.  It calls no cudaMalloc, cudaFree or other allocating routine.
+ *   It does not use the partition's decode scratch.
+ *   Computation: as vt_decode_step for the ATTN shard.  Attention runs as split-K over 16 slices
+ *   per KV head.  The slices are merged by the last one to finish, so results match
+ *   vt_decode_step to rounding, not bit for bit.
+ *   Arguments, layouts, ownership: as vt_decode_step.  kv is required.  Does not advance the KV
+ *   length.
+ *   Limits: the shard needs 256 + 8*h_s*dh + 64*hk_s*G*(dh+2) bytes (each region rounded up to
+ *   256 bytes; G = query heads per KV head), at most 1 MiB, and hk_s <= 64.  A larger shard
+ *   returns VT_ERR_INVALID_ARG with the byte count in vt_last_error().  An FFN shard returns
+ *   VT_ERR_INVALID_ARG (it uses no scratch; call vt_decode_step).
+ *   First call on a device: looks up the array's device address with cudaGetSymbolAddress, with
+ *   that device current, and keeps it.  Any failure is VT_ERR_CUDA.  Make that first call before
+ *   any stream capture on that device begins.
+ *   Must start at zero: only the 64 per-KV-head arrival counters at the start of the array.  The
+ *   module loader zeroes them, and every call leaves them at zero.
+ *   Races: the array is shared by every call in the process on that device.  Two calls in flight
+ *   at once, on different streams or host threads, corrupt each other.  Order them. */
+VT_API vt_status vt_decode_step_static(const vt_partition* part, vt_shard shard, const void* x, vt_kv* kv,
+                                float* out_partial, vt_stream stream);
 
 /* vt_prefill: n prompt rows through one shard (n >= 1).
  *   ATTN shard: rows sit at positions p0..p0+n-1 with p0 = current length of the layer; row i

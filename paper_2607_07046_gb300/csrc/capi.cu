@@ -918,6 +918,89 @@ extern "C" vt_status vt_decode_step(const vt_partition* p, vt_shard sh, const vo
     return ok();
 }
 
+// ATTN shard step with every intermediate in the module's static scratch array: the same QKV and
+// O kernels as decode_attn, with the split-K attention kernel of static_scratch.cu between them.
+// Touches neither the partition's decode scratch nor any allocator.
+extern "C" vt_status vt_decode_step_static(const vt_partition* p, vt_shard sh, const void* x, vt_kv* kv,
+                                           float* out, vt_stream stream) {
+    VT_TRY(check_shard(p, sh));
+    if (sh.block != VT_BLOCK_ATTN)
+        return fail(VT_ERR_INVALID_ARG, "vt_decode_step_static runs ATTN shards only (an FFN shard uses no scratch: call vt_decode_step)");
+    if (!x || !out) return fail(VT_ERR_INVALID_ARG, "x and out_partial must not be NULL");
+    if (!aligned16(x)) return fail(VT_ERR_INVALID_ARG, "x must be 16-byte aligned");
+    if (!kv || kv->p != p) return fail(VT_ERR_INVALID_ARG, "an ATTN shard needs this partition's KV cache");
+    if (kv->h_len[sh.layer] + 1 > kv->cap)
+        return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions", sh.layer, kv->h_len[sh.layer], kv->cap);
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(sh.layer, sh.device);
+    const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, dh = s.d_head, D = s.d_model, l = sh.layer, d = sh.device;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (hq == 0) {
+        VT_CUDA(launch_fill_zero_f32(out, D, st));
+        return ok();
+    }
+    const StaticAttnLayout lay = static_attn_layout(hq, hk, dh);
+    if (hk > kStaticMaxKvHeads || lay.bytes > kStaticScratchBytes)
+        return fail(VT_ERR_INVALID_ARG,
+                    "shard (layer %d, device %d) needs %zu bytes of static scratch for %d query and %d KV "
+                    "heads of dim %d; the array holds %zu bytes and %d KV heads",
+                    l, d, lay.bytes, hq, hk, dh, kStaticScratchBytes, kStaticMaxKvHeads);
+    void* base = nullptr;
+    cudaError_t ce = static_scratch_base(&base);
+    if (ce != cudaSuccess)
+        return fail(VT_ERR_CUDA, "looking up the static scratch address failed: %s", cudaGetErrorString(ce));
+    uint8_t* b = static_cast<uint8_t*>(base);
+    float* q = reinterpret_cast<float*>(b + lay.q);
+    float* attn = reinterpret_cast<float*>(b + lay.attn);
+
+    GemvArgs g{};
+    g.w = a.wqkv;
+    g.row_stride = D;
+    g.rows = (hq + 2 * hk) * dh;
+    g.k = D;
+    g.x = static_cast<const __half*>(x);
+    g.gain = a.norm;
+    g.eps = s.rms_eps;
+    g.out = q;
+    g.kcache = kv->k(l, d);
+    g.vcache = kv->v(l, d);
+    g.cap = kv->cap;
+    g.len = kv->len + l;
+    g.rope = p->m->rope;
+    g.dh = dh;
+    g.hq = hq;
+    g.hk = hk;
+    g.status = kv->status;
+    VT_CUDA(launch_gemv(kEpiQkvRope, g, st));
+
+    StaticAttnArgs t{};
+    t.q = q;
+    t.kcache = kv->k(l, d);
+    t.vcache = kv->v(l, d);
+    t.len = kv->len + l;
+    t.cap = kv->cap;
+    t.hk = hk;
+    t.group = s.n_heads / s.n_kv_heads;
+    t.dh = dh;
+    t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    t.part_ml = reinterpret_cast<float*>(b + lay.part_ml);
+    t.part_o = reinterpret_cast<float*>(b + lay.part_o);
+    t.counters = reinterpret_cast<uint32_t*>(b + lay.counters);
+    t.out = attn;
+    VT_CUDA(launch_attn_decode_static(t, st));
+
+    GemvArgs o{};
+    o.w = a.wo;
+    o.row_stride = (int64_t)hq * dh;
+    o.rows = D;
+    o.k = hq * dh;
+    o.vin = attn;
+    o.out = out;
+    o.status = kv->status;
+    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    return ok();
+}
+
 extern "C" vt_status vt_combine(const float* const* partials, int32_t n, int32_t rows, int32_t d,
                                 const void* residual, void* out, vt_stream stream) {
     if (!partials || !out || n < 1 || n > VT_MAX_DEVICES || rows < 0 || d < 0)

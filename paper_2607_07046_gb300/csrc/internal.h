@@ -171,6 +171,33 @@ struct PrefillFfnArgs {
     uint32_t* status;
 };
 vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err);
+
+// ------------------------------------------------------------------ static-scratch decode attention
+// (static_scratch.cu) split-K decode attention whose scratch is one file-scope __device__ array.
+constexpr size_t kStaticScratchBytes = (size_t)1 << 20;  // 1 MiB
+constexpr int kStaticSplits = 16;                        // position slices per KV head
+constexpr int kStaticMaxKvHeads = 64;                    // arrival counters
+constexpr int kStaticMaxDevices = 64;                    // cached symbol addresses
+
+struct StaticAttnLayout {  // byte offsets of the regions in the array
+    size_t counters, q, attn, part_ml, part_o, bytes;
+};
+StaticAttnLayout static_attn_layout(int hq, int hk, int dh);
+cudaError_t static_scratch_base(void** out);
+
+struct StaticAttnArgs {
+    const float* q;        // [hq][dh] rotated queries
+    const __half* kcache;  // [hk][cap][dh]
+    const __half* vcache;
+    const int32_t* len;
+    int cap, hk, group, dh;
+    float scale_log2;
+    float* part_ml;        // [hk][kStaticSplits][group][2] (max, sum) of each slice
+    float* part_o;         // [hk][kStaticSplits][group][dh] weighted V of each slice
+    uint32_t* counters;    // [hk] slices finished; zero between calls
+    float* out;            // [hq][dh]
+};
+cudaError_t launch_attn_decode_static(const StaticAttnArgs& a, cudaStream_t st);
 vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err);
 
 }  // namespace vt

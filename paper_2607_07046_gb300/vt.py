@@ -114,6 +114,7 @@ def lib() -> ctypes.CDLL:
             "vt_kv_read": (S, [_P, _I32, _I32, _I32, _P, _P]),
             "vt_kv_write_raw": (S, [_P, _I32, _I32, _I32, _P, _P]),
             "vt_decode_step": (S, [_P, vt_shard, _P, _P, _P, _P]),
+            "vt_decode_step_static": (S, [_P, vt_shard, _P, _P, _P, _P]),
             "vt_prefill": (S, [_P, vt_shard, _P, _I32, _P, _P, _P]),
             "vt_combine": (S, [ctypes.POINTER(_P), _I32, _I32, _I32, _P, _P, _P]),
             "vt_decode_token": (S, [_P, _P, _P, _P, _P]),
@@ -357,6 +358,17 @@ def vt_decode_step(part: int, shard: Tuple[int, int, int], x, kv: Optional[int],
     import torch
     _check(lib().vt_decode_step(part, vt_shard(*shard), _ptr(x, torch.float16), kv or None,
                                 _ptr(out_partial, torch.float32), _stream(stream)))
+
+
+def vt_decode_step_static(part: int, shard: Tuple[int, int, int], x, kv: Optional[int], out_partial,
+                          stream=None) -> None:
+    """ATTN-shard decode step that allocates nothing: every intermediate is in the library's
+    fixed 1 MiB device array (for callers that cannot allocate device memory while decoding).
+    Calls in flight at once race on that array; the first call on a device looks its address up
+    and should come before any stream capture."""
+    import torch
+    _check(lib().vt_decode_step_static(part, vt_shard(*shard), _ptr(x, torch.float16), kv or None,
+                                       _ptr(out_partial, torch.float32), _stream(stream)))
 
 
 def vt_prefill(part: int, shard: Tuple[int, int, int], x, n: int, kv: Optional[int], out_partial,
