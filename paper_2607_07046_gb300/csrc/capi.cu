@@ -574,7 +574,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         ds.attn = b.take<float>((size_t)std::max(hq, 1) * dh);
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
         p->max_hq = std::max(p->max_hq, hq);
-        p->max_ld = std::max(p->max_ld, round_up8(c));
+        p->max_ld = std::max(p->max_ld, round_up8(c + cols[d].begin % 8));
         (void)hk;
     }
     // ------------------------------------------------------------------ stack + prefill scratch
@@ -1064,16 +1064,19 @@ static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half*
             VT_CUDA(launch_fill_zero_f32(out, (int64_t)n * D, st));
             return VT_OK;
         }
+        if (s.d_ffn % 8 != 0) return fail(VT_ERR_SHAPE, "prefill needs d_ffn to be a multiple of 8");
         PrefillFfnArgs t{};
         t.n = n;
         t.d = D;
         t.c = c;
-        t.ld_down = s.d_model;
         t.eps = s.rms_eps;
         t.x = x;
         t.gain = f.norm;
         t.wgu = f.wgu;
-        t.wd = f.wdt;
+        t.ushift = f.c0 % 8;
+        t.wd = p->m->layer[sh.layer].w_down + (f.c0 - t.ushift);
+        t.wd_ld = s.d_ffn;
+        t.ldu = p->max_ld;
         t.xhat = p->p_xhat;
         t.u = p->p_u;
         t.out = out;

@@ -159,14 +159,20 @@ struct PrefillAttnArgs {
 };
 struct PrefillFfnArgs {
     int n, d, c;            // rows, d_model, shard columns
-    int ld_down;            // row stride of the down slice (c rounded up to 8)
     float eps;
     const __half* x;        // [n][d]
     const __half* gain;
     const __half* wgu;      // [2c][d], gate/up rows interleaved
-    const __half* wd;       // [d][ld_down]
+    // Down projection, read in place from the model's Wd [d][F]: wd points at column c0 - ushift
+    // (rounded down to a multiple of 8 so the operand starts on a 16-byte boundary), row stride
+    // wd_ld = F.  U carries the same shift: column ushift + j of U is shard column j, columns
+    // [0, ushift) are zero, so the extra Wd columns contribute nothing.
+    const __half* wd;
+    int64_t wd_ld;
+    int ushift;
+    int ldu;                // row stride of u (>= ushift + c, multiple of 8)
     __half* xhat;           // [n][d]
-    __half* u;              // [n][ld_down]
+    __half* u;              // [n][ldu]
     float* out;             // [n][d]
     uint32_t* status;
 };

@@ -1,18 +1,695 @@
-// Prefill-path kernels (dense prompt): placeholder until the tensor-core path lands.
+// Prefill-path kernels for one tensor-parallel shard (n prompt rows), sm_103a.
+//
+// What they compute (Voltron Section 2.1, prefill phase, per shard as in Section 3.2.1): the same
+// steps as decode, for n rows at positions p0 .. p0 + n - 1 (p0 = cached length of the layer):
+//   ATTN shard: X^ = RMSNorm(X); [Q;K;V] = X^ . Wqkv_s^T; RoPE on Q and K; K, V appended to the
+//               cache; causal attention (row i sees positions 0 .. p0 + i); partial = A . Wo_s^T.
+//   FFN shard:  X^ = RMSNorm(X); U = silu(X^ Wg_s^T) * (X^ Wu_s^T); partial = U . Wd_s^T.
+// The projections are dense contractions and run on the tensor cores (tcgen05.mma, accumulator
+// in tensor memory, operands staged by TMA); X^, Q, the attention output and U are fp16 operands,
+// accumulation and partials are fp32.
+//
+//   k_rmsnorm_rows   one CTA per row
+//   k_gemm           C = A . B^T, A [M][K] and B [N][K] fp16 (K contiguous), one 128 x 256 output
+//                    tile per CTA; epilogues: fp32 store, RoPE + q store + KV append, SwiGLU
+//   k_prefill_attn   causal flash attention, 64 query rows of one head per CTA (mma.sync)
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "device.cuh"
 #include "internal.h"
 
 namespace vt {
 
-cudaError_t init_prefill_kernels() { return cudaSuccess; }
+// ================================================================== tcgen05 / TMA primitives
 
-vt_status prefill_attn_shard(const PrefillAttnArgs&, cudaStream_t, std::string* err) {
-    *err = "prefill is not available in this build";
-    return VT_ERR_STATE;
+namespace tc {
+
+// 2-D tiled TMA load of box (x = inner coordinate in elements, y = row) into shared memory,
+// completing as transaction bytes on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
 }
 
-vt_status prefill_ffn_shard(const PrefillFfnArgs&, cudaStream_t, std::string* err) {
-    *err = "prefill is not available in this build";
-    return VT_ERR_STATE;
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D (tensor memory) (+)= A (shared, descriptor) . B (shared, descriptor), fp16 inputs, fp32 accumulate
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                        uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrives once on `bar` when every MMA this thread issued so far has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+// 32 lanes x 32 consecutive columns of 32-bit data: thread t of the warp gets lane (base + t).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Shared-memory matrix descriptor of a K-major operand tile written by TMA with the 128-byte
+// swizzle: rows of 64 fp16 (128 bytes), 8-row groups 1024 bytes apart.  The tile base is 1024-byte
+// aligned; stepping K by 16 elements inside the 128-byte row advances the start address by 32 bytes.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+    d |= (uint64_t)1 << 16;                    // leading-dimension offset (unused with this swizzle)
+    d |= (uint64_t)(1024 >> 4) << 32;          // stride between 8-row groups
+    d |= (uint64_t)1 << 46;                    // descriptor version
+    d |= (uint64_t)2 << 61;                    // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor: fp16 A and B (both K-major), fp32 accumulator, M x N.
+__host__ __device__ constexpr uint32_t idesc_f16(int m, int n) {
+    return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+}  // namespace tc
+
+// ================================================================== RMSNorm rows
+
+__global__ void __launch_bounds__(256) k_rmsnorm_rows(const __half* __restrict__ x, const __half* __restrict__ gain,
+                                                      float eps, int d, __half* __restrict__ y) {
+    __shared__ float red[8];
+    pdl_wait();
+    const __half* xr = x + (size_t)blockIdx.x * d;
+    __half* yr = y + (size_t)blockIdx.x * d;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+        const uint4 v = *reinterpret_cast<const uint4*>(xr + c * 8);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = h2_to_f2(w[e]);
+            ss = fmaf(f.x, f.x, ss);
+            ss = fmaf(f.y, f.y, ss);
+        }
+    }
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+    const float r = 1.0f / sqrtf(tot / (float)d + eps);
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+        const uint4 v = *reinterpret_cast<const uint4*>(xr + c * 8);
+        const uint4 g = *reinterpret_cast<const uint4*>(gain + c * 8);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w}, gw[4] = {g.x, g.y, g.z, g.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = h2_to_f2(w[e]), gg = h2_to_f2(gw[e]);
+            const __half2 h = __floats2half2_rn(f.x * r * gg.x, f.y * r * gg.y);
+            o[e] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        *reinterpret_cast<uint4*>(yr + c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+// ================================================================== tensor-core GEMM
+
+constexpr int kBM = 128, kBK = 64, kBN = 256, kStages = 4;
+constexpr int kGemmThreads = 192;  // warp 0: TMA, warp 1: MMA + tensor memory, warps 2-5: epilogue
+constexpr int kABytes = kBM * kBK * 2, kBBytes = kBN * kBK * 2, kStageBytes = kABytes + kBBytes;
+constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
+
+enum GemmEpi : int { kGemmF32 = 0, kGemmQkv = 1, kGemmSwiglu = 2 };
+
+struct GemmArgs {
+    int m, n, k_tiles;
+    // kGemmF32: c[row][col], row stride ldc
+    float* c;
+    int ldc;
+    // kGemmQkv: columns are head blocks of dh in RoPE-pair order (q heads, k heads, v heads)
+    __half* q;  // [m][hq][dh]
+    __half* kcache;
+    __half* vcache;
+    int hq, hk, dh, cap;
+    const int32_t* len;  // rows sit at positions *len + row_offset + row
+    int row_offset;
+    const float2* rope;
+    // kGemmSwiglu: columns (gate j, up j) interleaved; u[row][ushift + j], zeros in [0, ushift)
+    __half* u;
+    int ldu, ushift;
+    uint32_t* status;
+};
+
+template <int EPI>
+__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, int row, int col, const float (&v)[32],
+                                                    int pos) {
+    if constexpr (EPI == kGemmF32) {
+        float* dst = a.c + (size_t)row * a.ldc + col;
+        if (col + 32 <= a.n) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+                *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+        } else {
+            for (int j = 0; j < 32 && col + j < a.n; ++j) dst[j] = v[j];
+        }
+    } else if constexpr (EPI == kGemmQkv) {
+        if (col >= a.n) return;
+        const int dh = a.dh, half = dh / 2;
+        const int b = col / dh, i0 = (col % dh) / 2;  // head block; first pair of this chunk
+        __half lo[16], hi[16];
+        if (b < a.hq + a.hk) {
+            const float2* cs = a.rope + (size_t)pos * half + i0;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float2 r = cs[j];
+                const float x0 = v[2 * j], x1 = v[2 * j + 1];
+                lo[j] = __float2half_rn(x0 * r.x - x1 * r.y);
+                hi[j] = __float2half_rn(x0 * r.y + x1 * r.x);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                lo[j] = __float2half_rn(v[2 * j]);
+                hi[j] = __float2half_rn(v[2 * j + 1]);
+            }
+        }
+        __half* dst;
+        if (b < a.hq) dst = a.q + ((size_t)row * a.hq + b) * dh;
+        else if (b < a.hq + a.hk) dst = a.kcache + ((size_t)(b - a.hq) * a.cap + pos) * dh;
+        else dst = a.vcache + ((size_t)(b - a.hq - a.hk) * a.cap + pos) * dh;
+        const uint4* l4 = reinterpret_cast<const uint4*>(lo);
+        const uint4* h4 = reinterpret_cast<const uint4*>(hi);
+        uint4* d_lo = reinterpret_cast<uint4*>(dst + i0);
+        uint4* d_hi = reinterpret_cast<uint4*>(dst + i0 + half);
+        d_lo[0] = l4[0];
+        d_lo[1] = l4[1];
+        d_hi[0] = h4[0];
+        d_hi[1] = h4[1];
+    } else {
+        if (col >= a.n) return;
+        __half* dst = a.u + (size_t)row * a.ldu + a.ushift + col / 2;
+        if (col == 0)
+            for (int j = 0; j < a.ushift; ++j) dst[j - a.ushift] = __float2half_rn(0.f);
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+            if (col + 2 * j < a.n) dst[j] = __float2half_rn(silu(v[2 * j]) * v[2 * j + 1]);
+    }
+}
+
+// One 128 x 256 tile of C = A . B^T per CTA.  A k-tile is 64 columns of K: TMA brings the A and B
+// boxes (128-byte swizzle) into one of kStages stages; the MMA thread issues four 128 x 256 x 16
+// MMAs per stage into one tensor-memory accumulator (256 columns) and releases the stage through
+// tcgen05.commit; after the last k-tile the epilogue warps read the accumulator row by row
+// (warp w reads lanes 32 (w % 4) ..) and apply the epilogue.  Rows >= m and columns >= n come
+// from TMA's zero fill and are not stored.  Every wait is bounded; on a timeout the kernel sets
+// VT_DEV_WAIT_TIMEOUT, stops issuing, waits for the copies it issued, frees tensor memory and ends.
+template <int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, const __grid_constant__ GemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+    uint64_t* empty = full + kStages;
+    uint64_t* done = empty + kStages;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+    __shared__ int s_err;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * kBN, m0 = blockIdx.y * kBM;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(done, 1);
+        s_err = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(tmem_slot, kBN);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = *tmem_slot;
+    pdl_wait();  // A was written by the preceding kernel
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int issued = 0;
+            for (int i = 0; i < a.k_tiles; ++i) {
+                const int s = i % kStages;
+                if (i >= kStages && !mbar_wait(&empty[s], ((i / kStages) - 1) & 1)) {
+                    s_err = 1;
+                    set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+                    break;
+                }
+                if (*(volatile int*)&s_err) break;
+                uint8_t* st = smem + s * kStageBytes;
+                mbar_arrive_expect_tx(&full[s], kStageBytes);
+                tc::tma_load_2d(st, &ta, i * kBK, m0, &full[s]);
+                tc::tma_load_2d(st + kABytes, &tb, i * kBK, n0, &full[s]);
+                issued = i + 1;
+            }
+            // no copy may still be in flight when the CTA ends
+            for (int i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
+                if (!mbar_wait(&full[i % kStages], (i / kStages) & 1)) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_f16(kBM, kBN);
+            for (int i = 0; i < a.k_tiles; ++i) {
+                const int s = i % kStages;
+                if (!mbar_wait(&full[s], (i / kStages) & 1)) {
+                    s_err = 1;
+                    set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+                    break;
+                }
+                tc::fence_after();
+                const uint32_t sa = smem_u32(smem + s * kStageBytes), sb = sa + kABytes;
+#pragma unroll
+                for (int k = 0; k < kBK / 16; ++k)
+                    tc::mma_f16(tmem, tc::desc_sw128(sa + k * 32), tc::desc_sw128(sb + k * 32), idesc,
+                                (i | k) != 0);
+                tc::mma_commit(&empty[s]);
+            }
+            tc::mma_commit(done);
+        }
+    } else {
+        const int sub = warp & 3;  // tensor-memory lanes 32 sub .. 32 sub + 31
+        bool ok = mbar_wait(done, 0);
+        if (!ok) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+        // tcgen05.ld is warp-collective: the whole warp reads the accumulator or none of it
+        ok = __all_sync(0xffffffffu, ok && !*(volatile int*)&s_err);
+        tc::fence_after();
+        const int row = m0 + sub * 32 + lane;
+        int pos = 0;
+        bool row_ok = row < a.m;
+        if constexpr (EPI == kGemmQkv) {
+            pos = *a.len + a.row_offset + row;
+            if (row_ok && (pos < 0 || pos >= a.cap)) {
+                set_status(a.status, VT_DEV_KV_OVERFLOW);
+                row_ok = false;
+            }
+        }
+        if (ok) {
+            for (int c = 0; c < kBN; c += 32) {
+                uint32_t r[32];
+                tc::tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)c, r);
+                tc::tmem_ld_wait();
+                if (row_ok && n0 + c < a.n) {
+                    float v[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+                    gemm_epilogue_chunk<EPI>(a, row, n0 + c, v, pos);
+                }
+            }
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_dealloc(tmem, kBN);
+    }
+}
+
+// ================================================================== causal attention
+
+struct PrefillAttnKArgs {
+    const __half* q;  // [n][hq][dh]
+    const __half* kcache;
+    const __half* vcache;
+    const int32_t* len;
+    int row_offset, n, hq, group, cap;
+    float scale_log2;
+    __half* out;  // [n][hq * dh]
+};
+
+__device__ __forceinline__ void cp_async16(void* s, const void* g) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(s)), "l"(g) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
+    const __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+constexpr int kAttnRows = 64;  // query rows per CTA (16 per warp)
+constexpr int kAttnKeys = 64;  // cached positions per tile
+
+template <int DH>
+constexpr size_t prefill_attn_smem() {
+    return (size_t)4 * kAttnKeys * (DH + 8) * 2;  // K and V, two buffers each, padded rows
+}
+
+// Flash attention (online softmax) over the causal set.  Warp w owns query rows r0 + 16 w ..
+// + 15; S = Q K^T and O += P V use m16n8k16 tensor-core MMAs with fp32 accumulation; K/V tiles of
+// 64 positions are double-buffered in shared memory (rows padded by 16 bytes so the fragment
+// loads hit distinct banks).
+template <int DH>
+__global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ PrefillAttnKArgs a) {
+    constexpr int LDS = DH + 8, KC = DH / 16, DT = DH / 8;
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    __half* Ks = reinterpret_cast<__half*>(smem_raw);  // [2][64][LDS]
+    __half* Vs = Ks + 2 * kAttnKeys * LDS;              // [2][64][LDS]
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
+    const int h = blockIdx.y, j = h / a.group, r0 = blockIdx.x * kAttnRows;
+
+    pdl_wait();
+    const int P0 = *a.len + a.row_offset;
+    const int rlast = min(r0 + kAttnRows - 1, a.n - 1);
+    const int kend = min(P0 + rlast + 1, a.cap);  // positions [0, kend) are needed
+    const int nkb = (kend + kAttnKeys - 1) / kAttnKeys;
+    const __half* kbase = a.kcache + (size_t)j * a.cap * DH;
+    const __half* vbase = a.vcache + (size_t)j * a.cap * DH;
+
+    auto load_tile = [&](int kb, int buf) {
+        for (int c = tid; c < kAttnKeys * DH / 8; c += 128) {
+            const int r = c / (DH / 8), col = (c % (DH / 8)) * 8;
+            const int pos = kb * kAttnKeys + r;
+            __half* dk = Ks + (buf * kAttnKeys + r) * LDS + col;
+            __half* dv = Vs + (buf * kAttnKeys + r) * LDS + col;
+            if (pos < kend) {
+                cp_async16(dk, kbase + (size_t)pos * DH + col);
+                cp_async16(dv, vbase + (size_t)pos * DH + col);
+            } else {
+                *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
+            }
+        }
+        cp_async_commit();
+    };
+
+    const int qr0 = r0 + warp * 16;
+    uint32_t qa[KC][4];
+#pragma unroll
+    for (int kc = 0; kc < KC; ++kc)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int row = qr0 + g + (e & 1) * 8, col = kc * 16 + 2 * t + (e >> 1) * 8;
+            qa[kc][e] = row < a.n ? *reinterpret_cast<const uint32_t*>(a.q + ((size_t)row * a.hq + h) * DH + col) : 0u;
+        }
+    float o[DT][4];
+#pragma unroll
+    for (int d = 0; d < DT; ++d) o[d][0] = o[d][1] = o[d][2] = o[d][3] = 0.f;
+    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+    const int qpos[2] = {P0 + qr0 + g, P0 + qr0 + g + 8};
+    const int warp_last = P0 + qr0 + 15;
+
+    load_tile(0, 0);
+    for (int kb = 0; kb < nkb; ++kb) {
+        const int buf = kb & 1;
+        if (kb + 1 < nkb) {
+            load_tile(kb + 1, buf ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        if (kb * kAttnKeys <= warp_last) {
+            const __half* kt = Ks + buf * kAttnKeys * LDS;
+            float s[8][4];
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+                const __half* kr = kt + (nt * 8 + g) * LDS + 2 * t;
+#pragma unroll
+                for (int kc = 0; kc < KC; ++kc) {
+                    const uint32_t b0 = *reinterpret_cast<const uint32_t*>(kr + kc * 16);
+                    const uint32_t b1 = *reinterpret_cast<const uint32_t*>(kr + kc * 16 + 8);
+                    mma16816(s[nt], qa[kc], b0, b1);
+                }
+            }
+            float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int pos = kb * kAttnKeys + nt * 8 + 2 * t + (e & 1);
+                    const float v = pos <= qpos[e >> 1] ? s[nt][e] * a.scale_log2 : -INFINITY;
+                    s[nt][e] = v;
+                    mx[e >> 1] = fmaxf(mx[e >> 1], v);
+                }
+            float corr[2];
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+                const float mn = fmaxf(mrow[r], mx[r]);
+                corr[r] = mn == -INFINITY ? 1.f : exp2f(mrow[r] - mn);
+                mrow[r] = mn;
+            }
+            float ls[2] = {0.f, 0.f};
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float m = mrow[e >> 1];
+                    const float p = m == -INFINITY ? 0.f : exp2f(s[nt][e] - m);
+                    s[nt][e] = p;
+                    ls[e >> 1] += p;
+                }
+#pragma unroll
+            for (int r = 0; r < 2; ++r) lrow[r] = lrow[r] * corr[r] + ls[r];
+#pragma unroll
+            for (int d = 0; d < DT; ++d) {
+                o[d][0] *= corr[0];
+                o[d][1] *= corr[0];
+                o[d][2] *= corr[1];
+                o[d][3] *= corr[1];
+            }
+            const uint32_t vt_base = smem_u32(Vs + buf * kAttnKeys * LDS);
+#pragma unroll
+            for (int kk = 0; kk < kAttnKeys / 16; ++kk) {
+                const uint32_t pa[4] = {pack_h2(s[2 * kk][0], s[2 * kk][1]), pack_h2(s[2 * kk][2], s[2 * kk][3]),
+                                        pack_h2(s[2 * kk + 1][0], s[2 * kk + 1][1]),
+                                        pack_h2(s[2 * kk + 1][2], s[2 * kk + 1][3])};
+                const int vrow = kk * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
+#pragma unroll
+                for (int d = 0; d < DT; d += 2) {
+                    const int vcol = (d + (lane >> 4)) * 8;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4_trans(vt_base + (uint32_t)(vrow * LDS + vcol) * 2, b0, b1, b2, b3);
+                    mma16816(o[d], pa, b0, b1);
+                    mma16816(o[d + 1], pa, b2, b3);
+                }
+            }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+    }
+    const float inv[2] = {lrow[0] > 0.f ? 1.f / lrow[0] : 0.f, lrow[1] > 0.f ? 1.f / lrow[1] : 0.f};
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int row = qr0 + g + r * 8;
+        if (row >= a.n) continue;
+        __half* dst = a.out + (size_t)row * a.hq * DH + (size_t)h * DH + 2 * t;
+#pragma unroll
+        for (int d = 0; d < DT; ++d)
+            *reinterpret_cast<uint32_t*>(dst + d * 8) = pack_h2(o[d][2 * r] * inv[r], o[d][2 * r + 1] * inv[r]);
+    }
+}
+
+// ================================================================== host side
+
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t init_prefill_kernels() {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    if ((e = cudaFuncSetAttribute(k_gemm<kGemmF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_gemm<kGemmQkv>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_gemm<kGemmSwiglu>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)prefill_attn_smem<128>())) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_prefill_attn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)prefill_attn_smem<64>())) != cudaSuccess)
+        return e;
+    return cudaSuccess;
+}
+
+// K-major fp16 operand [rows][inner] with row stride `ld` elements, read in boxes of 64 x box_rows.
+static bool make_map(CUtensorMap* map, const void* base, int64_t inner, int64_t rows, int64_t ld, int box_rows,
+                     std::string* err) {
+    if (!g_encode) {
+        *err = "the tensor-map encoder is not available";
+        return false;
+    }
+    if (((uintptr_t)base & 15) != 0 || (ld * 2) % 16 != 0) {
+        *err = "a GEMM operand is not 16-byte aligned (base and row stride)";
+        return false;
+    }
+    const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                                estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+        return false;
+    }
+    return true;
+}
+
+template <int EPI>
+static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb, int m, int n, int k,
+                          const GemmArgs& base, cudaStream_t st, std::string* err) {
+    CUtensorMap ta, tb;
+    if (!make_map(&ta, A, k, m, lda, kBM, err) || !make_map(&tb, B, k, n, ldb, kBN, err)) return VT_ERR_INVALID_ARG;
+    GemmArgs a = base;
+    a.m = m;
+    a.n = n;
+    a.k_tiles = (k + kBK - 1) / kBK;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((n + kBN - 1) / kBN, (m + kBM - 1) / kBM);
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = kGemmSmem;
+    cfg.stream = st;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm<EPI>, ta, tb, a);
+    if (e != cudaSuccess) {
+        *err = std::string("GEMM launch failed: ") + cudaGetErrorString(e);
+        return VT_ERR_CUDA;
+    }
+    return VT_OK;
+}
+
+static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int n, int d, __half* y, cudaStream_t st,
+                             std::string* err) {
+    k_rmsnorm_rows<<<n, 256, 0, st>>>(x, gain, eps, d, y);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        *err = std::string("RMSNorm launch failed: ") + cudaGetErrorString(e);
+        return VT_ERR_CUDA;
+    }
+    return VT_OK;
+}
+
+vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {
+    vt_status r;
+    if ((r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
+    GemmArgs g{};
+    g.q = a.q;
+    g.kcache = a.kcache;
+    g.vcache = a.vcache;
+    g.hq = a.hq;
+    g.hk = a.hk;
+    g.dh = a.dh;
+    g.cap = a.cap;
+    g.len = a.len;
+    g.row_offset = a.row_offset;
+    g.rope = a.rope;
+    g.status = a.status;
+    if ((r = run_gemm<kGemmQkv>(a.xhat, a.d, a.wqkv, a.d, a.n, (a.hq + 2 * a.hk) * a.dh, a.d, g, st, err)) != VT_OK)
+        return r;
+
+    PrefillAttnKArgs t{};
+    t.q = a.q;
+    t.kcache = a.kcache;
+    t.vcache = a.vcache;
+    t.len = a.len;
+    t.row_offset = a.row_offset;
+    t.n = a.n;
+    t.hq = a.hq;
+    t.group = a.hq / a.hk;
+    t.cap = a.cap;
+    t.scale_log2 = a.scale_log2;
+    t.out = a.attn;
+    const dim3 grid((a.n + kAttnRows - 1) / kAttnRows, a.hq);
+    if (a.dh == 128) k_prefill_attn<128><<<grid, 128, prefill_attn_smem<128>(), st>>>(t);
+    else k_prefill_attn<64><<<grid, 128, prefill_attn_smem<64>(), st>>>(t);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        *err = std::string("prefill attention launch failed: ") + cudaGetErrorString(e);
+        return VT_ERR_CUDA;
+    }
+
+    GemmArgs o{};
+    o.c = a.out;
+    o.ldc = a.d;
+    o.status = a.status;
+    return run_gemm<kGemmF32>(a.attn, (int64_t)a.hq * a.dh, a.wo, (int64_t)a.hq * a.dh, a.n, a.d, a.hq * a.dh, o, st,
+                              err);
+}
+
+vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err) {
+    vt_status r;
+    if ((r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
+    GemmArgs g{};
+    g.u = a.u;
+    g.ldu = a.ldu;
+    g.ushift = a.ushift;
+    g.status = a.status;
+    if ((r = run_gemm<kGemmSwiglu>(a.xhat, a.d, a.wgu, a.d, a.n, 2 * a.c, a.d, g, st, err)) != VT_OK) return r;
+    GemmArgs o{};
+    o.c = a.out;
+    o.ldc = a.d;
+    o.status = a.status;
+    // K runs over the shifted columns [0, ushift + c) of U and the same columns of Wd from wd
+    return run_gemm<kGemmF32>(a.u, a.ldu, a.wd, a.wd_ld, a.n, a.d, a.ushift + a.c, o, st, err);
 }
 
 }  // namespace vt
