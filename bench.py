@@ -7,8 +7,10 @@ is one CUDA graph (vt_decode_token captured once) replayed K times; the KV lengt
 
 Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs resident in HBM;
 `e2e` is the same metric through the C ABI with host buffers (token id H2D, hidden state D2H,
-synchronised every step); `roofline` is the decode GEMV's achieved HBM bandwidth; `cpu_baseline` is
-the CPU oracle timed on a bounded sample.  `--impl reference` times the CPU oracle alone.
+synchronised every step); `roofline` is the fused FFN kernel's achieved HBM bandwidth;
+`cpu_baseline` is the CPU oracle timed on a bounded sample; `prefill` is the 512-token prompt of the
+7B prefill workload through the same stack (tok/s and tensor-core rate).  `--impl reference` times
+the CPU oracle alone.
 """
 from __future__ import annotations
 
@@ -123,11 +125,12 @@ def ffn_gemv_bytes(wl):
 
 
 def kernels_per_token(wl):
+    """Kernels of one vt_decode_token: per layer, 3 per non-empty ATTN shard (QKV GEMV,
+    attention, O GEMV), 1 per non-empty FFN shard (fused FFN), 2 combines; 1 KV advance."""
     n = 0
-    g = wl.n_heads // wl.n_kv_heads
     for (h0, h1), (c0, c1) in zip(wl.head_ranges, wl.ffn_ranges):
-        n += 3 if h1 > h0 else 1
-        n += 2 if c1 > c0 else 1
+        n += 3 if h1 > h0 else 0
+        n += 1 if c1 > c0 else 0
     return wl.n_layers * (n + 2) + 1
 
 
@@ -151,6 +154,68 @@ def cpu_baseline_decode(wl, layers=4, tokens=2):
             "sample": f"{tokens} decode tokens through layers 0-{layers - 1} of {wl.n_layers} at KV "
                       f"{L0}, 4-way TP shards; tok/s extrapolated x{wl.n_layers / layers:g} by layers",
             "seconds": round(dt, 2)}
+
+
+def prefill_gemm_flops(wl, n):
+    """Tensor-core FLOPs of an n-row prefill through the stack: QKV, O, gate/up and down
+    projections of every shard (2 flops per multiply-add)."""
+    D, H, Hk, dh, F = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn
+    return 2 * n * wl.n_layers * (D * (H + 2 * Hk) * dh + D * H * dh + 3 * D * F)
+
+
+def prefill_attn_flops(wl, n):
+    """Causal attention of an n-row prompt from position 0: QK^T and PV over i + 1 positions."""
+    return 4 * wl.d_head * wl.n_heads * wl.n_layers * n * (n + 1) // 2
+
+
+def run_prefill(vt, st, wl, stream, steps, warmup):
+    """The 512-token prompt of the 7B prefill workload through every layer (vt_prefill_tokens,
+    shards one after another), captured with the embedding and a KV rewind as one CUDA graph."""
+    import torch
+    wp = synthetic.WORKLOADS[4]
+    n, D = wp.prompt_len, wl.d_model
+    ids = torch.from_numpy(wp.token_ids(n, stream=3)).cuda()
+    x = torch.empty((n, D), dtype=torch.float16, device="cuda")
+    y = torch.empty((n, D), dtype=torch.float16, device="cuda")
+    vt.vt_kv_set_length(st.kv, -1, 0, stream)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(g, stream=stream):
+            vt.vt_embed(st.model, ids, x, stream)
+            vt.vt_prefill_tokens(st.part, st.kv, x, n, y, stream)
+            vt.vt_kv_advance(st.kv, -1, -n, stream)
+        for _ in range(warmup):
+            g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            g.replay()
+        e1.record(stream)
+    e1.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    finite = bool(torch.isfinite(y.float()).all().item())
+    _, _, tf_sustained, peak_kind = measured_peaks()
+    gemm = prefill_gemm_flops(wl, n)
+    tflops = gemm / (ms * 1e-3) / 1e12
+    n_dev = len(wl.head_ranges)
+    # kernels per prompt: embedding, the first RMSNorm, per layer (per ATTN shard: QKV GEMM,
+    # attention, O GEMM; combine + RMSNorm; per FFN shard: gate/up GEMM, down GEMM; combine +
+    # RMSNorm), KV advance and rewind
+    launches = 2 + wl.n_layers * (3 * n_dev + 1 + 2 * n_dev + 1) + 2
+    return {
+        "workload": f"llama2-7b-shaped prefill: {n}-token prompt (seeded ids, embedding gather), "
+                    f"{wl.n_layers} layers, even {n_dev}-way TP, shards one after another on 1 GPU",
+        "value": round(n / (ms * 1e-3), 1), "unit": "tok/s", "ms_per_prompt": round(ms, 4),
+        "steps": steps, "warmup": warmup,
+        "gemm_tflop_per_prompt": round(gemm / 1e12, 4),
+        "attn_gflop_per_prompt": round(prefill_attn_flops(wl, n) / 1e9, 2),
+        "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": tf_sustained,
+                     "unit": "TFLOP/s", "frac": round(tflops / tf_sustained, 4),
+                     "peak_kind": f"{peak_kind} sustained bf16 dense (fp16 dense has the same nominal rate)",
+                     "note": "GEMM FLOPs over the whole prompt time (RMSNorm, attention, combines "
+                             "included): a lower bound on the GEMM kernels' own rate"},
+        "gpu_launches": launches * steps, "finite": finite,
+    }
 
 
 def run_decode(args, rank, world):
@@ -285,7 +350,8 @@ def run_decode(args, rank, world):
             f1.record(stream)
         f1.synchronize()
         ffn_ms = f0.elapsed_time(f1) / reps
-        launches_ffn = wl.n_layers * st.n_devices * 2
+        launches_ffn = wl.n_layers * st.n_devices
+        prefill = run_prefill(vt, st, wl, stream, args.prefill_steps, 3) if args.prefill_steps > 0 else None
     finally:
         torch.cuda.synchronize()
         st.close()
@@ -323,8 +389,9 @@ def run_decode(args, rank, world):
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": "k_gemv (decode GEMV: gate/up + SwiGLU and down epilogues), FFN shard steps of "
-                      "32 layers x 4 shards replayed as one graph",
+            "kernel": "k_ffn (fused FFN shard: RMSNorm, gate/up GEMV + SwiGLU, down GEMV with bulk "
+                      "reduce-add), one launch per FFN shard step; 32 layers x 4 shards replayed as one "
+                      "graph (each step also clears its partial: a 16 KB fill kernel, timed with it)",
             "achieved": round(achieved, 1),
             "peak": hbm,
             "unit": "GB/s",
@@ -346,6 +413,9 @@ def run_decode(args, rank, world):
         "device_status": {"kv": kv_status, "partition": part_status},
         "setup_s": round(setup_s, 1),
     }
+    if prefill is not None:
+        line["prefill"] = prefill
+        line["gpu_launches"] += prefill["gpu_launches"]
     return line, clk.summary()
 
 
@@ -388,6 +458,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--prefill-steps", type=int, default=20,
+                    help="timed 512-token prefills after the decode measurement (0: skip)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: only the first N layers of the stack")
     args = ap.parse_args()

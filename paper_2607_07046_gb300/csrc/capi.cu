@@ -1020,8 +1020,10 @@ extern "C" vt_status vt_combine(const float* const* partials, int32_t n, int32_t
 
 // ------------------------------------------------------------------ prefill
 
+// xhat_ready: the partition's xhat scratch already holds RMSNorm(x) with this block's gain (the
+// whole-stack path computes it once per block, in the combine that produced x).
 static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half* x, int n, vt_kv* kv,
-                               float* out, int row_offset, cudaStream_t st) {
+                               float* out, int row_offset, cudaStream_t st, bool xhat_ready = false) {
     const vt_shapes& s = p->m->s;
     const int D = s.d_model;
     std::string err;
@@ -1051,6 +1053,7 @@ static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half*
         t.row_offset = row_offset;
         t.rope = p->m->rope;
         t.xhat = p->p_xhat;
+        t.xhat_ready = xhat_ready;
         t.q = p->p_q;
         t.attn = p->p_attn;
         t.out = out;
@@ -1078,6 +1081,7 @@ static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half*
         t.wd_ld = s.d_ffn;
         t.ldu = p->max_ld;
         t.xhat = p->p_xhat;
+        t.xhat_ready = xhat_ready;
         t.u = p->p_u;
         t.out = out;
         t.status = p->status;
@@ -1182,24 +1186,29 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
         c.count = (int64_t)rows * D;
         for (int d = 0; d < nd; ++d) c.parts[d] = p->partials + (size_t)d * kPrefillChunk * D;
         const __half* cur = static_cast<const __half*>(x_in) + (size_t)r0 * D;
+        // Every shard of a block normalises the same input with the same gain: the norm runs once
+        // per block, fused into the combine that produced the block's input.
+        VT_CUDA(launch_rmsnorm_rows(cur, p->m->layer[0].attn_norm, s.rms_eps, rows, D, p->p_xhat, st));
         for (int l = 0; l < s.n_layers; ++l) {
             for (int d = 0; d < nd; ++d) {
                 vt_shard sh{l, d, VT_BLOCK_ATTN};
                 VT_TRY(prefill_shard(p, sh, cur, rows, kv, p->partials + (size_t)d * kPrefillChunk * D,
-                                     r0, st));
+                                     r0, st, true));
             }
             c.residual = cur;
             c.out = p->hbuf;
-            VT_CUDA(launch_combine(c, st));
+            VT_CUDA(launch_combine_norm(c, rows, D, p->m->layer[l].ffn_norm, s.rms_eps, p->p_xhat, st));
             for (int d = 0; d < nd; ++d) {
                 vt_shard sh{l, d, VT_BLOCK_FFN};
                 VT_TRY(prefill_shard(p, sh, p->hbuf, rows, kv,
-                                     p->partials + (size_t)d * kPrefillChunk * D, r0, st));
+                                     p->partials + (size_t)d * kPrefillChunk * D, r0, st, true));
             }
-            __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) + (size_t)r0 * D : p->xbuf;
+            const bool last = l == s.n_layers - 1;
+            __half* dst = last ? static_cast<__half*>(x_out) + (size_t)r0 * D : p->xbuf;
             c.residual = p->hbuf;
             c.out = dst;
-            VT_CUDA(launch_combine(c, st));
+            VT_CUDA(launch_combine_norm(c, rows, D, last ? nullptr : p->m->layer[l + 1].attn_norm, s.rms_eps,
+                                        p->p_xhat, st));
             cur = dst;
         }
     }

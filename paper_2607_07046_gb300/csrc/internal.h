@@ -152,6 +152,7 @@ struct PrefillAttnArgs {
     const float2* rope;     // [max_seq][dh/2]
     // scratch
     __half* xhat;           // [n][d]
+    int xhat_ready;         // 1: xhat already holds RMSNorm(x) with this gain (skip the norm)
     __half* q;              // [n][hq][dh]
     __half* attn;           // [n][hq * dh]
     float* out;             // [n][d] partial
@@ -172,11 +173,17 @@ struct PrefillFfnArgs {
     int ushift;
     int ldu;                // row stride of u (>= ushift + c, multiple of 8)
     __half* xhat;           // [n][d]
+    int xhat_ready;         // as PrefillAttnArgs::xhat_ready
     __half* u;              // [n][ldu]
     float* out;             // [n][d]
     uint32_t* status;
 };
 vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err);
+// rows x d: out = fp16(residual + sum of partials); with gain, also xhat = RMSNorm(out) * gain
+cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __half* gain, float eps, __half* xhat,
+                                cudaStream_t st);
+cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
+                                cudaStream_t st);
 
 // ------------------------------------------------------------------ static-scratch decode attention
 // (static_scratch.cu) split-K decode attention whose scratch is one file-scope __device__ array.

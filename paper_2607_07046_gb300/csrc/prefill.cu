@@ -41,6 +41,18 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+// Pulls the box at (x, y) into L2 without writing shared memory.
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map), "r"(x), "r"(y)
+                 : "memory");
+}
+
+// 16-byte store into the shared memory of a CTA of the cluster (address from mapa).
+__device__ __forceinline__ void dsmem_st4(uint32_t addr, float a, float b, float c, float d) {
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+                 : "memory");
+}
+
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
                  : "memory");
@@ -143,6 +155,86 @@ __global__ void __launch_bounds__(256) k_rmsnorm_rows(const __half* __restrict__
     }
 }
 
+// ================================================================== combine + RMSNorm rows
+
+// One CTA per row: out = fp16(residual + sum_s parts[s]) (fp32, shards in order, as k_combine),
+// and, when gain is set, xhat = fp16(RMSNorm(out) * gain) computed from the rounded row: the input
+// every shard of the next block would normalise for itself.
+__global__ void __launch_bounds__(256) k_combine_norm(const __grid_constant__ CombineArgs a, int d,
+                                                      const __half* __restrict__ gain, float eps,
+                                                      __half* __restrict__ xhat) {
+    __shared__ float red[8];
+    pdl_wait();
+    const size_t row = blockIdx.x;
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+        const size_t e0 = row * d + (size_t)c * 8;
+        float acc[8];
+        if (a.residual) {
+            const uint4 r = *reinterpret_cast<const uint4*>(a.residual + e0);
+            const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 f = h2_to_f2(w[j]);
+                acc[2 * j] = f.x;
+                acc[2 * j + 1] = f.y;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] = 0.f;
+        }
+        for (int sh = 0; sh < a.n; ++sh) {
+            if (!a.parts[sh]) continue;
+            const float4 p0 = __ldcg(reinterpret_cast<const float4*>(a.parts[sh] + e0));
+            const float4 p1 = __ldcg(reinterpret_cast<const float4*>(a.parts[sh] + e0 + 4));
+            acc[0] += p0.x; acc[1] += p0.y; acc[2] += p0.z; acc[3] += p0.w;
+            acc[4] += p1.x; acc[5] += p1.y; acc[6] += p1.z; acc[7] += p1.w;
+        }
+        uint32_t o[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const __half2 h = __floats2half2_rn(acc[2 * j], acc[2 * j + 1]);
+            o[j] = *reinterpret_cast<const uint32_t*>(&h);
+            const float2 f = __half22float2(h);
+            ss = fmaf(f.x, f.x, ss);
+            ss = fmaf(f.y, f.y, ss);
+        }
+        *reinterpret_cast<uint4*>(a.out + e0) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+    if (!gain) return;
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+    const float r = 1.0f / sqrtf(tot / (float)d + eps);
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+        // this thread's own row elements, written above
+        const uint4 hv = *reinterpret_cast<const uint4*>(a.out + row * d + (size_t)c * 8);
+        const uint4 g = *reinterpret_cast<const uint4*>(gain + c * 8);
+        const uint32_t w[4] = {hv.x, hv.y, hv.z, hv.w}, gw[4] = {g.x, g.y, g.z, g.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 f = h2_to_f2(w[j]), gg = h2_to_f2(gw[j]);
+            const __half2 h = __floats2half2_rn(f.x * r * gg.x, f.y * r * gg.y);
+            o[j] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        *reinterpret_cast<uint4*>(xhat + row * d + (size_t)c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __half* gain, float eps, __half* xhat,
+                                cudaStream_t st) {
+    if (rows <= 0) return cudaSuccess;
+    if (d % 8 != 0 || d > 16384) return cudaErrorInvalidValue;
+    k_combine_norm<<<rows, 256, 0, st>>>(a, d, gain, eps, xhat);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
+                                cudaStream_t st);
+
 // ================================================================== tensor-core GEMM
 
 constexpr int kBM = 128, kBK = 64, kBN = 256, kStages = 4;
@@ -154,6 +246,8 @@ enum GemmEpi : int { kGemmF32 = 0, kGemmQkv = 1, kGemmSwiglu = 2 };
 
 struct GemmArgs {
     int m, n, k_tiles;
+    const __half* b;  // B [n][ldb] (prefetched into L2 by the epilogue warps while they wait)
+    int64_t ldb;
     // kGemmF32: c[row][col], row stride ldc
     float* c;
     int ldc;
@@ -171,69 +265,66 @@ struct GemmArgs {
     uint32_t* status;
 };
 
+// 16-byte slot of the split-K receive buffer that holds floats [4e, 4e + 4) of 32-column chunk
+// `chunk` of local row `lr`.  128-bit shared accesses are served 8 threads at a time; the slot
+// permutation keeps those 8 threads on distinct banks both for the writer (8 consecutive rows, one
+// chunk) and for the reader (one row, 8 consecutive chunks).
+__device__ __forceinline__ int recv_slot(int chunk, int e, int lr) { return chunk * 8 + (e ^ ((chunk + lr) & 7)); }
+
+// Epilogue of 4 consecutive columns [col, col + 4) of one output row (col a multiple of 4).
 template <int EPI>
-__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, int row, int col, const float (&v)[32],
-                                                    int pos) {
+__device__ __forceinline__ void gemm_epilogue_quad(const GemmArgs& a, int row, int col, float4 v, int pos) {
     if constexpr (EPI == kGemmF32) {
         float* dst = a.c + (size_t)row * a.ldc + col;
-        if (col + 32 <= a.n) {
-#pragma unroll
-            for (int j = 0; j < 32; j += 4)
-                *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+        if (col + 4 <= a.n) {
+            *reinterpret_cast<float4*>(dst) = v;
         } else {
-            for (int j = 0; j < 32 && col + j < a.n; ++j) dst[j] = v[j];
+            const float f[4] = {v.x, v.y, v.z, v.w};
+            for (int j = 0; j < 4 && col + j < a.n; ++j) dst[j] = f[j];
         }
     } else if constexpr (EPI == kGemmQkv) {
-        if (col >= a.n) return;
+        // columns (col, col + 1) and (col + 2, col + 3): RoPE pairs (i, i + dh/2) and (i + 1, ...)
         const int dh = a.dh, half = dh / 2;
-        const int b = col / dh, i0 = (col % dh) / 2;  // head block; first pair of this chunk
-        __half lo[16], hi[16];
+        const int b = col / dh, i = (col % dh) / 2;
+        float l0 = v.x, h0 = v.y, l1 = v.z, h1 = v.w;
         if (b < a.hq + a.hk) {
-            const float2* cs = a.rope + (size_t)pos * half + i0;
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const float2 r = cs[j];
-                const float x0 = v[2 * j], x1 = v[2 * j + 1];
-                lo[j] = __float2half_rn(x0 * r.x - x1 * r.y);
-                hi[j] = __float2half_rn(x0 * r.y + x1 * r.x);
-            }
-        } else {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                lo[j] = __float2half_rn(v[2 * j]);
-                hi[j] = __float2half_rn(v[2 * j + 1]);
-            }
+            const float4 cs = *reinterpret_cast<const float4*>(a.rope + (size_t)pos * half + i);
+            l0 = v.x * cs.x - v.y * cs.y;
+            h0 = v.x * cs.y + v.y * cs.x;
+            l1 = v.z * cs.z - v.w * cs.w;
+            h1 = v.z * cs.w + v.w * cs.z;
         }
         __half* dst;
         if (b < a.hq) dst = a.q + ((size_t)row * a.hq + b) * dh;
         else if (b < a.hq + a.hk) dst = a.kcache + ((size_t)(b - a.hq) * a.cap + pos) * dh;
         else dst = a.vcache + ((size_t)(b - a.hq - a.hk) * a.cap + pos) * dh;
-        const uint4* l4 = reinterpret_cast<const uint4*>(lo);
-        const uint4* h4 = reinterpret_cast<const uint4*>(hi);
-        uint4* d_lo = reinterpret_cast<uint4*>(dst + i0);
-        uint4* d_hi = reinterpret_cast<uint4*>(dst + i0 + half);
-        d_lo[0] = l4[0];
-        d_lo[1] = l4[1];
-        d_hi[0] = h4[0];
-        d_hi[1] = h4[1];
+        *reinterpret_cast<__half2*>(dst + i) = __floats2half2_rn(l0, l1);
+        *reinterpret_cast<__half2*>(dst + i + half) = __floats2half2_rn(h0, h1);
     } else {
-        if (col >= a.n) return;
+        // columns (gate, up) of intermediate columns col / 2 and col / 2 + 1
         __half* dst = a.u + (size_t)row * a.ldu + a.ushift + col / 2;
         if (col == 0)
             for (int j = 0; j < a.ushift; ++j) dst[j - a.ushift] = __float2half_rn(0.f);
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-            if (col + 2 * j < a.n) dst[j] = __float2half_rn(silu(v[2 * j]) * v[2 * j + 1]);
+        dst[0] = __float2half_rn(silu(v.x) * v.y);
+        if (col + 2 < a.n) dst[1] = __float2half_rn(silu(v.z) * v.w);
     }
 }
 
-// One 128 x 256 tile of C = A . B^T per CTA.  A k-tile is 64 columns of K: TMA brings the A and B
-// boxes (128-byte swizzle) into one of kStages stages; the MMA thread issues four 128 x 256 x 16
-// MMAs per stage into one tensor-memory accumulator (256 columns) and releases the stage through
-// tcgen05.commit; after the last k-tile the epilogue warps read the accumulator row by row
-// (warp w reads lanes 32 (w % 4) ..) and apply the epilogue.  Rows >= m and columns >= n come
-// from TMA's zero fill and are not stored.  Every wait is bounded; on a timeout the kernel sets
-// VT_DEV_WAIT_TIMEOUT, stops issuing, waits for the copies it issued, frees tensor memory and ends.
+// One 128 x 256 tile of C = A . B^T per CTA, or per cluster of S CTAs that split K.
+// A k-tile is 64 columns of K: TMA brings the A and B boxes (128-byte swizzle) into one of kStages
+// stages; the MMA thread issues four 128 x 256 x 16 MMAs per stage into one tensor-memory
+// accumulator (256 columns) and releases the stage through tcgen05.commit.  The CTA's B boxes are
+// first requested into L2 with TMA prefetches (the weights do not depend on the preceding kernel,
+// so this starts before griddepcontrol.wait), which hides the HBM latency the 4-stage ring cannot.
+//
+// Split K (gridDim.z = S > 1, one thread-block cluster per output tile): every CTA accumulates
+// k-tiles [k_tiles z / S, k_tiles (z + 1) / S).  After the last MMA of every CTA (cluster barrier),
+// the accumulators are reduce-scattered through distributed shared memory: tile row r belongs to
+// CTA r / ceil(128 / S), which receives every CTA's fp32 values of its rows into its (now free)
+// stage memory, adds the S contributions in rank order (so results do not depend on timing) and
+// runs the epilogue.  Rows >= m and columns >= n come from TMA's zero fill and are not stored.
+// Every wait is bounded; on a timeout the kernel sets VT_DEV_WAIT_TIMEOUT, stops issuing, waits
+// for the copies it issued, still reaches both cluster barriers, frees tensor memory and ends.
 template <int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, const __grid_constant__ GemmArgs a) {
@@ -247,6 +338,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n0 = blockIdx.x * kBN, m0 = blockIdx.y * kBM;
+    const int S = gridDim.z, z = blockIdx.z;
+    const int kt0 = (int)((int64_t)a.k_tiles * z / S), kt1 = (int)((int64_t)a.k_tiles * (z + 1) / S);
+    const int nk = kt1 - kt0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -267,10 +361,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t tmem = *tmem_slot;
     pdl_wait();  // A was written by the preceding kernel
 
+    bool ok = true;
     if (warp == 0) {
         if (lane == 0) {
             int issued = 0;
-            for (int i = 0; i < a.k_tiles; ++i) {
+            for (int i = 0; i < nk; ++i) {
                 const int s = i % kStages;
                 if (i >= kStages && !mbar_wait(&empty[s], ((i / kStages) - 1) & 1)) {
                     s_err = 1;
@@ -280,18 +375,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (*(volatile int*)&s_err) break;
                 uint8_t* st = smem + s * kStageBytes;
                 mbar_arrive_expect_tx(&full[s], kStageBytes);
-                tc::tma_load_2d(st, &ta, i * kBK, m0, &full[s]);
-                tc::tma_load_2d(st + kABytes, &tb, i * kBK, n0, &full[s]);
+                tc::tma_load_2d(st, &ta, (kt0 + i) * kBK, m0, &full[s]);
+                tc::tma_load_2d(st + kABytes, &tb, (kt0 + i) * kBK, n0, &full[s]);
                 issued = i + 1;
             }
-            // no copy may still be in flight when the CTA ends
+            // no copy may still be in flight when the stage memory is reused or the CTA ends
             for (int i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
                 if (!mbar_wait(&full[i % kStages], (i / kStages) & 1)) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
         }
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16(kBM, kBN);
-            for (int i = 0; i < a.k_tiles; ++i) {
+            for (int i = 0; i < nk; ++i) {
                 const int s = i % kStages;
                 if (!mbar_wait(&full[s], (i / kStages) & 1)) {
                     s_err = 1;
@@ -309,33 +404,89 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tc::mma_commit(done);
         }
     } else {
-        const int sub = warp & 3;  // tensor-memory lanes 32 sub .. 32 sub + 31
-        bool ok = mbar_wait(done, 0);
-        if (!ok) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+        // While the main loop runs, pull this CTA's slice of B into L2 (one prefetch per 128-byte
+        // line, k-tile by k-tile), so the TMA loads of later stages hit L2 instead of HBM.
+        {
+            const int t = threadIdx.x - 64;
+            for (int i = kt0; i < kt1; ++i)
+                for (int r = t; r < kBN; r += kGemmThreads - 64)
+                    if (n0 + r < a.n)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(a.b + (size_t)(n0 + r) * a.ldb + (size_t)i * kBK));
+        }
+        // one lane per warp polls the barrier (128 pollers would compete with the TMA and MMA
+        // threads for issue slots and shared-memory bandwidth during the whole main loop)
+        if (lane == 0) {
+            ok = mbar_wait(done, 0);
+            if (!ok) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+            ok = ok && !*(volatile int*)&s_err;
+        }
+        __syncwarp();
         // tcgen05.ld is warp-collective: the whole warp reads the accumulator or none of it
-        ok = __all_sync(0xffffffffu, ok && !*(volatile int*)&s_err);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         tc::fence_after();
-        const int row = m0 + sub * 32 + lane;
-        int pos = 0;
-        bool row_ok = row < a.m;
-        if constexpr (EPI == kGemmQkv) {
-            pos = *a.len + a.row_offset + row;
-            if (row_ok && (pos < 0 || pos >= a.cap)) {
-                set_status(a.status, VT_DEV_KV_OVERFLOW);
-                row_ok = false;
+    }
+
+    // Epilogue.  recv[slot][local row][256] (fp32, 16-byte groups permuted by recv_slot) lives in
+    // the stage memory, free once the accumulator is complete (and, with split K, once every CTA
+    // of the cluster has passed the first cluster barrier).  Tile row r belongs to CTA
+    // r / rows_per of the cluster; every CTA sends each row of its accumulator to the owner's
+    // slot `z` (its own rank), the owner adds the S slots in rank order, and each warp then writes
+    // whole rows (lane = 4 consecutive columns) so every store instruction covers 512 bytes.
+    float* recv = reinterpret_cast<float*>(smem);
+    const int rows_per = (kBM + S - 1) / S;
+    if (S > 1) cluster_sync();  // every CTA's MMAs have completed; stage memory is free everywhere
+    if (warp >= 2 && ok) {
+        const int sub = warp & 3, tr = sub * 32 + lane;  // tile row held by this thread
+        const int owner = tr / rows_per, lr = tr - owner * rows_per;
+        float* row_dst = recv + (size_t)(z * rows_per + lr) * kBN;
+        const uint32_t dst = S > 1 ? dsmem_addr(row_dst, (uint32_t)owner) : smem_u32(row_dst);
+        for (int c = 0; c < kBN; c += 32) {
+            uint32_t r[32];
+            tc::tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)c, r);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const uint32_t at = dst + (uint32_t)recv_slot(c / 32, e, lr) * 16;
+                if (S > 1)
+                    tc::dsmem_st4(at, __uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                  __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+                else
+                    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(at), "f"(__uint_as_float(r[4 * e])),
+                                 "f"(__uint_as_float(r[4 * e + 1])), "f"(__uint_as_float(r[4 * e + 2])),
+                                 "f"(__uint_as_float(r[4 * e + 3]))
+                                 : "memory");
             }
         }
-        if (ok) {
-            for (int c = 0; c < kBN; c += 32) {
-                uint32_t r[32];
-                tc::tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)c, r);
-                tc::tmem_ld_wait();
-                if (row_ok && n0 + c < a.n) {
-                    float v[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-                    gemm_epilogue_chunk<EPI>(a, row, n0 + c, v, pos);
+    }
+    if (S > 1) cluster_sync();  // every contribution has landed (all threads of every CTA)
+    else if (warp >= 2) asm volatile("bar.sync 1, %0;" ::"n"(kGemmThreads - 64) : "memory");  // the 4 epilogue warps
+    if (warp >= 2) {
+        const int r0 = z * rows_per, nr = min(kBM, r0 + rows_per) - r0;
+        int len0 = 0;
+        if constexpr (EPI == kGemmQkv) len0 = *a.len + a.row_offset;
+        for (int lr = warp - 2; lr < nr; lr += (kGemmThreads - 64) / 32) {
+            const int row = m0 + r0 + lr;
+            if (row >= a.m) break;
+            const int pos = len0 + row;
+            if constexpr (EPI == kGemmQkv) {
+                if (pos < 0 || pos >= a.cap) {
+                    if (lane == 0) set_status(a.status, VT_DEV_KV_OVERFLOW);
+                    continue;
                 }
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int f = h * 32 + lane;  // float4 index in the row
+                const int col = n0 + 4 * f;
+                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int sl = 0; sl < S; ++sl) {
+                    const uint4 x = lds128(recv + (size_t)(sl * rows_per + lr) * kBN + recv_slot(f / 8, f % 8, lr) * 4);
+                    v.x += __uint_as_float(x.x);
+                    v.y += __uint_as_float(x.y);
+                    v.z += __uint_as_float(x.z);
+                    v.w += __uint_as_float(x.w);
+                }
+                if (col < a.n) gemm_epilogue_quad<EPI>(a, row, col, v, pos);
             }
         }
     }
@@ -547,6 +698,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
 // ================================================================== host side
 
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+constexpr int kMaxSplit = 4;
+static int g_split_clusters[kMaxSplit + 1];  // co-resident clusters of S GEMM CTAs (index S)
 
 cudaError_t init_prefill_kernels() {
     void* fn = nullptr;
@@ -561,6 +714,26 @@ cudaError_t init_prefill_kernels() {
         return e;
     if ((e = cudaFuncSetAttribute(k_gemm<kGemmSwiglu>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem)) != cudaSuccess)
         return e;
+    // how many clusters of S GEMM CTAs fit at once (the split factor's wave size)
+    for (int sp = 2; sp <= kMaxSplit; ++sp) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(1, 1, sp * 64);
+        cfg.blockDim = dim3(kGemmThreads);
+        cfg.dynamicSmemBytes = kGemmSmem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 1;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = sp;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int nc = 0;
+        if (cudaOccupancyMaxActiveClusters(&nc, k_gemm<kGemmF32>, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            nc = 0;
+        }
+        g_split_clusters[sp] = nc;
+    }
     if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)prefill_attn_smem<128>())) != cudaSuccess)
         return e;
@@ -595,6 +768,27 @@ static bool make_map(CUtensorMap* map, const void* base, int64_t inner, int64_t 
     return true;
 }
 
+// Split factor for `tiles` output tiles of `k_tiles` k-tiles, from a time model of one launch:
+// per wave, a fixed cost (first loads, epilogue) plus the k-tiles of one split; with S > 1, the
+// cluster reduction of the accumulators.  The constants are measured on GB300 (microseconds).
+static int choose_split(int tiles, int k_tiles) {
+    constexpr double kTile = 0.33, kFixed = 4.0, kReduce = 3.5;
+    int best = 1;
+    double best_t = 1e30;
+    for (int s = 1; s <= kMaxSplit; ++s) {
+        if (s > 1 && k_tiles / s < 4) break;
+        const int per_wave = s == 1 ? g_num_sms : g_split_clusters[s];
+        if (per_wave < 1) continue;
+        const int waves = (tiles + per_wave - 1) / per_wave;
+        const double t = waves * (kFixed + kTile * k_tiles / s) + (s > 1 ? kReduce : 0.0);
+        if (t < best_t - 1e-9) {
+            best = s;
+            best_t = t;
+        }
+    }
+    return best;
+}
+
 template <int EPI>
 static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb, int m, int n, int k,
                           const GemmArgs& base, cudaStream_t st, std::string* err) {
@@ -603,12 +797,23 @@ static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb
     GemmArgs a = base;
     a.m = m;
     a.n = n;
+    a.b = static_cast<const __half*>(B);
+    a.ldb = ldb;
     a.k_tiles = (k + kBK - 1) / kBK;
+    const int tiles_n = (n + kBN - 1) / kBN, tiles_m = (m + kBM - 1) / kBM;
+    const int split = choose_split(tiles_n * tiles_m, a.k_tiles);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((n + kBN - 1) / kBN, (m + kBM - 1) / kBM);
+    cfg.gridDim = dim3(tiles_n, tiles_m, split);
     cfg.blockDim = dim3(kGemmThreads);
     cfg.dynamicSmemBytes = kGemmSmem;
     cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = split;
+    cfg.attrs = attr;
+    cfg.numAttrs = split > 1 ? 1 : 0;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm<EPI>, ta, tb, a);
     if (e != cudaSuccess) {
         *err = std::string("GEMM launch failed: ") + cudaGetErrorString(e);
@@ -617,10 +822,16 @@ static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb
     return VT_OK;
 }
 
+cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
+                                cudaStream_t st) {
+    if (rows <= 0) return cudaSuccess;
+    k_rmsnorm_rows<<<rows, 256, 0, st>>>(x, gain, eps, d, y);
+    return cudaGetLastError();
+}
+
 static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int n, int d, __half* y, cudaStream_t st,
                              std::string* err) {
-    k_rmsnorm_rows<<<n, 256, 0, st>>>(x, gain, eps, d, y);
-    const cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_rmsnorm_rows(x, gain, eps, n, d, y, st);
     if (e != cudaSuccess) {
         *err = std::string("RMSNorm launch failed: ") + cudaGetErrorString(e);
         return VT_ERR_CUDA;
@@ -630,7 +841,7 @@ static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int
 
 vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {
     vt_status r;
-    if ((r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
+    if (!a.xhat_ready && (r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
     GemmArgs g{};
     g.q = a.q;
     g.kcache = a.kcache;
@@ -677,7 +888,7 @@ vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::str
 
 vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err) {
     vt_status r;
-    if ((r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
+    if (!a.xhat_ready && (r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
     GemmArgs g{};
     g.u = a.u;
     g.ldu = a.ldu;
