@@ -34,6 +34,10 @@ import synthetic  # noqa: E402
 METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline"
 FALLBACK_HBM_GBS = 6800.0
 
+# DRAM bytes (read + write) of one launch of the dominant decode kernel, from one ncu capture of
+# that kernel as it is built now (profiles/k_ffn_7b_decode.md); None once the kernel changes.
+K_FFN_DRAM_BYTES_PER_LAUNCH = 67_711_488 + 159_232
+
 
 def measured_peaks():
     p = ROOT / "MEASURED_PEAKS.json"
@@ -134,25 +138,29 @@ def kernels_per_token(wl):
     return wl.n_layers * (n + 2) + 1
 
 
-def cpu_baseline_decode(wl, layers=4, tokens=2):
-    """The oracle (as it stands) on `layers` layers x `tokens` decode tokens at KV 1024; tok/s is
-    extrapolated to the full stack by the layer ratio."""
+def cpu_baseline_decode(wl, layers=4, budget_s=12.0, max_tokens=512):
+    """The oracle (as it stands) on `layers` layers, decoding teacher-forced tokens from KV 1024
+    until about `budget_s` seconds of CPU time have passed; tok/s is extrapolated to the full
+    stack by the layer ratio."""
     import oracle
     oracle.num_threads()
     L0 = wl.kv_len
     ws = [wl.layer_weights(l) for l in range(layers)]
-    caches = [wl.kv_fill(l, L0, L0 + tokens + 1) for l in range(layers)]
+    caches = [wl.kv_fill(l, L0, L0 + max_tokens + 1) for l in range(layers)]
     t0 = time.perf_counter()
-    for t in range(tokens):
-        x = wl.hidden(1, stream=500 + t)
+    tokens = 0
+    while tokens < max_tokens and (tokens < 2 or time.perf_counter() - t0 < budget_s):
+        x = wl.hidden(1, stream=500 + tokens)
         for l in range(layers):
-            _, x, _, _ = oracle.tp_layer(wl, ws[l], x, L0 + t, *caches[l])
+            _, x, _, _ = oracle.tp_layer(wl, ws[l], x, L0 + tokens, *caches[l])
+        tokens += 1
     dt = time.perf_counter() - t0
     per_token = dt / tokens * (wl.n_layers / layers)
     return {"value": round(1.0 / per_token, 4), "unit": "tok/s", "cores": oracle.num_threads(),
             "kind": "oracle",
-            "sample": f"{tokens} decode tokens through layers 0-{layers - 1} of {wl.n_layers} at KV "
-                      f"{L0}, 4-way TP shards; tok/s extrapolated x{wl.n_layers / layers:g} by layers",
+            "sample": f"{tokens} teacher-forced decode tokens through layers 0-{layers - 1} of "
+                      f"{wl.n_layers} from KV {L0}, 4-way TP shards, fp64 oracle; tok/s "
+                      f"extrapolated x{wl.n_layers / layers:g} by layers",
             "seconds": round(dt, 2)}
 
 
@@ -399,7 +407,7 @@ def run_decode(args, rank, world):
             "peak_kind": f"{peak_kind} copy bandwidth",
             "bytes_per_launch": int(ffn_bytes / launches_ffn),
             "launch_ms": round(ffn_ms / launches_ffn, 6),
-            "traffic": None,
+            "traffic": K_FFN_DRAM_BYTES_PER_LAUNCH,
         },
         "step_roofline": {
             "achieved": round(step_bytes / (ms_per_step * 1e-3) / 1e9, 1),
