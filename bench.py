@@ -2,12 +2,13 @@
 
 One step = one decode token through all 32 layers: for each layer every ATTN shard (4 of them),
 the on-device combine, every FFN shard, the combine; then the KV lengths advance.  The token step
-is one CUDA graph (vt_decode_token captured once) replayed K times; the KV length runs
-1024 -> 1151 and rewinds to 1024 every 128 steps (the 128-step schedule of the workload).
+is one CUDA graph of vt_decode_token (one fused cooperative kernel) replayed K times; the KV length
+runs 1024 -> 1151 and rewinds to 1024 every 128 steps (the 128-step schedule of the workload).
 
 Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs resident in HBM;
 `e2e` is the same metric through the C ABI with host buffers (token id H2D, hidden state D2H,
-synchronised every step); `roofline` is the fused FFN kernel's achieved HBM bandwidth;
+synchronised every step); `roofline` is the token kernel's achieved HBM bandwidth (algorithmic
+bytes of the step over its time); `sharded_token` times the same token as per-shard kernels;
 `cpu_baseline` is the CPU oracle timed on a bounded sample; `prefill` is the 512-token prompt of the
 7B prefill workload through the same stack (tok/s and tensor-core rate).  `--impl reference` times
 the CPU oracle alone.
@@ -34,9 +35,9 @@ import synthetic  # noqa: E402
 METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline"
 FALLBACK_HBM_GBS = 6800.0
 
-# DRAM bytes (read + write) of one launch of the dominant decode kernel, from one ncu capture of
-# that kernel as it is built now (profiles/k_ffn_7b_decode.md); None once the kernel changes.
-K_FFN_DRAM_BYTES_PER_LAUNCH = 67_711_488 + 159_232
+# DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
+# that kernel as it is built now; None until captured, and again once the kernel changes.
+K_TOKEN_DRAM_BYTES_PER_LAUNCH = None
 
 
 def measured_peaks():
@@ -121,11 +122,6 @@ def decode_bytes_per_token(wl, kv_mean):
     w = 2 * (D * (H + 2 * Hk) * dh + D * H * dh + 3 * D * F + 2 * D)
     kv = 2 * 2 * Hk * dh * (kv_mean + 1)
     return L * (w + kv)
-
-
-def ffn_gemv_bytes(wl):
-    D, F = wl.d_model, wl.d_ffn
-    return wl.n_layers * 2 * 3 * D * F
 
 
 def kernels_per_token(wl):
@@ -226,6 +222,53 @@ def run_prefill(vt, st, wl, stream, steps, warmup):
     }
 
 
+class TokenSchedule:
+    """Replays one decode token per step as a CUDA graph of `entry` (a whole-token entry point):
+    g_tok is one token; g_rew is one token followed by a rewind of every KV length by the
+    schedule length (the last step of each 128-step schedule 1024 -> 1151)."""
+
+    def __init__(self, vt, st, entry, xin, xout, stream, sched, kv_len):
+        import torch
+        self.vt, self.st, self.stream, self.sched, self.kv_len = vt, st, stream, sched, kv_len
+        self.g_tok, self.g_rew = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(self.g_tok, stream=stream):
+                entry(st.part, st.kv, xin, xout, stream)
+            with torch.cuda.graph(self.g_rew, stream=stream):
+                entry(st.part, st.kv, xin, xout, stream)
+                vt.vt_kv_advance(st.kv, -1, -sched, stream)
+        self.reset()
+
+    def reset(self):
+        # the captures moved the host-side length mirror; put device and host back at kv_len
+        self.vt.vt_kv_set_length(self.st.kv, -1, self.kv_len, self.stream)
+        self.pos = 0
+
+    def step(self):
+        self.pos += 1
+        if self.pos == self.sched:
+            self.g_rew.replay()
+            self.pos = 0
+        else:
+            self.g_tok.replay()
+
+
+def time_tokens(torch, sch, stream, steps, warmup):
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            sch.step()
+    stream.synchronize()
+    sch.reset()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(steps):
+            sch.step()
+        e1.record(stream)
+    e1.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
 def run_decode(args, rank, world):
     import torch
 
@@ -255,40 +298,20 @@ def run_decode(args, rank, world):
         vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
         setup_s = time.perf_counter() - t_setup
         D = wl.d_model
+        fused, why = vt.vt_decode_token_fused_available(st.part)
         ids = torch.from_numpy(wl.token_ids(1, stream=1)).cuda()
         xin = torch.empty(D, dtype=torch.float16, device="cuda")
         xout = torch.empty(D, dtype=torch.float16, device="cuda")
         with torch.cuda.stream(stream):
             vt.vt_embed(st.model, ids, xin, stream)
         stream.synchronize()
-        # One graph per token: g_tok is one vt_decode_token; g_rew is one vt_decode_token followed
-        # by a rewind of the KV lengths by 128 (the last step of each 128-step schedule).
-        g_tok, g_rew = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-        with torch.cuda.stream(stream):
-            with torch.cuda.graph(g_tok, stream=stream):
-                vt.vt_decode_token(st.part, st.kv, xin, xout, stream)
-            with torch.cuda.graph(g_rew, stream=stream):
-                vt.vt_decode_token(st.part, st.kv, xin, xout, stream)
-                vt.vt_kv_advance(st.kv, -1, -sched, stream)
-        # the captures moved the host-side length mirror; put device and host back at kv_len
-        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
-        pos = 0
-
-        def step():
-            nonlocal pos
-            pos += 1
-            if pos == sched:
-                g_rew.replay()
-                pos = 0
-            else:
-                g_tok.replay()
+        sch = TokenSchedule(vt, st, vt.vt_decode_token, xin, xout, stream, sched, wl.kv_len)
 
         with torch.cuda.stream(stream):
             for _ in range(args.warmup):
-                step()
+                sch.step()
         stream.synchronize()
-        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
-        pos = 0
+        sch.reset()
         if world > 1:
             torch.distributed.barrier()
         torch.cuda.synchronize()
@@ -297,7 +320,7 @@ def run_decode(args, rank, world):
             with torch.cuda.stream(stream):
                 e0.record(stream)
                 for _ in range(args.steps):
-                    step()
+                    sch.step()
                 e1.record(stream)
             e1.synchronize()
         torch.cuda.synchronize()
@@ -311,54 +334,38 @@ def run_decode(args, rank, world):
         part_status = vt.vt_partition_status(st.part, clear=True)
 
         # -------------------------------------------------------------- e2e through host buffers
-        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
-        pos = 0
+        sch.reset()
         ids_host = torch.from_numpy(wl.token_ids(max(args.steps, 1), stream=2)).pin_memory()
         ids_dev = torch.empty(1, dtype=torch.int32, device="cuda")
         out_host = torch.empty(D, dtype=torch.float16).pin_memory()
         e2e_steps = max(1, min(args.steps, 256))
+
+        def e2e_step(i):
+            ids_dev.copy_(ids_host[i:i + 1], non_blocking=True)
+            vt.vt_embed(st.model, ids_dev, xin, stream)
+            sch.step()
+            out_host.copy_(xout, non_blocking=True)
+            stream.synchronize()
+
         with torch.cuda.stream(stream):
             for i in range(min(3, e2e_steps)):
-                ids_dev.copy_(ids_host[i:i + 1], non_blocking=True)
-                vt.vt_embed(st.model, ids_dev, xin, stream)
-                step()
-                out_host.copy_(xout, non_blocking=True)
-                stream.synchronize()
-        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
-        pos = 0
+                e2e_step(i)
+        sch.reset()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
             for i in range(e2e_steps):
-                ids_dev.copy_(ids_host[i:i + 1], non_blocking=True)
-                vt.vt_embed(st.model, ids_dev, xin, stream)
-                step()
-                out_host.copy_(xout, non_blocking=True)
-                stream.synchronize()
+                e2e_step(i)
         e2e_s = (time.perf_counter() - t0) / e2e_steps
         e2e_finite = bool(np.isfinite(out_host.numpy().astype(np.float32)).all())
 
-        # -------------------------------------------------------------- decode GEMV roofline
-        # The FFN shard steps of every layer and shard (gate/up GEMV with SwiGLU + down GEMV) as
-        # one graph: the GEMV kernel family is the dominant cost of the token step.
-        parts = [torch.empty(D, dtype=torch.float32, device="cuda") for _ in range(st.n_devices)]
-        g2 = torch.cuda.CUDAGraph()
-        with torch.cuda.stream(stream):
-            with torch.cuda.graph(g2, stream=stream):
-                for l in range(wl.n_layers):
-                    for d in range(st.n_devices):
-                        vt.vt_decode_step(st.part, (l, d, 1), xout, None, parts[d], stream)
-            for _ in range(3):
-                g2.replay()
-            reps = max(3, min(20, args.steps // 4 + 3))
-            f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            f0.record(stream)
-            for _ in range(reps):
-                g2.replay()
-            f1.record(stream)
-        f1.synchronize()
-        ffn_ms = f0.elapsed_time(f1) / reps
-        launches_ffn = wl.n_layers * st.n_devices
+        # -------------------------------------------------------------- per-shard kernels, for context
+        sharded_ms = None
+        if args.sharded_steps > 0:
+            sch2 = TokenSchedule(vt, st, vt.vt_decode_token_sharded, xin, xout, stream, sched, wl.kv_len)
+            sharded_ms = time_tokens(torch, sch2, stream, args.sharded_steps, 3)
+            del sch2
+        sch.reset()
         prefill = run_prefill(vt, st, wl, stream, args.prefill_steps, 3) if args.prefill_steps > 0 else None
     finally:
         torch.cuda.synchronize()
@@ -368,8 +375,8 @@ def run_decode(args, rank, world):
     kv_mean = wl.kv_len + (min(args.steps, sched) - 1) / 2.0
     step_bytes = decode_bytes_per_token(wl, kv_mean)
     value = world * 1000.0 / ms_per_step
-    ffn_bytes = ffn_gemv_bytes(wl)
-    achieved = ffn_bytes / (ffn_ms * 1e-3) / 1e9
+    achieved = step_bytes / (ms_per_step * 1e-3) / 1e9
+    launches_per_token = 1 if fused else kernels_per_token(wl)
     line = {
         "metric": METRIC,
         "value": round(value, 3),
@@ -390,37 +397,37 @@ def run_decode(args, rank, world):
             "kv_len_start": wl.kv_len,
             "kv_schedule_steps": sched,
             "partition": "heads 8/8/8/8, ffn 2752 x 4",
-            "graph": "one CUDA graph per token (vt_decode_token), PDL between kernels",
+            "token_kernel": "fused: one cooperative kernel per token" if fused
+                            else f"per-shard kernels ({why})",
+            "graph": "one CUDA graph per token (vt_decode_token)",
             "l2": "no flush: the 13 GB of weights streamed per step exceed the 129 MB L2",
             "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
             "hbm_bytes_per_step": int(step_bytes),
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": "k_ffn (fused FFN shard: RMSNorm, gate/up GEMV + SwiGLU, down GEMV with bulk "
-                      "reduce-add), one launch per FFN shard step; 32 layers x 4 shards replayed as one "
-                      "graph (each step also clears its partial: a 16 KB fill kernel, timed with it)",
+            "kernel": ("k_decode_token (the whole token: every shard of every layer in one "
+                       "cooperative launch, so the kernel's launch time is the step time)") if fused
+                      else "the whole token step (per-shard kernels)",
             "achieved": round(achieved, 1),
             "peak": hbm,
             "unit": "GB/s",
             "frac": round(achieved / hbm, 4),
             "peak_kind": f"{peak_kind} copy bandwidth",
-            "bytes_per_launch": int(ffn_bytes / launches_ffn),
-            "launch_ms": round(ffn_ms / launches_ffn, 6),
-            "traffic": K_FFN_DRAM_BYTES_PER_LAUNCH,
-        },
-        "step_roofline": {
-            "achieved": round(step_bytes / (ms_per_step * 1e-3) / 1e9, 1),
-            "peak": hbm, "unit": "GB/s",
-            "frac": round(step_bytes / (ms_per_step * 1e-3) / 1e9 / hbm, 4),
-            "note": f"whole token step vs {peak_kind} HBM copy bandwidth",
+            "bytes_per_launch": int(step_bytes) if fused else None,
+            "launch_ms": round(ms_per_step, 5),
+            "traffic": K_TOKEN_DRAM_BYTES_PER_LAUNCH if fused else None,
         },
         "e2e": {"value": round(world / e2e_s, 3), "unit": "tok/s", "h2d_bytes_per_step": 4,
                 "d2h_bytes_per_step": 2 * D, "finite": e2e_finite},
-        "gpu_launches": kernels_per_token(wl) * args.steps + (args.steps // sched),
+        "gpu_launches": launches_per_token * args.steps + (args.steps // sched),
         "device_status": {"kv": kv_status, "partition": part_status},
         "setup_s": round(setup_s, 1),
     }
+    if sharded_ms is not None:
+        line["sharded_token"] = {"ms_per_step": round(sharded_ms, 5), "value": round(1000.0 / sharded_ms, 3),
+                                 "unit": "tok/s", "steps": args.sharded_steps,
+                                 "note": "vt_decode_token_sharded: per-shard kernels with PDL, for context"}
     if prefill is not None:
         line["prefill"] = prefill
         line["gpu_launches"] += prefill["gpu_launches"]
@@ -468,6 +475,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--prefill-steps", type=int, default=20,
                     help="timed 512-token prefills after the decode measurement (0: skip)")
+    ap.add_argument("--sharded-steps", type=int, default=64,
+                    help="timed tokens of the per-shard entry point, for context (0: skip)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: only the first N layers of the stack")
     args = ap.parse_args()

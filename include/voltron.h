@@ -279,14 +279,36 @@ VT_API vt_status vt_combine(const float* const* partials, int32_t n, int32_t row
                      const void* residual, void* out, vt_stream stream);
 
 /* ---------------------------------------------------------------- whole stack ------------------
- * vt_decode_token: one decode token through every layer, shards one after another:
- *   for each layer: every ATTN shard (vt_decode_step), vt_combine with the residual; every FFN
- *   shard, vt_combine; then every layer's KV length advances by one.
- *   x_in, x_out: device fp16 [D]; they may be the same buffer.  Uses buffers owned by the
- *   partition, so one partition runs one vt_decode_token / vt_prefill_tokens at a time.
+ * vt_decode_token: one decode token through every layer (Voltron Section 2.1, decode phase; the
+ *   tensor-parallel layer of Section 3.2.1): for each layer, every ATTN shard (as vt_decode_step)
+ *   and the combine with the residual; every FFN shard and the combine; then every layer's KV
+ *   length advances by one.
+ *   x_in, x_out: device fp16 [D], 16-byte aligned; they may be the same buffer.  Uses buffers
+ *   owned by the partition, so one partition runs one vt_decode_token / vt_prefill_tokens at a
+ *   time (stream-ordered).
+ *   When vt_decode_token_fused_available() says so, the whole token is ONE cooperative kernel
+ *   launch (one CTA per SM): each CTA streams its share of every shard's weights and cached K/V
+ *   through a shared-memory ring, shards are processed in order within each phase, and the CTAs
+ *   meet at four grid barriers per layer.  Results equal the per-shard kernels' within fp32
+ *   rounding (the FFN partials are summed with atomics, so they repeat only to fp32 rounding).
+ *   Every wait in that kernel is bounded: a CTA that gives up sets VT_DEV_WAIT_TIMEOUT in the KV
+ *   status word, the token's output is then undefined, and vt_kv_status(..., clear = 1) (or
+ *   vt_partition_status) must be called before the next token to re-arm the grid barrier.
+ *   Otherwise (unsupported shapes, or x_out not 16-byte aligned) it runs vt_decode_token_sharded.
+ *   The launch can be captured in a CUDA graph.
  */
 VT_API vt_status vt_decode_token(const vt_partition* part, vt_kv* kv, const void* x_in, void* x_out,
                           vt_stream stream);
+/* The same token as a sequence of per-shard kernels (3 per ATTN shard, 1 per FFN shard, one
+ * combine per block, one length update), linked by programmatic dependent launch. */
+VT_API vt_status vt_decode_token_sharded(const vt_partition* part, vt_kv* kv, const void* x_in,
+                                         void* x_out, vt_stream stream);
+/* 1 if vt_decode_token runs as one fused kernel for this partition, else 0; *why (optional)
+ * receives the reason when it does not (valid while the partition lives).  Fused needs a
+ * device with cooperative launch, d_model a multiple of 8 and at most 6144, d_head 64 or 128,
+ * 1, 2 or 4 query heads per KV head, at most as many KV heads as SMs, at most 256 layers, and
+ * at most 256 QKV rows per SM. */
+VT_API int32_t vt_decode_token_fused_available(const vt_partition* part, const char** why);
 /* vt_prefill_tokens: n prompt rows through every layer (same order as vt_decode_token), then
  * every layer's KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same. */
 VT_API vt_status vt_prefill_tokens(const vt_partition* part, vt_kv* kv, const void* x_in, int32_t n,

@@ -102,6 +102,8 @@ cudaError_t init_library() {
         g_init_err = init_decode_kernels();
         if (g_init_err != cudaSuccess) return;
         g_init_err = init_prefill_kernels();
+        if (g_init_err != cudaSuccess) return;
+        g_init_err = init_token_kernels();
     });
     return g_init_err;
 }
@@ -170,6 +172,11 @@ struct vt_partition {
     __half* p_attn = nullptr;   // [kPrefillChunk][max_hq dh]
     __half* p_u = nullptr;      // [kPrefillChunk][max_ld]
     int max_hq = 0, max_ld = 0;
+    // persistent decode-token kernel: shapes and scratch (the KV object adds its tables)
+    bool tok_ok = false;
+    std::string tok_why;
+    TokPlan tok_plan;
+    TokArgs tok_base{};
 
     const AttnShard& a(int l, int d) const { return attn[(size_t)l * n_dev + d]; }
     const FfnShard& f(int l, int d) const { return ffn[(size_t)l * n_dev + d]; }
@@ -182,6 +189,7 @@ struct vt_kv {
     int32_t* len = nullptr;  // device [n_layers]
     std::vector<int32_t> h_len;
     uint32_t* status = nullptr;
+    void* tok_tab = nullptr;  // device [n_layers][n_dev] TokShardPtrs, then [n_layers] TokLayerPtrs
     Allocator* alloc() const { return &p->m->alloc; }
     __half* k(int l, int d) const { return static_cast<__half*>(buf[(size_t)l * p->n_dev + d]); }
     __half* v(int l, int d) const {
@@ -597,6 +605,43 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         p->p_u = b.take<__half>(R * std::max(p->max_ld, 8));
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
     }
+    // ------------------------------------------------------------------ decode-token kernel
+    {
+        TokArgs& t = p->tok_base;
+        t = TokArgs{};
+        t.n_layers = s.n_layers;
+        t.n_dev = n;
+        t.d = D;
+        t.dh = dh;
+        t.group = g;
+        t.n_kv = s.n_kv_heads;
+        t.eps = s.rms_eps;
+        t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+        t.rope = m->rope;
+        for (int d = 0; d < n; ++d) {
+            t.hq[d] = heads[d].end - heads[d].begin;
+            t.hk[d] = t.hq[d] / g;
+            t.h0[d] = heads[d].begin;
+            t.kv0[d] = heads[d].begin / g;
+            t.cols[d] = cols[d].end - cols[d].begin;
+        }
+        p->tok_ok = token_plan(t, p->max_hq, &p->tok_plan, &p->tok_why);
+        if (p->tok_ok) {
+            const size_t bytes = 2 * align256((size_t)H * dh * 4) + 2 * align256((size_t)n * D * 4) +
+                                 align256(token_state_floats(p->tok_plan.grid, g, dh) * 4) +
+                                 align256((size_t)kTokSyncWords * 4);
+            void* q;
+            if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
+            Bump b{static_cast<uint8_t*>(q)};
+            t.q_all = b.take<float>((size_t)H * dh);
+            t.attn_part = b.take<float>((size_t)n * D);
+            t.ffn_part = b.take<float>((size_t)n * D);
+            t.states = b.take<float>(token_state_floats(p->tok_plan.grid, g, dh));
+            t.attn_out = b.take<float>((size_t)H * dh);
+            t.sync = b.take<uint32_t>(kTokSyncWords);
+            VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
+        }
+    }
     VT_CUDA(cudaStreamSynchronize(st));
     *out = p;
     return ok();
@@ -604,17 +649,23 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
 
 extern "C" int32_t vt_partition_devices(const vt_partition* p) { return p ? p->n_dev : 0; }
 
-static vt_status read_status(uint32_t* dev, uint32_t* flags, int32_t clear) {
+// With `clear`, also re-arms the decode-token kernel's grid barrier and abort word: a token that
+// gave up on a wait leaves them in an unknown state (the call that read the flags synchronised the
+// device, so no kernel is using them).
+static vt_status read_status(uint32_t* dev, uint32_t* flags, int32_t clear, uint32_t* tok_sync) {
     if (!flags) return fail(VT_ERR_INVALID_ARG, "flags is NULL");
     VT_CUDA(cudaDeviceSynchronize());
     VT_CUDA(cudaMemcpy(flags, dev, 4, cudaMemcpyDeviceToHost));
-    if (clear) VT_CUDA(cudaMemset(dev, 0, 4));
+    if (clear) {
+        VT_CUDA(cudaMemset(dev, 0, 4));
+        if (tok_sync) VT_CUDA(cudaMemset(tok_sync, 0, (size_t)kTokSyncWords * sizeof(uint32_t)));
+    }
     return ok();
 }
 
 extern "C" vt_status vt_partition_status(vt_partition* p, uint32_t* flags, int32_t clear) {
     if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
-    return read_status(p->status, flags, clear);
+    return read_status(p->status, flags, clear, p->tok_base.sync);
 }
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
@@ -682,6 +733,7 @@ extern "C" void vt_kv_destroy(vt_kv* kv) {
     Allocator* A = kv->alloc();
     for (void* b : kv->buf) A->put(b);
     A->put(kv->len);
+    A->put(kv->tok_tab);
     delete kv;
 }
 
@@ -724,6 +776,44 @@ extern "C" vt_status vt_kv_create(const vt_partition* p, int32_t cap, vt_stream 
     kv->len = reinterpret_cast<int32_t*>(mb);
     kv->status = reinterpret_cast<uint32_t*>(mb + align256((size_t)s.n_layers * 4));
     kv->h_len.assign(s.n_layers, 0);
+    // pointer tables of the decode-token kernel (host copies live until the synchronise below)
+    std::vector<TokShardPtrs> tsh;
+    std::vector<TokLayerPtrs> tly;
+    if (p->tok_ok) {
+        const int L = s.n_layers, n = p->n_dev;
+        tsh.resize((size_t)L * n);
+        tly.resize(L);
+        for (int l = 0; l < L; ++l) {
+            tly[l].attn_norm = p->m->layer[l].attn_norm;
+            tly[l].ffn_norm = p->m->layer[l].ffn_norm;
+            for (int d = 0; d < n; ++d) {
+                const AttnShard& a = p->a(l, d);
+                const FfnShard& f = p->f(l, d);
+                TokShardPtrs& t = tsh[(size_t)l * n + d];
+                t.wqkv = a.wqkv;
+                t.wo = a.wo;
+                t.wgu = f.wgu;
+                t.wdt = f.wdt;
+                t.kc = a.kv1 > a.kv0 ? kv->k(l, d) : nullptr;
+                t.vc = a.kv1 > a.kv0 ? kv->v(l, d) : nullptr;
+            }
+        }
+        const size_t tb = align256(tsh.size() * sizeof(TokShardPtrs)) + tly.size() * sizeof(TokLayerPtrs);
+        kv->tok_tab = A->get(tb);
+        if (!kv->tok_tab) {
+            vt_kv_destroy(kv);
+            return fail(VT_ERR_ALLOC, "allocating the decode-token tables failed");
+        }
+        uint8_t* tp = static_cast<uint8_t*>(kv->tok_tab);
+        cudaError_t te = cudaMemcpyAsync(tp, tsh.data(), tsh.size() * sizeof(TokShardPtrs), cudaMemcpyHostToDevice, st);
+        if (te == cudaSuccess)
+            te = cudaMemcpyAsync(tp + align256(tsh.size() * sizeof(TokShardPtrs)), tly.data(),
+                                 tly.size() * sizeof(TokLayerPtrs), cudaMemcpyHostToDevice, st);
+        if (te != cudaSuccess) {
+            vt_kv_destroy(kv);
+            return fail(VT_ERR_CUDA, "uploading the decode-token tables failed: %s", cudaGetErrorString(te));
+        }
+    }
     cudaError_t e = cudaMemsetAsync(mb, 0, meta, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) {
@@ -777,7 +867,7 @@ extern "C" vt_status vt_kv_length(vt_kv* kv, int32_t layer, vt_stream stream, in
 
 extern "C" vt_status vt_kv_status(vt_kv* kv, uint32_t* flags, int32_t clear) {
     if (!kv) return fail(VT_ERR_INVALID_ARG, "kv is NULL");
-    return read_status(kv->status, flags, clear);
+    return read_status(kv->status, flags, clear, kv->p->tok_base.sync);
 }
 
 static vt_status kv_copy(const vt_kv* kv, int32_t l, int32_t d, int32_t n_pos, void* kh,
@@ -1115,8 +1205,7 @@ extern "C" vt_status vt_prefill(const vt_partition* p, vt_shard sh, const void* 
 
 // ------------------------------------------------------------------ whole stack
 
-extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
-                                     vt_stream stream) {
+static vt_status check_token_args(const vt_partition* p, vt_kv* kv, const void* x_in, const void* x_out) {
     if (!p || !kv || kv->p != p || !x_in || !x_out)
         return fail(VT_ERR_INVALID_ARG, "bad vt_decode_token arguments");
     if (!aligned16(x_in)) return fail(VT_ERR_INVALID_ARG, "x_in must be 16-byte aligned");
@@ -1124,6 +1213,37 @@ extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const voi
     for (int l = 0; l < s.n_layers; ++l)
         if (kv->h_len[l] + 1 > kv->cap)
             return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions", l, kv->h_len[l], kv->cap);
+    return VT_OK;
+}
+
+extern "C" int32_t vt_decode_token_fused_available(const vt_partition* p, const char** why) {
+    if (why) *why = p ? (p->tok_ok ? "" : p->tok_why.c_str()) : "partition is NULL";
+    return p && p->tok_ok ? 1 : 0;
+}
+
+extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
+                                     vt_stream stream) {
+    VT_TRY(check_token_args(p, kv, x_in, x_out));
+    if (!p->tok_ok || !kv->tok_tab || !aligned16(x_out)) return vt_decode_token_sharded(p, kv, x_in, x_out, stream);
+    const vt_shapes& s = p->m->s;
+    TokArgs t = p->tok_base;
+    t.cap = kv->cap;
+    t.shard = static_cast<const TokShardPtrs*>(kv->tok_tab);
+    t.layer = reinterpret_cast<const TokLayerPtrs*>(static_cast<const uint8_t*>(kv->tok_tab) +
+                                                    align256((size_t)s.n_layers * p->n_dev * sizeof(TokShardPtrs)));
+    t.len = kv->len;
+    t.x_in = static_cast<const __half*>(x_in);
+    t.x_out = static_cast<__half*>(x_out);
+    t.status = kv->status;
+    VT_CUDA(launch_decode_token(t, p->tok_plan, (cudaStream_t)stream));
+    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
+    return ok();
+}
+
+extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
+                                             vt_stream stream) {
+    VT_TRY(check_token_args(p, kv, x_in, x_out));
+    const vt_shapes& s = p->m->s;
     cudaStream_t st = (cudaStream_t)stream;
     const int D = s.d_model, n = p->n_dev;
     // One fp32 partial buffer per shard serves both blocks: the O projection stores the ATTN

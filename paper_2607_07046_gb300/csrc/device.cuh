@@ -173,6 +173,45 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
+// Named barrier over `nthreads` threads (a multiple of 32) of the CTA.
+__device__ __forceinline__ void consumer_bar(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// R row partials per lane -> lane l with l % (32 / R) == 0 returns the warp total of row
+// l / (32 / R).  Each level halves the values a lane carries: lanes whose bit `o` is set keep the
+// upper half and send the lower half to their partner, and vice versa.
+template <int R>
+__device__ __forceinline__ float multi_row_sum(float (&v)[8], int lane) {
+    if constexpr (R == 8) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const bool hi = lane & 16;
+            const float send = hi ? v[i] : v[i + 4];
+            v[i] = (hi ? v[i + 4] : v[i]) + __shfl_xor_sync(0xffffffffu, send, 16);
+        }
+    }
+    if constexpr (R >= 4) {
+        constexpr int o = R == 8 ? 8 : 16;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const bool hi = lane & o;
+            const float send = hi ? v[i] : v[i + 2];
+            v[i] = (hi ? v[i + 2] : v[i]) + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    if constexpr (R >= 2) {
+        constexpr int o = R == 8 ? 4 : (R == 4 ? 8 : 16);
+        const bool hi = lane & o;
+        const float send = hi ? v[0] : v[1];
+        v[0] = (hi ? v[1] : v[0]) + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+    constexpr int first = R == 8 ? 2 : (R == 4 ? 4 : (R == 2 ? 8 : 16));
+#pragma unroll
+    for (int o = first; o >= 1; o >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    return v[0];
+}
+
 __device__ __forceinline__ void set_status(uint32_t* status, uint32_t bits) {
     if (status) atomicOr(status, bits);
 }

@@ -213,4 +213,65 @@ struct StaticAttnArgs {
 cudaError_t launch_attn_decode_static(const StaticAttnArgs& a, cudaStream_t st);
 vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err);
 
+
+// ------------------------------------------------------------------ persistent decode token (token.cu)
+// One cooperative launch computes a whole decode token through every layer of a partition.
+constexpr int kTokWarps = 8;                         // consumer warps
+constexpr int kTokConsumers = kTokWarps * 32;
+constexpr int kTokThreads = kTokConsumers + 32;      // + one producer warp
+constexpr int kTokStageBytes = 32768;                // one stage of the copy ring
+constexpr int kTokMinStages = 3, kTokMaxStages = 8;
+constexpr int kTokMaxSeg = 2;                        // KV heads a CTA's attention slice touches
+constexpr int kTokMaxGroup = 4;                      // query heads per KV head
+constexpr int kTokMaxD = 6144;
+constexpr int kTokMaxLayers = 256;
+constexpr int kTokMaxGrid = 1024;
+// words of TokArgs::sync (zero at creation; zeroed again by a status clear)
+constexpr int kTokSyncEpoch = 0;                            // barriers completed by earlier launches
+constexpr int kTokSyncAbort = 2;                            // nonzero: the token gave up on a wait
+constexpr int kTokSyncFlags = 64;                           // [grid] epoch of each CTA's last arrival
+constexpr int kTokSyncWords = kTokSyncFlags + kTokMaxGrid;
+
+struct TokShardPtrs {  // one (layer, device) shard; null weights for an empty block
+    const __half* wqkv;  // [(hq + 2 hk) dh][D], RoPE-pair row order
+    const __half* wo;    // [D][hq dh]
+    const __half* wgu;   // [2c][D], gate/up rows interleaved
+    const __half* wdt;   // [c][D]
+    __half* kc;          // [hk][cap][dh]
+    __half* vc;
+};
+struct TokLayerPtrs {
+    const __half* attn_norm;  // [D]
+    const __half* ffn_norm;   // [D]
+};
+
+struct TokArgs {
+    int n_layers, n_dev, d, dh, group, cap, n_kv, stages, uni_floats, slot_floats;
+    int hq[VT_MAX_DEVICES], hk[VT_MAX_DEVICES], h0[VT_MAX_DEVICES], kv0[VT_MAX_DEVICES],
+        cols[VT_MAX_DEVICES];
+    float eps, scale_log2;
+    const TokShardPtrs* shard;  // [n_layers][n_dev]
+    const TokLayerPtrs* layer;  // [n_layers]
+    int32_t* len;               // [n_layers] device KV lengths (advanced by the kernel)
+    const float2* rope;         // [max_seq][dh/2]
+    const __half* x_in;         // [D]
+    __half* x_out;              // [D]
+    float* q_all;               // [H][dh] rotated queries of the token
+    float* attn_part;           // [n_dev][D]
+    float* ffn_part;            // [n_dev][D] (zeroed inside the kernel before use)
+    float* states;              // [grid][kTokMaxSeg][group][dh + 2] attention slice states
+    float* attn_out;            // [H][dh] merged attention output of the token
+    uint32_t* sync;             // kTokSync* words: barrier epoch, abort word, per-CTA arrival flags
+    uint32_t* status;
+};
+struct TokPlan {  // host-side launch geometry
+    int grid = 0, stages = 0, uni_floats = 0, slot_floats = 0, variant = 0;
+    size_t smem = 0;
+};
+// Fills `plan` and returns true when the fused kernel supports the partition's shapes.
+bool token_plan(const TokArgs& a, int max_hq, TokPlan* plan, std::string* why);
+cudaError_t launch_decode_token(const TokArgs& a, const TokPlan& plan, cudaStream_t st);
+size_t token_state_floats(int grid, int group, int dh);
+cudaError_t init_token_kernels();
+
 }  // namespace vt

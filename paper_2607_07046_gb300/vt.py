@@ -118,6 +118,8 @@ def lib() -> ctypes.CDLL:
             "vt_prefill": (S, [_P, vt_shard, _P, _I32, _P, _P, _P]),
             "vt_combine": (S, [ctypes.POINTER(_P), _I32, _I32, _I32, _P, _P, _P]),
             "vt_decode_token": (S, [_P, _P, _P, _P, _P]),
+            "vt_decode_token_sharded": (S, [_P, _P, _P, _P, _P]),
+            "vt_decode_token_fused_available": (_I32, [_P, ctypes.POINTER(ctypes.c_char_p)]),
             "vt_prefill_tokens": (S, [_P, _P, _P, _I32, _P, _P]),
         }
         for name, (res, args) in sig.items():
@@ -390,6 +392,19 @@ def vt_decode_token(part: int, kv: int, x_in, x_out, stream=None) -> None:
     import torch
     _check(lib().vt_decode_token(part, kv, _ptr(x_in, torch.float16), _ptr(x_out, torch.float16),
                                  _stream(stream)))
+
+
+def vt_decode_token_sharded(part: int, kv: int, x_in, x_out, stream=None) -> None:
+    import torch
+    _check(lib().vt_decode_token_sharded(part, kv, _ptr(x_in, torch.float16),
+                                         _ptr(x_out, torch.float16), _stream(stream)))
+
+
+def vt_decode_token_fused_available(part: int):
+    """(available, reason): whether vt_decode_token runs as one fused kernel for this partition."""
+    why = ctypes.c_char_p()
+    ok = lib().vt_decode_token_fused_available(part, ctypes.byref(why))
+    return bool(ok), (why.value or b"").decode()
 
 
 def vt_prefill_tokens(part: int, kv: int, x_in, n: int, x_out, stream=None) -> None:
