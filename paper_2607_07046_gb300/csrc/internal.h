@@ -246,7 +246,7 @@ struct TokLayerPtrs {
 };
 
 struct TokArgs {
-    int n_layers, n_dev, d, dh, group, cap, n_kv, stages, uni_floats, slot_floats;
+    int n_layers, n_dev, d, dh, group, cap, n_kv, stages, uni_floats, slot_floats, ffn_gcol;
     int hq[VT_MAX_DEVICES], hk[VT_MAX_DEVICES], h0[VT_MAX_DEVICES], kv0[VT_MAX_DEVICES],
         cols[VT_MAX_DEVICES];
     float eps, scale_log2;
@@ -265,7 +265,7 @@ struct TokArgs {
     uint32_t* status;
 };
 struct TokPlan {  // host-side launch geometry
-    int grid = 0, stages = 0, uni_floats = 0, slot_floats = 0, variant = 0;
+    int grid = 0, stages = 0, uni_floats = 0, slot_floats = 0, variant = 0, ffn_gcol = 0;
     size_t smem = 0;
 };
 // Fills `plan` and returns true when the fused kernel supports the partition's shapes.

@@ -280,10 +280,9 @@ __device__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epo
         int ok = live ? 1 : 0;
         uint32_t* flags = a.sync + kTokSyncFlags;
         if (ok) {
-            if (lane == 0) {
-                __threadfence();
-                st_release(flags + blockIdx.x, epoch);
-            }
+            // the CTA's writes precede this store through the CTA barrier above, and a release
+            // store makes them visible to every thread that acquires the flag
+            if (lane == 0) st_release(flags + blockIdx.x, epoch);
             uint32_t i = 0;
             while (true) {
                 bool mine = true;
@@ -434,6 +433,24 @@ __device__ __forceinline__ void prefetch_bgain(const __half* gain, const MmaLane
         if (o2 >= L) o2 -= L;
         gf[i][0] = *reinterpret_cast<const uint32_t*>(gain + ml.bseg + off);
         gf[i][1] = *reinterpret_cast<const uint32_t*>(gain + ml.bseg + o2);
+        off += 16;
+        if (off >= L) off -= L;
+    }
+}
+
+// B fragments of this lane from hi / lo fp16 copies of the input in shared memory.
+template <int STEPS>
+__device__ __forceinline__ void load_bfrags_h(const __half* xh, const __half* xl, const MmaLane& ml, int L,
+                                              uint32_t (&bh)[STEPS][2], uint32_t (&bl)[STEPS][2]) {
+    int off = ml.boff0;
+#pragma unroll
+    for (int i = 0; i < STEPS; ++i) {
+        int o2 = off + 8;
+        if (o2 >= L) o2 -= L;
+        bh[i][0] = *reinterpret_cast<const uint32_t*>(xh + ml.bseg + off);
+        bh[i][1] = *reinterpret_cast<const uint32_t*>(xh + ml.bseg + o2);
+        bl[i][0] = *reinterpret_cast<const uint32_t*>(xl + ml.bseg + off);
+        bl[i][1] = *reinterpret_cast<const uint32_t*>(xl + ml.bseg + o2);
         off += 16;
         if (off >= L) off -= L;
     }
@@ -730,9 +747,10 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
 
     const MmaGeom gd = mma_geom(D);
     const int rps_d = gd.R;
-    // FFN columns per group: the gate/up rows of the group, then its down rows (at most 64
-    // columns, so the gate/up row partials of a group fit the slots)
-    const int gcol = min(16 * rps_d, 64);
+    // FFN columns per group: all gate/up rows of the group, then its down rows.  A CTA's columns
+    // of one shard form one group when they fit the slots (at most 128 columns), which keeps the
+    // input fragments and the down-projection accumulators from being live at the same time.
+    const int gcol = a.ffn_gcol;
     Ring ring{ring_base, full, empty, S, 0u, 0, 0u};
 
     if (warp == kTokWarps) {
@@ -1006,12 +1024,18 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                 const MmaGeom go = mma_geom(K);
                 const MmaLane mlo = mma_lane(go, warp, lane);
                 if (mma_ok(K)) {
+                    // the rows' steps match the kernel's: B fragments in registers; else from shared memory
+                    const bool regs = go.L == 16 * STEPS;
+                    if (regs) load_bfrags_h<STEPS>(xh, xl, mlo, go.L, bh, bl);
                     int rowbase = 0;
                     for (int r = r0; r < r1; r += go.R) {
                         const int n = min(go.R, r1 - r);
                         const uint8_t* st = ring_acquire(ring, live, a);
                         if (!st) continue;
-                        stage_mma_smem(ring_s + (uint32_t)(st - ring_base), n, K, go, mlo, rowbase, xh, xl, slots);
+                        if (regs)
+                            stage_mma_regs<STEPS>(ring_s + (uint32_t)(st - ring_base), n, K, go, mlo, rowbase, bh, bl, slots);
+                        else
+                            stage_mma_smem(ring_s + (uint32_t)(st - ring_base), n, K, go, mlo, rowbase, xh, xl, slots);
                         ring_release(ring, lane);
                         rowbase += n;
                     }
@@ -1045,11 +1069,6 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
         // h = x + sum of the ATTN partials (shards in order), rounded to fp16
         combine_norm(a.attn_part, true, false);
         for_ffn_pieces(a, c, NC, [&](int s, int j0, int j1) {
-            float acc[MC][8];
-#pragma unroll
-            for (int m = 0; m < MC; ++m)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[m][e] = 0.f;
             for (int g = j0; g < j1; g += gcol) {
                 const int ng = min(gcol, j1 - g);
                 for (int r = 2 * g; r < 2 * (g + ng); r += rps_d) {
@@ -1062,6 +1081,11 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                 consumer_bar(1, kTokConsumers);
                 if (tid < ng) act[tid] = silu(row_total(slots, 2 * tid, gd.spr)) * row_total(slots, 2 * tid + 1, gd.spr);
                 consumer_bar(1, kTokConsumers);
+                float acc[MC][8];
+#pragma unroll
+                for (int m = 0; m < MC; ++m)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[m][e] = 0.f;
                 for (int r = g; r < g + ng; r += rps_d) {
                     const int n = min(rps_d, g + ng - r);
                     const uint8_t* st = ring_acquire(ring, live, a);
@@ -1082,15 +1106,15 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                     }
                     ring_release(ring, lane);
                 }
-            }
-            if (live) {
+                if (live) {
 #pragma unroll
-                for (int m = 0; m < MC; ++m) {
-                    const int ch = tid + kTokConsumers * m;
-                    if (ch < nch) {
-                        float4* dst = reinterpret_cast<float4*>(a.ffn_part + (size_t)s * D + ch * 8);
-                        atomicAdd(dst, make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]));
-                        atomicAdd(dst + 1, make_float4(acc[m][4], acc[m][5], acc[m][6], acc[m][7]));
+                    for (int m = 0; m < MC; ++m) {
+                        const int ch = tid + kTokConsumers * m;
+                        if (ch < nch) {
+                            float4* dst = reinterpret_cast<float4*>(a.ffn_part + (size_t)s * D + ch * 8);
+                            atomicAdd(dst, make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]));
+                            atomicAdd(dst + 1, make_float4(acc[m][4], acc[m][5], acc[m][6], acc[m][7]));
+                        }
                     }
                 }
             }
@@ -1194,7 +1218,9 @@ bool token_plan(const TokArgs& a, int max_hq, TokPlan* plan, std::string* why) {
     int64_t n_o = 0;
     for (int s = 0; s < a.n_dev; ++s) n_o += a.hq[s] > 0 ? a.d : 0;
     const int64_t qkv_rows = 2 * ((pairs + grid - 1) / grid), o_rows = (n_o + grid - 1) / grid + 1;
-    const int gcol = std::min(16 * gd.R, 64);
+    int64_t ffn_tot = 0;
+    for (int s = 0; s < a.n_dev; ++s) ffn_tot += a.cols[s];
+    const int gcol = (int)std::min<int64_t>((ffn_tot + grid - 1) / grid + 1, 128);
     int64_t slot = qkv_rows * gd.spr;
     slot = std::max<int64_t>(slot, (int64_t)2 * gcol * gd.spr);
     slot = std::max<int64_t>(slot, o_rows * o_spr);
@@ -1219,6 +1245,7 @@ bool token_plan(const TokArgs& a, int max_hq, TokPlan* plan, std::string* why) {
     plan->stages = stages;
     plan->uni_floats = uni;
     plan->slot_floats = (int)slot;
+    plan->ffn_gcol = gcol;
     plan->variant = vi;
     plan->smem = smem;
     return true;
@@ -1229,6 +1256,7 @@ cudaError_t launch_decode_token(const TokArgs& args, const TokPlan& plan, cudaSt
     a.stages = plan.stages;
     a.uni_floats = plan.uni_floats;
     a.slot_floats = plan.slot_floats;
+    a.ffn_gcol = plan.ffn_gcol;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(plan.grid);
     cfg.blockDim = dim3(kTokThreads);
