@@ -264,10 +264,47 @@ struct TokArgs {
     uint32_t* sync;             // kTokSync* words: barrier epoch, abort word, per-CTA arrival flags
     uint32_t* status;
 };
+// Geometry of the tensor-core GEMV over one 32 KB stage of rows of length K (token_kernel.cuh).
+struct MmaGeom {
+    int R;    // rows per stage
+    int NP;   // row pairs per stage
+    int WP;   // warps per row pair (each takes 8 segments of K / WP)
+    int L;    // segment length
+    int spr;  // partial sums per row (8 WP)
+};
+
+__host__ __device__ inline MmaGeom mma_geom(int K) {
+    MmaGeom g;
+    int r = kTokStageBytes / (2 * K);
+    g.R = r < 1 ? 1 : (r > 64 ? 64 : r);
+    g.NP = (g.R + 1) / 2;
+    g.WP = g.NP >= 5 ? 1 : (g.NP >= 3 ? 2 : (g.NP == 2 ? 4 : 8));
+    g.L = K / (8 * g.WP);
+    g.spr = 8 * g.WP;
+    return g;
+}
+// The tensor-core path needs whole 16-element steps in every segment.
+__host__ __device__ inline bool mma_ok(int K) {
+    const MmaGeom g = mma_geom(K);
+    return K % (8 * g.WP) == 0 && g.L >= 16 && g.L % 16 == 0;
+}
+
 struct TokPlan {  // host-side launch geometry
     int grid = 0, stages = 0, uni_floats = 0, slot_floats = 0, variant = 0, ffn_gcol = 0;
     size_t smem = 0;
 };
+// One compiled variant of the kernel: tensor-core steps per row segment (STEPS), fp32 chunks per
+// thread of a D-vector (MC), head dim, query heads per KV head, and whether the O rows may use the
+// shared-memory or CUDA-core paths (shards whose rows do not match STEPS).
+struct TokVariant {
+    int steps, mc, dh, group;
+    bool osmem;
+    cudaError_t (*init)(int optin, size_t* dyn_max);
+    cudaError_t (*occupancy)(int* per_sm, size_t smem);
+    cudaError_t (*launch)(const TokArgs& a, const cudaLaunchConfig_t& cfg);
+};
+int token_variants_workloads(const TokVariant** out);  // token_v1.cu
+int token_variants_small(const TokVariant** out);      // token_v2.cu
 // Fills `plan` and returns true when the fused kernel supports the partition's shapes.
 bool token_plan(const TokArgs& a, int max_hq, TokPlan* plan, std::string* why);
 cudaError_t launch_decode_token(const TokArgs& a, const TokPlan& plan, cudaStream_t st);

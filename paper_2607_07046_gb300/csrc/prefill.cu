@@ -359,6 +359,22 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc::fence_after();
     const uint32_t tmem = *tmem_slot;
+    // B (the weights) does not depend on the preceding kernel: the B halves of the first stages
+    // and the L2 prefetch of the CTA's remaining B tiles are issued before griddepcontrol.wait, so
+    // they stream while the preceding kernel finishes; A, which it wrote, is loaded after the wait.
+    const int pre = nk < kStages ? nk : kStages;
+    if (warp == 0 && lane == 0) {
+        for (int i = 0; i < pre; ++i) {
+            mbar_arrive_expect_tx(&full[i], kStageBytes);
+            tc::tma_load_2d(smem + i * kStageBytes + kABytes, &tb, (kt0 + i) * kBK, n0, &full[i]);
+        }
+    } else if (warp >= 2) {
+        const int t = threadIdx.x - 64;
+        for (int i = kt0 + pre; i < kt1; ++i)
+            for (int r = t; r < kBN; r += kGemmThreads - 64)
+                if (n0 + r < a.n)
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.b + (size_t)(n0 + r) * a.ldb + (size_t)i * kBK));
+    }
     pdl_wait();  // A was written by the preceding kernel
 
     bool ok = true;
@@ -374,12 +390,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 }
                 if (*(volatile int*)&s_err) break;
                 uint8_t* st = smem + s * kStageBytes;
-                mbar_arrive_expect_tx(&full[s], kStageBytes);
-                tc::tma_load_2d(st, &ta, (kt0 + i) * kBK, m0, &full[s]);
-                tc::tma_load_2d(st + kABytes, &tb, (kt0 + i) * kBK, n0, &full[s]);
+                if (i < pre) {  // B of this stage is already on its way
+                    tc::tma_load_2d(st, &ta, (kt0 + i) * kBK, m0, &full[s]);
+                } else {
+                    mbar_arrive_expect_tx(&full[s], kStageBytes);
+                    tc::tma_load_2d(st, &ta, (kt0 + i) * kBK, m0, &full[s]);
+                    tc::tma_load_2d(st + kABytes, &tb, (kt0 + i) * kBK, n0, &full[s]);
+                }
                 issued = i + 1;
             }
-            // no copy may still be in flight when the stage memory is reused or the CTA ends
+            // no copy may still be in flight when the stage memory is reused or the CTA ends (after an
+            // early stop this includes the B halves issued before griddepcontrol.wait: their stages
+            // never complete, and the bounded wait outlasts the copies)
+            if (issued < pre) issued = pre;
             for (int i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
                 if (!mbar_wait(&full[i % kStages], (i / kStages) & 1)) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
         }
@@ -404,15 +427,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tc::mma_commit(done);
         }
     } else {
-        // While the main loop runs, pull this CTA's slice of B into L2 (one prefetch per 128-byte
-        // line, k-tile by k-tile), so the TMA loads of later stages hit L2 instead of HBM.
-        {
-            const int t = threadIdx.x - 64;
-            for (int i = kt0; i < kt1; ++i)
-                for (int r = t; r < kBN; r += kGemmThreads - 64)
-                    if (n0 + r < a.n)
-                        asm volatile("prefetch.global.L2 [%0];" ::"l"(a.b + (size_t)(n0 + r) * a.ldb + (size_t)i * kBK));
-        }
         // one lane per warp polls the barrier (128 pollers would compete with the TMA and MMA
         // threads for issue slots and shared-memory bandwidth during the whole main loop)
         if (lane == 0) {
