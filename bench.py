@@ -36,8 +36,9 @@ METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
-# that kernel as it is built now; None until captured, and again once the kernel changes.
-K_TOKEN_DRAM_BYTES_PER_LAUNCH = None
+# that kernel as it is built now (mean of the 12 launches of the 7B launch list); None until
+# captured, and again once the kernel changes.
+K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_505_242_325
 
 
 def measured_peaks():
@@ -416,7 +417,7 @@ def run_decode(args, rank, world):
             "peak_kind": f"{peak_kind} copy bandwidth",
             "bytes_per_launch": int(step_bytes) if fused else None,
             "launch_ms": round(ms_per_step, 5),
-            "traffic": K_TOKEN_DRAM_BYTES_PER_LAUNCH if fused else None,
+            "traffic": K_TOKEN_DRAM_BYTES_PER_LAUNCH if fused and not args.layers else None,
         },
         "e2e": {"value": round(world / e2e_s, 3), "unit": "tok/s", "h2d_bytes_per_step": 4,
                 "d2h_bytes_per_step": 2 * D, "finite": e2e_finite},
