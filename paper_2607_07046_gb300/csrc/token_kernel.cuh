@@ -237,14 +237,17 @@ __device__ __forceinline__ void ring_release(Ring& r, int lane) {
 // flag has reached it: warp 0 polls all flags (a few loads per lane) and the fence after the
 // poll orders the CTA's later reads after the others' writes.  No two CTAs write one word, so
 // arrivals do not queue behind each other.  Called by all consumer threads; returns false when
-// the token is aborted (then it does not wait).
+// the token is aborted (then it does not wait).  Out of line, like the other helpers called from
+// several places: the kernel is larger than the instruction cache, and every miss waits behind
+// the weight stream for its L2 round trip (one copy of the barrier instead of four measured 7%
+// of the token time).
 __device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
-__device__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epoch) {
+__device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epoch) {
     consumer_bar(1, kTokConsumers);
     const int lane = threadIdx.x & 31;
     if (threadIdx.x < 32) {
@@ -485,7 +488,7 @@ __device__ __forceinline__ void stage_mma_smem(uint32_t st, int nrows, int K, co
 
 // Sum of the spr partial sums of a row, in slot order.
 // (spr is a multiple of 8; four interleaved partial sums, added in a fixed order)
-__device__ __forceinline__ float row_total(const float* slots, int row, int spr) {
+__device__ __noinline__ float row_total(const float* slots, int row, int spr) {
     const float* r = slots + row * spr;
     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
     for (int i = 0; i < spr; i += 4) {
