@@ -218,7 +218,13 @@ vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::strin
 // One cooperative launch computes a whole decode token through every layer of a partition.
 constexpr int kTokWarps = 8;                         // consumer warps
 constexpr int kTokConsumers = kTokWarps * 32;
-constexpr int kTokThreads = kTokConsumers + 32;      // + one producer warp
+// + one warpgroup holding the producer warp (the other three warps leave at once): a whole
+// warpgroup, so that it can hand registers to the consumers with setmaxnreg
+constexpr int kTokThreads = kTokConsumers + 128;
+constexpr int kTokLaunchRegs = 168;                // per thread at launch: 65536 / 384, rounded down to 8
+constexpr int kTokProducerRegs = 56, kTokConsumerRegs = 224;
+static_assert(128 * kTokProducerRegs + kTokConsumers * kTokConsumerRegs <= kTokThreads * kTokLaunchRegs,
+              "the register split must fit in the registers the block is launched with");
 constexpr int kTokStageBytes = 32768;                // one stage of the copy ring
 constexpr int kTokMinStages = 3, kTokMaxStages = 8;
 constexpr int kTokMaxSeg = 2;                        // KV heads a CTA's attention slice touches

@@ -26,7 +26,7 @@
 //   O          rows of all shards' Wo, shard after shard, into the shard partials
 //   FFN        intermediate columns of all shards: gate/up rows, SwiGLU, then the matching rows
 //              of the transposed down slice, accumulated per CTA and added into the shard
-//              partial with vector atomics (so FFN partials repeat only to fp32 rounding)
+//              partial with one bulk reduction (so FFN partials repeat only to fp32 rounding)
 // The matrix-vector products run on the tensor cores (mma.sync; see the tensor-core GEMV notes
 // below); the FFN down projection, a sum of scaled rows, runs on the CUDA cores.
 // Every shard's partial depends on that shard's weights only, and the combines add the shards in
@@ -137,6 +137,7 @@ bool token_plan(const TokArgs& a, int max_hq, TokPlan* plan, std::string* why) {
     // while the O rows' partial sums use the first half
     const int64_t table = (int64_t)a.n_kv * (grid / std::max(1, a.n_kv) + 3);
     slot = std::max<int64_t>(slot, 2 * std::max<int64_t>(table, o_rows * o_spr));
+    slot = std::max<int64_t>(slot, a.d);  // the FFN phase stages a D-vector there for its bulk reduction
     if (slot > 16384) return no("too much per-CTA work for the partial-sum slots");
     const int uni = std::max(max_hq * a.dh, kTokWarps * a.group * (a.dh + 2));
     int stages = kTokMaxStages;

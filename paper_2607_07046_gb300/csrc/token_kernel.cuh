@@ -773,9 +773,12 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
     const int gcol = a.ffn_gcol;
     Ring ring{ring_base, full, empty, S, 0u, 0, 0u, true};
 
-    if (warp == kTokWarps) {
+    if (warp >= kTokWarps) {
         // ================================================================ producer
-        if (lane == 0) {
+        // the producer warpgroup keeps kTokProducerRegs registers per thread and gives the rest
+        // to the two consumer warpgroups (both sides of the split run before any wait)
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kTokProducerRegs));
+        if (warp == kTokWarps && lane == 0) {
             bool live = true;
             auto issue = [&](const void* s0, uint32_t b0, const void* s1, uint32_t b1) {
                 if (!live) return;
@@ -844,6 +847,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
     }
 
     // ==================================================================== consumers (256 threads)
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kTokConsumerRegs));
     bool live = ld_volatile(a.sync + kTokSyncAbort) == 0;
     uint32_t epoch = s_epoch;
     const uint32_t ring_s = smem_u32(ring_base);
@@ -1080,17 +1084,23 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                     }
                     ring_release(ring, lane);
                 }
-                if (live) {
+                // the group's D-vector goes to the slots (free once the activations are computed) and
+                // is added into the shard partial by one bulk reduction: a few hundred line-sized
+                // additions in the L2 instead of thousands of vector atomics, which the CTA's barrier
+                // arrival would have to wait for
 #pragma unroll
-                    for (int m = 0; m < MC; ++m) {
-                        const int ch = tid + kTokConsumers * m;
-                        if (ch < nch) {
-                            float4* dst = reinterpret_cast<float4*>(a.ffn_part + (size_t)s * D + ch * 8);
-                            atomicAdd(dst, make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]));
-                            atomicAdd(dst + 1, make_float4(acc[m][4], acc[m][5], acc[m][6], acc[m][7]));
-                        }
+                for (int m = 0; m < MC; ++m) {
+                    const int ch = tid + kTokConsumers * m;
+                    if (ch < nch) {
+                        float4* v = reinterpret_cast<float4*>(slots + ch * 8);
+                        v[0] = make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]);
+                        v[1] = make_float4(acc[m][4], acc[m][5], acc[m][6], acc[m][7]);
                     }
                 }
+                fence_proxy_async_smem();
+                consumer_bar(1, kTokConsumers);
+                if (tid == 0 && live) bulk_reduce_add_f32(a.ffn_part + (size_t)s * D, slots, (uint32_t)D * 4u);
+                consumer_bar(1, kTokConsumers);  // the reduction has read the slots
             }
         });
         if (l + 1 < a.n_layers) prefetch_bgain<STEPS>(a.layer[l + 1].attn_norm, mld, gd.L, gf);
