@@ -234,18 +234,14 @@ __device__ __forceinline__ void ring_release(Ring& r, int lane) {
 // Barrier over the CTAs of the (cooperative) launch.  Barrier i of a launch has epoch
 // base + i + 1, base being the count of barriers of all earlier launches (sync[kTokSyncEpoch]).
 // A CTA arrives by publishing the epoch in its own flag (release) and waits until every CTA's
-// flag has reached it: warp 0 polls all flags (a few loads per lane) and the fence after the
-// poll orders the CTA's later reads after the others' writes.  No two CTAs write one word, so
+// flag has reached it: warp 0 polls all flags with acquire loads (a few per lane), and the CTA
+// barrier that follows orders every consumer thread's later reads after the other CTAs' writes
+// (no full fence: under the weight stream one costs about a microsecond per barrier).  No two CTAs write one word, so
 // arrivals do not queue behind each other.  Called by all consumer threads; returns false when
 // the token is aborted (then it does not wait).  Out of line, like the other helpers called from
 // several places: the kernel is larger than the instruction cache, and every miss waits behind
 // the weight stream for its L2 round trip (one copy of the barrier instead of four measured 7%
 // of the token time).
-__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
-    uint32_t v;
-    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
 
 __device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epoch) {
     consumer_bar(1, kTokConsumers);
@@ -261,7 +257,7 @@ __device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live,
             // polls, so a poll costs one L2 round trip
             for (uint32_t i = 1;; ++i) {
                 bool mine = true;
-                for (int x = lane; x < (int)gridDim.x; x += 32) mine &= (int32_t)(ld_relaxed(flags + x) - epoch) >= 0;
+                for (int x = lane; x < (int)gridDim.x; x += 32) mine &= (int32_t)(ld_acquire(flags + x) - epoch) >= 0;
                 if (__all_sync(0xffffffffu, mine)) break;
                 if ((i & 63) == 0) {
                     int stop = 0;
@@ -278,8 +274,8 @@ __device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live,
                     }
                 }
             }
-            __threadfence();
-            if (lane == 0 && ok && ld_volatile(a.sync + kTokSyncAbort)) ok = 0;
+            // no second look at the abort word here: it costs an L2 round trip on every barrier,
+            // and a CTA that aborts after arriving is seen at the next wait
         }
         if (lane == 0) *s_flag = ok;
     }
@@ -1099,7 +1095,11 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                 }
                 fence_proxy_async_smem();
                 consumer_bar(1, kTokConsumers);
-                if (tid == 0 && live) bulk_reduce_add_f32(a.ffn_part + (size_t)s * D, slots, (uint32_t)D * 4u);
+                if (tid == 0 && live) {
+                    bulk_reduce_add_f32(a.ffn_part + (size_t)s * D, slots, (uint32_t)D * 4u);
+                    // the reduction's writes (async proxy) before the barrier's release store
+                    asm volatile("fence.proxy.async;" ::: "memory");
+                }
                 consumer_bar(1, kTokConsumers);  // the reduction has read the slots
             }
         });
