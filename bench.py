@@ -10,8 +10,9 @@ Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs r
 synchronised every step); `roofline` is the token kernel's achieved HBM bandwidth (algorithmic
 bytes of the step over its time); `sharded_token` times the same token as per-shard kernels;
 `cpu_baseline` is the CPU oracle timed on a bounded sample; `prefill` is the 512-token prompt of the
-7B prefill workload through the same stack (tok/s and tensor-core rate).  `--impl reference` times
-the CPU oracle alone.
+7B prefill workload through the same stack (tok/s and tensor-core rate); `other_workloads` are the
+13B (uneven 3-way, KV 2048) and 8B GQA (4-way, KV 4096) decode shapes timed the same way.
+`--impl reference` times the CPU oracle alone.
 """
 from __future__ import annotations
 
@@ -38,7 +39,7 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
 # that kernel as it is built now (mean of the 12 launches of the 7B launch list); None until
 # captured, and again once the kernel changes.
-K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_503_546_603
+K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_503_825_067
 
 
 def measured_peaks():
@@ -435,6 +436,61 @@ def run_decode(args, rank, world):
     return line, clk.summary()
 
 
+def run_decode_workload(cid, steps, warmup):
+    """Decode tok/s of one more workload (the 13B uneven 3-way and the 8B GQA 4-way shapes), timed
+    like the headline one: vt_decode_token replayed as a CUDA graph over the workload's KV schedule
+    (kv_len -> kv_len + decode_steps - 1, then rewound), inputs resident on the device."""
+    import torch
+
+    from paper_2607_07046_gb300 import vt
+    from paper_2607_07046_gb300.stack import Stack
+
+    wl = synthetic.WORKLOADS[cid]
+    sched = wl.decode_steps
+    cap = wl.kv_len + sched + 8
+    stream = torch.cuda.Stream()
+    t_setup = time.perf_counter()
+    with torch.cuda.stream(stream):
+        st = Stack(shapes_for(vt, wl, cap), wl.layer_weights, wl.head_ranges, wl.ffn_ranges, cap, stream=stream)
+    try:
+        g = wl.n_heads // wl.n_kv_heads
+        for l in range(wl.n_layers):
+            kc, vc = wl.kv_fill(l, wl.kv_len)
+            for d, (h0, h1) in enumerate(wl.head_ranges):
+                if h1 > h0:
+                    vt.vt_kv_write_raw(st.kv, l, d, kc[h0 // g:h1 // g], vc[h0 // g:h1 // g])
+        vt.vt_kv_set_length(st.kv, -1, wl.kv_len, stream)
+        setup_s = time.perf_counter() - t_setup
+        fused, why = vt.vt_decode_token_fused_available(st.part)
+        xin = torch.from_numpy(wl.hidden(1).reshape(-1)).cuda()
+        xout = torch.empty_like(xin)
+        stream.synchronize()
+        sch = TokenSchedule(vt, st, vt.vt_decode_token, xin, xout, stream, sched, wl.kv_len)
+        ms = time_tokens(torch, sch, stream, steps, warmup)
+        finite = bool(torch.isfinite(xout.float()).all().item())
+        status = {"kv": vt.vt_kv_status(st.kv, clear=True), "partition": vt.vt_partition_status(st.part, clear=True)}
+        del sch
+    finally:
+        torch.cuda.synchronize()
+        st.close()
+    hbm, _, _, peak_kind = measured_peaks()
+    kv_mean = wl.kv_len + (min(steps, sched) - 1) / 2.0
+    step_bytes = decode_bytes_per_token(wl, kv_mean)
+    achieved = step_bytes / (ms * 1e-3) / 1e9
+    return {
+        "workload": wl.name,
+        "shape": f"{wl.n_layers} layers, D {wl.d_model}, {wl.n_heads} query / {wl.n_kv_heads} KV heads x "
+                 f"{wl.d_head}, FFN {wl.d_ffn}; heads {[h1 - h0 for h0, h1 in wl.head_ranges]}, "
+                 f"FFN columns {[c1 - c0 for c0, c1 in wl.ffn_ranges]}; KV {wl.kv_len} -> {wl.kv_len + sched - 1}",
+        "value": round(1000.0 / ms, 3), "unit": "tok/s", "ms_per_step": round(ms, 5), "steps": steps,
+        "token_kernel": "fused: one cooperative kernel per token" if fused else f"per-shard kernels ({why})",
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(achieved / hbm, 4), "peak_kind": f"{peak_kind} copy bandwidth",
+                     "bytes_per_launch": int(step_bytes)},
+        "device_status": status, "finite": finite, "setup_s": round(setup_s, 1),
+    }
+
+
 # ------------------------------------------------------------------ reference arm (CPU oracle)
 
 def run_reference(args):
@@ -480,6 +536,8 @@ def main():
                     help="timed tokens of the per-shard entry point, for context (0: skip)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: only the first N layers of the stack")
+    ap.add_argument("--other-steps", type=int, default=64,
+                    help="timed tokens of the 13B and 8B decode workloads, 1 GPU only (0: skip)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -494,6 +552,8 @@ def main():
         torch.distributed.init_process_group("nccl")
     line, clocks = run_decode(args, rank, world)
     line["clocks"] = clocks
+    if world == 1 and args.other_steps > 0 and not args.layers:
+        line["other_workloads"] = [run_decode_workload(cid, args.other_steps, 8) for cid in (3, 5)]
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_decode(synthetic.WORKLOADS[2])
     if world > 1:

@@ -209,7 +209,7 @@ __device__ __forceinline__ bool mbar_try_wait_suspend(uint64_t* bar, uint32_t pa
 __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, const uint32_t* abort_word) {
     for (uint32_t i = 0; i < kTokWaitPolls; ++i) {
         if (mbar_try_wait_suspend(bar, parity)) return true;
-        if ((i & 7) == 7 && ld_volatile(abort_word)) return false;
+        if ((i & 63) == 63 && ld_volatile(abort_word)) return false;  // rare: an L2 round trip
     }
     return false;
 }
