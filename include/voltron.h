@@ -65,6 +65,7 @@ typedef int32_t vt_status;
 #define VT_ERR_CUDA 8             /* a CUDA runtime call failed (text in vt_last_error) */
 #define VT_ERR_ALLOC 9            /* the allocator returned NULL */
 #define VT_ERR_STATE 10           /* object not ready (e.g. a layer's weights never loaded) */
+#define VT_ERR_PLAN_MEMORY 11     /* the devices' memory budgets cannot hold the block */
 
 #define VT_MAX_DEVICES 16
 
@@ -137,6 +138,32 @@ VT_API const char* vt_version(void);
 VT_API vt_status vt_shapes_validate(const vt_shapes* shapes);
 VT_API vt_status vt_partition_validate(const vt_shapes* shapes, int32_t n_devices,
                                 const vt_range* head_ranges, const vt_range* ffn_col_ranges);
+
+/* ---------------------------------------------------------------- planning (host only) --------
+ * vt_plan_tp_shares: the heterogeneity-aware tensor-parallel split of one block (Voltron Section
+ * 4.2.1, layer allocation under TP: shards are assigned greedily to devices by their performance,
+ * to balance the execution time across devices and so limit stragglers; within each device's
+ * memory budget, Section 4.2.1 and Fig. 5).
+ *
+ * The block is cut into equal units: for VT_BLOCK_ATTN one KV group (n_heads / n_kv_heads query
+ * heads with their KV head); for VT_BLOCK_FFN `col_unit` FFN columns (the last unit is shorter
+ * when col_unit does not divide d_ffn; col_unit is ignored for ATTN).  A unit's bytes are its
+ * fp16 weights (ATTN: its QKV rows and O columns, plus its K and V cache at max_seq positions;
+ * FFN: its gate, up and down columns).  Decode streams every shard byte once per token, so device
+ * d takes units_d * unit_bytes / rate[d] seconds (rate: bytes per second, > 0).  Units are given
+ * one at a time to the device that would finish its share soonest with one more unit (ties: the
+ * lower device index), among the devices whose share still fits in mem_bytes[d] (nullable: no
+ * limit); for equal units this minimises the slowest device's time.  The shares are written as
+ * contiguous ranges in device order (ranges[n_devices]: query heads for ATTN, columns for FFN;
+ * a device may get an empty range), valid for vt_partition_create.  makespan (nullable) receives
+ * the slowest device's time in seconds.
+ * Errors: VT_ERR_INVALID_ARG (NULL shapes / rate / ranges, n_devices outside [1, VT_MAX_DEVICES],
+ * a rate that is not finite and positive, a negative or NaN budget, col_unit < 1 for FFN),
+ * VT_ERR_SHAPE (invalid shapes), VT_ERR_PLAN_MEMORY (some unit fits on no device).  Nothing is
+ * written on error. */
+VT_API vt_status vt_plan_tp_shares(const vt_shapes* shapes, vt_block block, int32_t n_devices,
+                                   const double* rate, const double* mem_bytes, int32_t col_unit,
+                                   vt_range* ranges, double* makespan);
 
 /* ---------------------------------------------------------------- model ------------------------
  * vt_model_create: allocates device storage for every layer in the canonical (unpartitioned)

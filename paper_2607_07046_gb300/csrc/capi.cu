@@ -16,6 +16,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -259,6 +260,66 @@ extern "C" vt_status vt_partition_validate(const vt_shapes* s, int32_t n, const 
     if (!heads || !cols) return fail(VT_ERR_INVALID_ARG, "range arrays must not be NULL");
     VT_TRY(check_ranges(heads, n, s->n_heads, s->n_heads / s->n_kv_heads, "head"));
     VT_TRY(check_ranges(cols, n, s->d_ffn, 1, "ffn column"));
+    return ok();
+}
+
+// ================================================================== planning
+
+// Heterogeneity-aware TP shares of one block (Voltron Section 4.2.1): equal units handed out one
+// at a time to the device that finishes soonest with one more, within the memory budgets.
+extern "C" vt_status vt_plan_tp_shares(const vt_shapes* s, vt_block block, int32_t n, const double* rate,
+                                       const double* mem, int32_t col_unit, vt_range* ranges,
+                                       double* makespan) {
+    if (!s || !rate || !ranges) return fail(VT_ERR_INVALID_ARG, "shapes, rate and ranges must not be NULL");
+    VT_TRY(vt_shapes_validate(s));
+    if (n < 1 || n > VT_MAX_DEVICES) return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
+    if (block != VT_BLOCK_ATTN && block != VT_BLOCK_FFN) return fail(VT_ERR_INVALID_ARG, "unknown block %d", (int)block);
+    for (int d = 0; d < n; ++d) {
+        if (!(rate[d] > 0.0) || !std::isfinite(rate[d]))
+            return fail(VT_ERR_INVALID_ARG, "rate[%d] must be finite and positive", d);
+        if (mem && !(mem[d] >= 0.0)) return fail(VT_ERR_INVALID_ARG, "mem_bytes[%d] must be >= 0", d);
+    }
+    const double D = s->d_model, dh = s->d_head;
+    const int g = s->n_heads / s->n_kv_heads;
+    int units, per_unit;   // units, and heads or columns per unit
+    double unit_bytes;
+    if (block == VT_BLOCK_ATTN) {
+        units = s->n_kv_heads;
+        per_unit = g;
+        // QKV rows (g query heads, one K and one V head), O columns, and the K / V cache
+        unit_bytes = 2.0 * ((g + 2) * dh * D + D * g * dh) + 2.0 * 2.0 * s->max_seq * dh;
+    } else {
+        if (col_unit < 1) return fail(VT_ERR_INVALID_ARG, "col_unit must be >= 1");
+        per_unit = col_unit;
+        units = (s->d_ffn + col_unit - 1) / col_unit;
+        unit_bytes = 2.0 * 3.0 * D * col_unit;  // gate, up and down columns
+    }
+    std::vector<int> cnt(n, 0);
+    for (int u = 0; u < units; ++u) {
+        int best = -1;
+        double best_t = 0.0;
+        for (int d = 0; d < n; ++d) {
+            if (mem && (cnt[d] + 1) * unit_bytes > mem[d]) continue;
+            const double t = (cnt[d] + 1) * unit_bytes / rate[d];
+            if (best < 0 || t < best_t) {
+                best = d;
+                best_t = t;
+            }
+        }
+        if (best < 0) return fail(VT_ERR_PLAN_MEMORY, "unit %d of %d fits on no device", u, units);
+        ++cnt[best];
+    }
+    const int total = block == VT_BLOCK_ATTN ? s->n_heads : s->d_ffn;
+    int at = 0;
+    double worst = 0.0;
+    for (int d = 0; d < n; ++d) {
+        const int e = std::min(total, at + cnt[d] * per_unit);
+        ranges[d].begin = at;
+        ranges[d].end = e;
+        at = e;
+        worst = std::max(worst, cnt[d] * unit_bytes / rate[d]);
+    }
+    if (makespan) *makespan = worst;
     return ok();
 }
 

@@ -27,6 +27,7 @@ VT_ERR_KV_CAPACITY = 7
 VT_ERR_CUDA = 8
 VT_ERR_ALLOC = 9
 VT_ERR_STATE = 10
+VT_ERR_PLAN_MEMORY = 11
 VT_MAX_DEVICES = 16
 VT_DEV_KV_OVERFLOW = 1
 VT_DEV_WAIT_TIMEOUT = 2
@@ -88,6 +89,9 @@ def lib() -> ctypes.CDLL:
             "vt_shapes_validate": (S, [ctypes.POINTER(vt_shapes)]),
             "vt_partition_validate": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(vt_range),
                                           ctypes.POINTER(vt_range)]),
+            "vt_plan_tp_shares": (S, [ctypes.POINTER(vt_shapes), _I32, _I32, ctypes.POINTER(ctypes.c_double),
+                                      ctypes.POINTER(ctypes.c_double), _I32, ctypes.POINTER(vt_range),
+                                      ctypes.POINTER(ctypes.c_double)]),
             "vt_model_create": (S, [ctypes.POINTER(vt_shapes), ctypes.POINTER(vt_layer_weights), _P,
                                     ctypes.POINTER(vt_allocator), _P, ctypes.POINTER(_P)]),
             "vt_model_load_layer": (S, [_P, _I32, ctypes.POINTER(vt_layer_weights), _P]),
@@ -207,6 +211,24 @@ def vt_partition_validate(shapes: vt_shapes, head_ranges, ffn_col_ranges) -> int
         raise ValueError("one head range and one FFN range per device")
     return int(lib().vt_partition_validate(ctypes.byref(shapes), n, _ranges(head_ranges),
                                            _ranges(ffn_col_ranges)))
+
+
+def vt_plan_tp_shares(shapes: vt_shapes, block: int, rate, mem_bytes=None, col_unit: int = 1):
+    """Heterogeneity-aware TP shares of one block: (ranges per device, makespan in seconds).
+    rate: bytes per second of each device; mem_bytes: per-device budget for the block's shard, or
+    None.  Raises VtError on a failed status."""
+    n = len(rate)
+    r = (ctypes.c_double * max(1, n))(*[float(x) for x in rate])
+    m = None
+    if mem_bytes is not None:
+        if len(mem_bytes) != n:
+            raise ValueError("one memory budget per device")
+        m = (ctypes.c_double * max(1, n))(*[float(x) for x in mem_bytes])
+    out = (vt_range * max(1, n))()
+    ms = ctypes.c_double(0.0)
+    _check(lib().vt_plan_tp_shares(ctypes.byref(shapes), int(block), n, r, m, int(col_unit), out,
+                                   ctypes.byref(ms)))
+    return [(out[d].begin, out[d].end) for d in range(n)], ms.value
 
 
 # ------------------------------------------------------------------ model

@@ -1,0 +1,164 @@
+"""Heterogeneity-aware tensor-parallel shares (Voltron Section 4.2.1: under TP, shards go to
+devices greedily by performance so that their execution times balance; within the memory budgets).
+Host only: vt_plan_tp_shares launches nothing.
+
+Pins: the 13B workload's stated 50/30/20 split of heads and FFN columns; even splits for equal
+devices; KV-group alignment under GQA; the minimum makespan over every split, by brute force, on
+small blocks; the block's bytes from the layer definition; memory budgets."""
+from __future__ import annotations
+
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+import synthetic
+
+
+def shapes(vt, wl, max_seq=None):
+    return vt.make_shapes(wl.n_layers, wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn,
+                          0, wl.kv_len + 8 if max_seq is None else max_seq, wl.rms_eps, wl.rope_theta)
+
+
+def block_bytes(wl, block, max_seq):
+    """fp16 bytes of a whole ATTN or FFN block of one layer, from the layer's definition."""
+    D, H, Hk, dh, F = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn
+    if block == 0:
+        wqkv = (H + 2 * Hk) * dh * D
+        wo = D * H * dh
+        cache = 2 * Hk * max_seq * dh
+        return 2 * (wqkv + wo + cache)
+    return 2 * 3 * D * F
+
+
+def sizes(ranges):
+    return [b - a for a, b in ranges]
+
+
+def contiguous(ranges, total):
+    at = 0
+    for a, b in ranges:
+        assert a == at and b >= a
+        at = b
+    assert at == total
+
+
+def test_13b_fifty_thirty_twenty(vtlib):
+    """Device rates 5:3:2 give the 13B workload's own partition: heads 20/12/8, FFN columns
+    6912/4147/2765 (the integer split of 13824 in that ratio with the smallest makespan)."""
+    wl = synthetic.WORKLOADS[3]
+    s = shapes(vtlib, wl)
+    heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, [5.0, 3.0, 2.0])
+    cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, [5.0, 3.0, 2.0])
+    assert heads == list(wl.head_ranges) == [(0, 20), (20, 32), (32, 40)]
+    assert cols == list(wl.ffn_ranges) == [(0, 6912), (6912, 11059), (11059, 13824)]
+    assert vtlib.vt_partition_validate(s, heads, cols) == vtlib.VT_OK
+
+
+def test_equal_devices_split_evenly(vtlib):
+    wl = synthetic.WORKLOADS[2]
+    s = shapes(vtlib, wl)
+    heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, [1.0] * 4)
+    cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, [1.0] * 4)
+    assert heads == list(wl.head_ranges) and cols == list(wl.ffn_ranges)
+
+
+def test_gqa_shares_are_whole_kv_groups(vtlib):
+    wl = synthetic.WORKLOADS[5]   # 32 query heads, 8 KV heads
+    s = shapes(vtlib, wl)
+    heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, [3.0, 1.0])
+    assert heads == [(0, 24), (24, 32)]
+    heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, [1.0, 1.0, 1.0, 1.0])
+    assert heads == list(wl.head_ranges)
+    for rates in ([7.0, 1.0, 2.5], [1.0, 100.0], [2.0, 2.0, 1.0, 0.5, 3.0]):
+        heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, rates)
+        assert all(a % 4 == 0 and b % 4 == 0 for a, b in heads)
+        cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates, col_unit=64)
+        assert vtlib.vt_partition_validate(s, heads, cols) == vtlib.VT_OK
+
+
+def test_one_device_takes_the_whole_block(vtlib):
+    """The makespan of a single device is the block's bytes (from the layer definition) over its rate."""
+    for cid in (1, 2, 5):
+        wl = synthetic.WORKLOADS[cid]
+        max_seq = wl.kv_len + 8
+        s = shapes(vtlib, wl, max_seq)
+        for block in (0, 1):
+            r, ms = vtlib.vt_plan_tp_shares(s, block, [2.5e12])
+            assert r == [(0, wl.n_heads if block == 0 else wl.d_ffn)]
+            assert ms == pytest.approx(block_bytes(wl, block, max_seq) / 2.5e12, rel=1e-12)
+
+
+def brute_force(units, rates, cap=None):
+    """Smallest makespan over every split of `units` equal units (unit time 1 / rate)."""
+    best = math.inf
+    n = len(rates)
+    for cuts in itertools.product(range(units + 1), repeat=n - 1):
+        c = list(cuts) + [units - sum(cuts)]
+        if c[-1] < 0:
+            continue
+        if cap is not None and any(c[d] > cap[d] for d in range(n)):
+            continue
+        best = min(best, max(c[d] / rates[d] for d in range(n)))
+    return best
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_greedy_reaches_the_brute_force_minimum(vtlib, seed):
+    rng = np.random.default_rng(500 + seed)
+    n = int(rng.integers(2, 4))
+    rates = [float(x) for x in rng.uniform(0.2, 5.0, n)]
+    F = int(rng.integers(1, 14))
+    s = vtlib.make_shapes(1, 256, 4, 4, 64, F, 0, 64)
+    cols, ms = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates)
+    contiguous(cols, F)
+    unit = 2 * 3 * 256
+    best = brute_force(F, rates)
+    assert ms == pytest.approx(best * unit, rel=1e-12)
+    assert max(c * unit / r for c, r in zip(sizes(cols), rates)) == pytest.approx(ms, rel=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_memory_budgets_are_respected_and_still_minimal(vtlib, seed):
+    rng = np.random.default_rng(700 + seed)
+    rates = [float(x) for x in rng.uniform(0.5, 4.0, 3)]
+    F = 12
+    unit = 2 * 3 * 256
+    cap = [int(x) for x in rng.integers(2, 9, 3)]
+    if sum(cap) < F:
+        cap[0] = F
+    s = vtlib.make_shapes(1, 256, 4, 4, 64, F, 0, 64)
+    cols, ms = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates, mem_bytes=[c * unit for c in cap])
+    contiguous(cols, F)
+    assert all(n <= c for n, c in zip(sizes(cols), cap))
+    assert ms == pytest.approx(brute_force(F, rates, cap) * unit, rel=1e-12)
+
+
+def test_the_fastest_device_fills_first_up_to_its_budget(vtlib):
+    s = vtlib.make_shapes(1, 256, 4, 4, 64, 100, 0, 64)
+    unit = 2 * 3 * 256
+    cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, [100.0, 1.0], mem_bytes=[30 * unit, 1e30])
+    assert sizes(cols) == [30, 70]
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, [1.0, 1.0], mem_bytes=[30 * unit, 60 * unit])
+    assert e.value.status == vtlib.VT_ERR_PLAN_MEMORY
+
+
+def test_column_units_and_a_short_last_unit(vtlib):
+    s = vtlib.make_shapes(1, 256, 4, 4, 64, 1000, 0, 64)
+    cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, [1.0, 1.0, 1.0], col_unit=64)
+    contiguous(cols, 1000)
+    assert all(a % 64 == 0 for a, _ in cols)
+    assert sizes(cols) == [384, 320, 296]   # 16 units of 64 (the last one 40 columns): 6 / 5 / 5
+
+
+@pytest.mark.parametrize("rates,kw", [
+    ([0.0, 1.0], {}), ([-1.0], {}), ([float("nan")], {}), ([float("inf")], {}), ([], {}),
+    ([1.0] * 17, {}), ([1.0], dict(col_unit=0)), ([1.0, 1.0], dict(mem_bytes=[1.0, float("nan")])),
+])
+def test_invalid_arguments(vtlib, rates, kw):
+    s = vtlib.make_shapes(1, 256, 4, 4, 64, 100, 0, 64)
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates, **kw)
+    assert e.value.status == vtlib.VT_ERR_INVALID_ARG
