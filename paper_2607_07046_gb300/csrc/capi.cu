@@ -169,10 +169,11 @@ struct vt_partition {
     __half* xbuf = nullptr;     // [kPrefillChunk][D]
     // prefill scratch
     __half* p_xhat = nullptr;   // [kPrefillChunk][D]
-    __half* p_q = nullptr;      // [kPrefillChunk][max_hq][dh]
-    __half* p_attn = nullptr;   // [kPrefillChunk][max_hq dh]
-    __half* p_u = nullptr;      // [kPrefillChunk][max_ld]
+    __half* p_q = nullptr;      // [n_dev] slots of [kPrefillChunk][max_hq][dh], q_slot halves apart
+    __half* p_attn = nullptr;   // [n_dev] slots of [kPrefillChunk][max_hq dh]
+    __half* p_u = nullptr;      // [n_dev] slots of [kPrefillChunk][max_ld], u_slot halves apart
     int max_hq = 0, max_ld = 0;
+    size_t q_slot = 0, u_slot = 0;
     // persistent decode-token kernel: shapes and scratch (the KV object adds its tables)
     bool tok_ok = false;
     std::string tok_why;
@@ -649,9 +650,11 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     // ------------------------------------------------------------------ stack + prefill scratch
     {
         const size_t R = kPrefillChunk;
+        // q, attention output and u: one slot per shard, so the shards of a block run together
+        p->q_slot = align256(R * std::max(p->max_hq, 1) * dh * 2) / 2;
+        p->u_slot = align256(R * std::max(p->max_ld, 8) * 2) / 2;
         const size_t bytes = align256(4) + align256((size_t)n * D * 4) + align256((size_t)n * R * D * 4) + 2 * align256(R * D * 2) +
-                             align256(R * D * 2) + 2 * align256(R * std::max(p->max_hq, 1) * dh * 2) +
-                             align256(R * std::max(p->max_ld, 8) * 2);
+                             align256(R * D * 2) + 2 * (size_t)n * p->q_slot * 2 + (size_t)n * p->u_slot * 2;
         void* q;
         if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
         Bump b{static_cast<uint8_t*>(q)};
@@ -661,9 +664,9 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         p->hbuf = b.take<__half>(R * D);
         p->xbuf = b.take<__half>(R * D);
         p->p_xhat = b.take<__half>(R * D);
-        p->p_q = b.take<__half>(R * std::max(p->max_hq, 1) * dh);
-        p->p_attn = b.take<__half>(R * std::max(p->max_hq, 1) * dh);
-        p->p_u = b.take<__half>(R * std::max(p->max_ld, 8));
+        p->p_q = b.take<__half>((size_t)n * p->q_slot);
+        p->p_attn = b.take<__half>((size_t)n * p->q_slot);
+        p->p_u = b.take<__half>((size_t)n * p->u_slot);
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
     }
     // ------------------------------------------------------------------ decode-token kernel
@@ -1171,8 +1174,62 @@ extern "C" vt_status vt_combine(const float* const* partials, int32_t n, int32_t
 
 // ------------------------------------------------------------------ prefill
 
-// xhat_ready: the partition's xhat scratch already holds RMSNorm(x) with this block's gain (the
-// whole-stack path computes it once per block, in the combine that produced x).
+// Arguments of one shard's prefill.  xhat_ready: the partition's xhat scratch already holds
+// RMSNorm(x) with this block's gain (the whole-stack path computes it once per block, in the
+// combine that produced x).  slot: the shard's q / attention / u scratch slot.
+static void attn_args(const vt_partition* p, vt_shard sh, const __half* x, int n, vt_kv* kv, float* out,
+                      int row_offset, bool xhat_ready, int slot, PrefillAttnArgs* t) {
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(sh.layer, sh.device);
+    *t = PrefillAttnArgs{};
+    t->n = n;
+    t->d = s.d_model;
+    t->dh = s.d_head;
+    t->hq = a.h1 - a.h0;
+    t->hk = a.kv1 - a.kv0;
+    t->eps = s.rms_eps;
+    t->scale_log2 = (float)(1.4426950408889634 / sqrt((double)s.d_head));
+    t->x = x;
+    t->gain = a.norm;
+    t->wqkv = a.wqkv;
+    t->wo = a.wo;
+    t->kcache = kv->k(sh.layer, sh.device);
+    t->vcache = kv->v(sh.layer, sh.device);
+    t->cap = kv->cap;
+    t->len = kv->len + sh.layer;
+    t->row_offset = row_offset;
+    t->rope = p->m->rope;
+    t->xhat = p->p_xhat;
+    t->xhat_ready = xhat_ready;
+    t->q = p->p_q + (size_t)slot * p->q_slot;
+    t->attn = p->p_attn + (size_t)slot * p->q_slot;
+    t->out = out;
+    t->status = kv->status;
+}
+
+static void ffn_args(const vt_partition* p, vt_shard sh, const __half* x, int n, float* out, bool xhat_ready,
+                     int slot, PrefillFfnArgs* t) {
+    const vt_shapes& s = p->m->s;
+    const FfnShard& f = p->f(sh.layer, sh.device);
+    *t = PrefillFfnArgs{};
+    t->n = n;
+    t->d = s.d_model;
+    t->c = f.c1 - f.c0;
+    t->eps = s.rms_eps;
+    t->x = x;
+    t->gain = f.norm;
+    t->wgu = f.wgu;
+    t->ushift = f.c0 % 8;
+    t->wd = p->m->layer[sh.layer].w_down + (f.c0 - t->ushift);
+    t->wd_ld = s.d_ffn;
+    t->ldu = p->max_ld;
+    t->xhat = p->p_xhat;
+    t->xhat_ready = xhat_ready;
+    t->u = p->p_u + (size_t)slot * p->u_slot;
+    t->out = out;
+    t->status = p->status;
+}
+
 static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half* x, int n, vt_kv* kv,
                                float* out, int row_offset, cudaStream_t st, bool xhat_ready = false) {
     const vt_shapes& s = p->m->s;
@@ -1180,65 +1237,54 @@ static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half*
     std::string err;
     if (sh.block == VT_BLOCK_ATTN) {
         const AttnShard& a = p->a(sh.layer, sh.device);
-        const int hq = a.h1 - a.h0;
-        if (hq == 0) {
+        if (a.h1 == a.h0) {
             VT_CUDA(launch_fill_zero_f32(out, (int64_t)n * D, st));
             return VT_OK;
         }
-        PrefillAttnArgs t{};
-        t.n = n;
-        t.d = D;
-        t.dh = s.d_head;
-        t.hq = hq;
-        t.hk = a.kv1 - a.kv0;
-        t.eps = s.rms_eps;
-        t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)s.d_head));
-        t.x = x;
-        t.gain = a.norm;
-        t.wqkv = a.wqkv;
-        t.wo = a.wo;
-        t.kcache = kv->k(sh.layer, sh.device);
-        t.vcache = kv->v(sh.layer, sh.device);
-        t.cap = kv->cap;
-        t.len = kv->len + sh.layer;
-        t.row_offset = row_offset;
-        t.rope = p->m->rope;
-        t.xhat = p->p_xhat;
-        t.xhat_ready = xhat_ready;
-        t.q = p->p_q;
-        t.attn = p->p_attn;
-        t.out = out;
-        t.status = kv->status;
+        PrefillAttnArgs t;
+        attn_args(p, sh, x, n, kv, out, row_offset, xhat_ready, 0, &t);
         vt_status r = prefill_attn_shard(t, st, &err);
         if (r != VT_OK) return fail(r, "%s", err.c_str());
     } else {
         const FfnShard& f = p->f(sh.layer, sh.device);
-        const int c = f.c1 - f.c0;
-        if (c == 0) {
+        if (f.c1 == f.c0) {
             VT_CUDA(launch_fill_zero_f32(out, (int64_t)n * D, st));
             return VT_OK;
         }
         if (s.d_ffn % 8 != 0) return fail(VT_ERR_SHAPE, "prefill needs d_ffn to be a multiple of 8");
-        PrefillFfnArgs t{};
-        t.n = n;
-        t.d = D;
-        t.c = c;
-        t.eps = s.rms_eps;
-        t.x = x;
-        t.gain = f.norm;
-        t.wgu = f.wgu;
-        t.ushift = f.c0 % 8;
-        t.wd = p->m->layer[sh.layer].w_down + (f.c0 - t.ushift);
-        t.wd_ld = s.d_ffn;
-        t.ldu = p->max_ld;
-        t.xhat = p->p_xhat;
-        t.xhat_ready = xhat_ready;
-        t.u = p->p_u;
-        t.out = out;
-        t.status = p->status;
+        PrefillFfnArgs t;
+        ffn_args(p, sh, x, n, out, xhat_ready, 0, &t);
         vt_status r = prefill_ffn_shard(t, st, &err);
         if (r != VT_OK) return fail(r, "%s", err.c_str());
     }
+    return VT_OK;
+}
+
+// Every shard of one block of layer l, on `rows` rows whose normalised input is in p_xhat: the
+// shards' GEMMs run as one launch per GEMM of the block (empty shards get a zero partial).
+static vt_status prefill_block(const vt_partition* p, int l, vt_block block, const __half* x, int rows, vt_kv* kv,
+                               int row_offset, cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const int D = s.d_model;
+    PrefillAttnArgs at[VT_MAX_DEVICES];
+    PrefillFfnArgs ft[VT_MAX_DEVICES];
+    int n = 0;
+    for (int d = 0; d < p->n_dev; ++d) {
+        float* out = p->partials + (size_t)d * kPrefillChunk * D;
+        const vt_shard sh{l, d, block};
+        const bool empty = block == VT_BLOCK_ATTN ? p->a(l, d).h1 == p->a(l, d).h0 : p->f(l, d).c1 == p->f(l, d).c0;
+        if (empty) {
+            VT_CUDA(launch_fill_zero_f32(out, (int64_t)rows * D, st));
+            continue;
+        }
+        if (block == VT_BLOCK_ATTN) attn_args(p, sh, x, rows, kv, out, row_offset, true, d, &at[n++]);
+        else ffn_args(p, sh, x, rows, out, true, d, &ft[n++]);
+    }
+    if (block == VT_BLOCK_FFN && n > 0 && s.d_ffn % 8 != 0)
+        return fail(VT_ERR_SHAPE, "prefill needs d_ffn to be a multiple of 8");
+    std::string err;
+    const vt_status r = block == VT_BLOCK_ATTN ? prefill_attn_group(at, n, st, &err) : prefill_ffn_group(ft, n, st, &err);
+    if (r != VT_OK) return fail(r, "%s", err.c_str());
     return VT_OK;
 }
 
@@ -1371,19 +1417,11 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
         // per block, fused into the combine that produced the block's input.
         VT_CUDA(launch_rmsnorm_rows(cur, p->m->layer[0].attn_norm, s.rms_eps, rows, D, p->p_xhat, st));
         for (int l = 0; l < s.n_layers; ++l) {
-            for (int d = 0; d < nd; ++d) {
-                vt_shard sh{l, d, VT_BLOCK_ATTN};
-                VT_TRY(prefill_shard(p, sh, cur, rows, kv, p->partials + (size_t)d * kPrefillChunk * D,
-                                     r0, st, true));
-            }
+            VT_TRY(prefill_block(p, l, VT_BLOCK_ATTN, cur, rows, kv, r0, st));
             c.residual = cur;
             c.out = p->hbuf;
             VT_CUDA(launch_combine_norm(c, rows, D, p->m->layer[l].ffn_norm, s.rms_eps, p->p_xhat, st));
-            for (int d = 0; d < nd; ++d) {
-                vt_shard sh{l, d, VT_BLOCK_FFN};
-                VT_TRY(prefill_shard(p, sh, p->hbuf, rows, kv,
-                                     p->partials + (size_t)d * kPrefillChunk * D, r0, st, true));
-            }
+            VT_TRY(prefill_block(p, l, VT_BLOCK_FFN, p->hbuf, rows, kv, r0, st));
             const bool last = l == s.n_layers - 1;
             __half* dst = last ? static_cast<__half*>(x_out) + (size_t)r0 * D : p->xbuf;
             c.residual = p->hbuf;

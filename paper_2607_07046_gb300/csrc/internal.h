@@ -179,6 +179,10 @@ struct PrefillFfnArgs {
     uint32_t* status;
 };
 vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err);
+// the shards of one block at once (all with the same rows and normalised input): one launch per
+// GEMM of the block for every shard
+vt_status prefill_attn_group(const PrefillAttnArgs* a, int n, cudaStream_t st, std::string* err);
+vt_status prefill_ffn_group(const PrefillFfnArgs* a, int n, cudaStream_t st, std::string* err);
 // rows x d: out = fp16(residual + sum of partials); with gain, also xhat = RMSNorm(out) * gain
 cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __half* gain, float eps, __half* xhat,
                                 cudaStream_t st);

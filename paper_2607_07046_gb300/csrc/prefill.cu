@@ -265,6 +265,17 @@ struct GemmArgs {
     uint32_t* status;
 };
 
+// Up to kGemmGroups independent GEMMs of the same row count in one launch (the shards of one
+// block, which share M and often A): group g owns the CTAs with blockIdx.x in
+// [tile_end[g - 1], tile_end[g]), one per 256-column tile of its N.
+constexpr int kGemmGroups = 8;
+struct GemmGroup {
+    int n_groups;
+    int tile_end[kGemmGroups];
+    CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
+    GemmArgs a[kGemmGroups];
+};
+
 // 16-byte slot of the split-K receive buffer that holds floats [4e, 4e + 4) of 32-column chunk
 // `chunk` of local row `lr`.  128-bit shared accesses are served 8 threads at a time; the slot
 // permutation keeps those 8 threads on distinct banks both for the writer (8 consecutive rows, one
@@ -326,8 +337,12 @@ __device__ __forceinline__ void gemm_epilogue_quad(const GemmArgs& a, int row, i
 // Every wait is bounded; on a timeout the kernel sets VT_DEV_WAIT_TIMEOUT, stops issuing, waits
 // for the copies it issued, still reaches both cluster barriers, frees tensor memory and ends.
 template <int EPI>
-__global__ void __launch_bounds__(kGemmThreads, 1)
-    k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, const __grid_constant__ GemmArgs a) {
+__global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant__ GemmGroup G) {
+    int g = 0;
+    while (g + 1 < G.n_groups && (int)blockIdx.x >= G.tile_end[g]) ++g;
+    const CUtensorMap& ta = G.ta[g];
+    const CUtensorMap& tb = G.tb[g];
+    const GemmArgs& a = G.a[g];
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
@@ -337,7 +352,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __shared__ int s_err;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * kBN, m0 = blockIdx.y * kBM;
+    const int n0 = ((int)blockIdx.x - (g > 0 ? G.tile_end[g - 1] : 0)) * kBN, m0 = blockIdx.y * kBM;
     const int S = gridDim.z, z = blockIdx.z;
     const int kt0 = (int)((int64_t)a.k_tiles * z / S), kt1 = (int)((int64_t)a.k_tiles * (z + 1) / S);
     const int nk = kt1 - kt0;
@@ -785,12 +800,14 @@ static bool make_map(CUtensorMap* map, const void* base, int64_t inner, int64_t 
 // Split factor for `tiles` output tiles of `k_tiles` k-tiles, from a time model of one launch:
 // per wave, a fixed cost (first loads, epilogue) plus the k-tiles of one split; with S > 1, the
 // cluster reduction of the accumulators.  The constants are measured on GB300 (microseconds).
-static int choose_split(int tiles, int k_tiles) {
+// k_tiles: the longest GEMM of the launch (its time); min_k_tiles: the shortest, which must still
+// give every CTA of a split at least 4 k-tiles (a CTA without k-tiles has no accumulator).
+static int choose_split(int tiles, int k_tiles, int min_k_tiles) {
     constexpr double kTile = 0.33, kFixed = 4.0, kReduce = 3.5;
     int best = 1;
     double best_t = 1e30;
     for (int s = 1; s <= kMaxSplit; ++s) {
-        if (s > 1 && k_tiles / s < 4) break;
+        if (s > 1 && min_k_tiles / s < 4) break;
         const int per_wave = s == 1 ? g_num_sms : g_split_clusters[s];
         if (per_wave < 1) continue;
         const int waves = (tiles + per_wave - 1) / per_wave;
@@ -803,37 +820,71 @@ static int choose_split(int tiles, int k_tiles) {
     return best;
 }
 
+// One GEMM of a grouped launch: C_g = A_g . B_g^T with m rows (shared by the group), n_g columns
+// and k_g inner elements; `base` carries the epilogue's pointers.
+struct GemmSpec {
+    const void* A;
+    int64_t lda;
+    const void* B;
+    int64_t ldb;
+    int n, k;
+    GemmArgs base;
+};
+
+// Launches the GEMMs of `specs` (all with m rows) kGemmGroups at a time, one CTA (or split-K
+// cluster) per output tile of every GEMM: the shards of a block fill the GPU together instead of
+// a few tiles each.
+template <int EPI>
+static vt_status run_gemm_group(const GemmSpec* specs, int n_specs, int m, cudaStream_t st, std::string* err) {
+    for (int g0 = 0; g0 < n_specs; g0 += kGemmGroups) {
+        const int ng = std::min(kGemmGroups, n_specs - g0);
+        GemmGroup G{};
+        G.n_groups = ng;
+        int tiles_n = 0, max_k_tiles = 1, min_k_tiles = 1 << 30;
+        for (int g = 0; g < ng; ++g) {
+            const GemmSpec& sp = specs[g0 + g];
+            if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) || !make_map(&G.tb[g], sp.B, sp.k, sp.n, sp.ldb, kBN, err))
+                return VT_ERR_INVALID_ARG;
+            GemmArgs& a = G.a[g];
+            a = sp.base;
+            a.m = m;
+            a.n = sp.n;
+            a.b = static_cast<const __half*>(sp.B);
+            a.ldb = sp.ldb;
+            a.k_tiles = (sp.k + kBK - 1) / kBK;
+            max_k_tiles = std::max(max_k_tiles, a.k_tiles);
+            min_k_tiles = std::min(min_k_tiles, a.k_tiles);
+            tiles_n += (sp.n + kBN - 1) / kBN;
+            G.tile_end[g] = tiles_n;
+        }
+        const int tiles_m = (m + kBM - 1) / kBM;
+        const int split = choose_split(tiles_n * tiles_m, max_k_tiles, min_k_tiles);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(tiles_n, tiles_m, split);
+        cfg.blockDim = dim3(kGemmThreads);
+        cfg.dynamicSmemBytes = kGemmSmem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 1;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = split;
+        cfg.attrs = attr;
+        cfg.numAttrs = split > 1 ? 1 : 0;
+        const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm<EPI>, G);
+        if (e != cudaSuccess) {
+            *err = std::string("GEMM launch failed: ") + cudaGetErrorString(e);
+            return VT_ERR_CUDA;
+        }
+    }
+    return VT_OK;
+}
+
 template <int EPI>
 static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb, int m, int n, int k,
                           const GemmArgs& base, cudaStream_t st, std::string* err) {
-    CUtensorMap ta, tb;
-    if (!make_map(&ta, A, k, m, lda, kBM, err) || !make_map(&tb, B, k, n, ldb, kBN, err)) return VT_ERR_INVALID_ARG;
-    GemmArgs a = base;
-    a.m = m;
-    a.n = n;
-    a.b = static_cast<const __half*>(B);
-    a.ldb = ldb;
-    a.k_tiles = (k + kBK - 1) / kBK;
-    const int tiles_n = (n + kBN - 1) / kBN, tiles_m = (m + kBM - 1) / kBM;
-    const int split = choose_split(tiles_n * tiles_m, a.k_tiles);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(tiles_n, tiles_m, split);
-    cfg.blockDim = dim3(kGemmThreads);
-    cfg.dynamicSmemBytes = kGemmSmem;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = split;
-    cfg.attrs = attr;
-    cfg.numAttrs = split > 1 ? 1 : 0;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm<EPI>, ta, tb, a);
-    if (e != cudaSuccess) {
-        *err = std::string("GEMM launch failed: ") + cudaGetErrorString(e);
-        return VT_ERR_CUDA;
-    }
-    return VT_OK;
+    const GemmSpec sp{A, lda, B, ldb, n, k, base};
+    return run_gemm_group<EPI>(&sp, 1, m, st, err);
 }
 
 cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
@@ -853,9 +904,7 @@ static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int
     return VT_OK;
 }
 
-vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {
-    vt_status r;
-    if (!a.xhat_ready && (r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
+static GemmSpec qkv_spec(const PrefillAttnArgs& a) {
     GemmArgs g{};
     g.q = a.q;
     g.kcache = a.kcache;
@@ -868,9 +917,19 @@ vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::str
     g.row_offset = a.row_offset;
     g.rope = a.rope;
     g.status = a.status;
-    if ((r = run_gemm<kGemmQkv>(a.xhat, a.d, a.wqkv, a.d, a.n, (a.hq + 2 * a.hk) * a.dh, a.d, g, st, err)) != VT_OK)
-        return r;
+    return GemmSpec{a.xhat, a.d, a.wqkv, a.d, (a.hq + 2 * a.hk) * a.dh, a.d, g};
+}
 
+static GemmSpec o_spec(const PrefillAttnArgs& a) {
+    GemmArgs o{};
+    o.c = a.out;
+    o.ldc = a.d;
+    o.status = a.status;
+    const int K = a.hq * a.dh;
+    return GemmSpec{a.attn, K, a.wo, K, a.d, K, o};
+}
+
+static vt_status prefill_attention(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {
     PrefillAttnKArgs t{};
     t.q = a.q;
     t.kcache = a.kcache;
@@ -891,30 +950,58 @@ vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::str
         *err = std::string("prefill attention launch failed: ") + cudaGetErrorString(e);
         return VT_ERR_CUDA;
     }
+    return VT_OK;
+}
 
-    GemmArgs o{};
-    o.c = a.out;
-    o.ldc = a.d;
-    o.status = a.status;
-    return run_gemm<kGemmF32>(a.attn, (int64_t)a.hq * a.dh, a.wo, (int64_t)a.hq * a.dh, a.n, a.d, a.hq * a.dh, o, st,
-                              err);
+vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {
+    return prefill_attn_group(&a, 1, st, err);
+}
+
+// The shards of one ATTN block: one QKV launch for all of them, their attention, one O launch.
+// Every shard has its own q, attention and output buffers; they share the normalised input.
+vt_status prefill_attn_group(const PrefillAttnArgs* a, int n, cudaStream_t st, std::string* err) {
+    if (n < 1) return VT_OK;
+    vt_status r;
+    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, st, err)) != VT_OK)
+        return r;
+    GemmSpec specs[VT_MAX_DEVICES];
+    for (int i = 0; i < n; ++i) specs[i] = qkv_spec(a[i]);
+    if ((r = run_gemm_group<kGemmQkv>(specs, n, a[0].n, st, err)) != VT_OK) return r;
+    for (int i = 0; i < n; ++i)
+        if ((r = prefill_attention(a[i], st, err)) != VT_OK) return r;
+    for (int i = 0; i < n; ++i) specs[i] = o_spec(a[i]);
+    return run_gemm_group<kGemmF32>(specs, n, a[0].n, st, err);
 }
 
 vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::string* err) {
+    return prefill_ffn_group(&a, 1, st, err);
+}
+
+// The shards of one FFN block: one gate/up (+ SwiGLU) launch and one down launch for all of them.
+vt_status prefill_ffn_group(const PrefillFfnArgs* a, int n, cudaStream_t st, std::string* err) {
+    if (n < 1) return VT_OK;
     vt_status r;
-    if (!a.xhat_ready && (r = run_rmsnorm(a.x, a.gain, a.eps, a.n, a.d, a.xhat, st, err)) != VT_OK) return r;
-    GemmArgs g{};
-    g.u = a.u;
-    g.ldu = a.ldu;
-    g.ushift = a.ushift;
-    g.status = a.status;
-    if ((r = run_gemm<kGemmSwiglu>(a.xhat, a.d, a.wgu, a.d, a.n, 2 * a.c, a.d, g, st, err)) != VT_OK) return r;
-    GemmArgs o{};
-    o.c = a.out;
-    o.ldc = a.d;
-    o.status = a.status;
-    // K runs over the shifted columns [0, ushift + c) of U and the same columns of Wd from wd
-    return run_gemm<kGemmF32>(a.u, a.ldu, a.wd, a.wd_ld, a.n, a.d, a.ushift + a.c, o, st, err);
+    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, st, err)) != VT_OK)
+        return r;
+    GemmSpec specs[VT_MAX_DEVICES];
+    for (int i = 0; i < n; ++i) {
+        GemmArgs g{};
+        g.u = a[i].u;
+        g.ldu = a[i].ldu;
+        g.ushift = a[i].ushift;
+        g.status = a[i].status;
+        specs[i] = GemmSpec{a[i].xhat, a[i].d, a[i].wgu, a[i].d, 2 * a[i].c, a[i].d, g};
+    }
+    if ((r = run_gemm_group<kGemmSwiglu>(specs, n, a[0].n, st, err)) != VT_OK) return r;
+    for (int i = 0; i < n; ++i) {
+        GemmArgs o{};
+        o.c = a[i].out;
+        o.ldc = a[i].d;
+        o.status = a[i].status;
+        // K runs over the shifted columns [0, ushift + c) of U and the same columns of Wd from wd
+        specs[i] = GemmSpec{a[i].u, a[i].ldu, a[i].wd, a[i].wd_ld, a[i].d, a[i].ushift + a[i].c, o};
+    }
+    return run_gemm_group<kGemmF32>(specs, n, a[0].n, st, err);
 }
 
 }  // namespace vt

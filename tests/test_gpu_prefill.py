@@ -234,6 +234,37 @@ def test_prefill_tokens_two_layer_stack(vtlib):
                 assert_close(vg, caches[l][1][k0:k1, :n], f"layer {l} v dev {d}")
 
 
+@pytest.mark.parametrize("H,Hk,heads,cols", UNEVEN)
+def test_prefill_tokens_uneven_and_gqa_partitions(vtlib, H, Hk, heads, cols):
+    """vt_prefill_tokens runs every shard of a block in one launch per GEMM: uneven, empty and GQA
+    partitions through two layers against the oracle chained layer by layer."""
+    vt = vtlib
+    wl = synthetic.small("uneven-stack", n_layers=2, d_model=512, n_heads=H, n_kv_heads=Hk, d_head=64,
+                         d_ffn=1408, head_ranges=heads, ffn_ranges=cols, kv_len=0, decode_steps=1,
+                         prompt_len=140, model_id=92)
+    n, cap = 140, 160
+    X = wl.hidden(n, stream=10)
+    ref = X
+    caches = []
+    for l in range(2):
+        kc, vc = oracle.new_cache(wl, cap)
+        _, ref, _, _ = oracle.tp_layer(wl, wl.layer_weights(l), ref, 0, kc, vc)
+        caches.append((kc, vc))
+    with build(vt, wl, cap) as st:
+        out = torch.empty((n, wl.d_model), dtype=torch.float16, device="cuda")
+        vt.vt_prefill_tokens(st.part, st.kv, dev(X), n, out)
+        assert_close(host(out), ref, f"prefill stack H={H} Hk={Hk} {heads}")
+        for l in range(2):
+            for d, hr in enumerate(wl.head_ranges):
+                k0, k1 = kv_range(wl, hr)
+                if k1 == k0:
+                    continue
+                kg, vg = vt.vt_kv_read(st.kv, l, d, n, k1 - k0, wl.d_head)
+                assert_close(kg, caches[l][0][k0:k1, :n], f"layer {l} k dev {d}")
+                assert_close(vg, caches[l][1][k0:k1, :n], f"layer {l} v dev {d}")
+        assert vt.vt_kv_status(st.kv) == 0 and vt.vt_partition_status(st.part) == 0
+
+
 def test_decode_after_prefill_equals_longer_prefill(vtlib):
     """GPU only: decoding token M after a prefill of M rows gives row M of a prefill of M + 1 rows."""
     vt = vtlib
