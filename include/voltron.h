@@ -317,7 +317,8 @@ VT_API vt_status vt_combine(const float* const* partials, int32_t n, int32_t row
  *   launch (one CTA per SM): each CTA streams its share of every shard's weights and cached K/V
  *   through a shared-memory ring, shards are processed in order within each phase, and the CTAs
  *   meet at four grid barriers per layer.  Results equal the per-shard kernels' within fp32
- *   rounding (the FFN partials are summed with atomics, so they repeat only to fp32 rounding).
+ *   rounding (the FFN partials are summed by bulk reductions in the L2 in arrival order, so they
+ *   repeat only to fp32 rounding).
  *   Every wait in that kernel is bounded: a CTA that gives up sets VT_DEV_WAIT_TIMEOUT in the KV
  *   status word, the token's output is then undefined, and vt_kv_status(..., clear = 1) (or
  *   vt_partition_status) must be called before the next token to re-arm the grid barrier.

@@ -12,7 +12,8 @@
 // matrix-vector products: as separate kernels that is hundreds of launches of 5-20 us, and the
 // ramp-up and tail of each leave HBM idle for a large share of the token.  Here every CTA (one
 // per SM) streams a fixed slice of every layer's weights, and of the cached K/V rows, through a
-// ring of shared-memory stages that a producer warp fills with bulk copies.  The copies depend on
+// ring of shared-memory stages that a producer warp (the one working warp of a third warpgroup,
+// which hands its registers to the consumers) fills with bulk copies.  The copies depend on
 // nothing the token computes, so the producer runs ahead of the arithmetic.  Eight consumer warps
 // do the arithmetic and meet the other CTAs at four grid barriers per layer (after QKV, after
 // attention, after O, after the FFN); while they wait, the ring keeps filling.
