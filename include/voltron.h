@@ -165,6 +165,37 @@ VT_API vt_status vt_plan_tp_shares(const vt_shapes* shapes, vt_block block, int3
                                    const double* rate, const double* mem_bytes, int32_t col_unit,
                                    vt_range* ranges, double* makespan);
 
+/* vt_plan_layers: the layer-wise hybrid parallelism plan (Voltron Section 4.2.1): the blocks of
+ * the stack (ATTN then FFN of layer 0, then of layer 1, ...) are planned one after another.  For
+ * each block both strategies are estimated and the one with the lower time is kept (ties: MP):
+ *   MP: the whole block on the device with the highest rate whose remaining memory holds it; if the
+ *       activations are on another device they are sent first (one transfer of tokens * D fp16).
+ *   TP: shares from vt_plan_tp_shares on the remaining memory; the device holding the input
+ *       broadcasts it once (one transfer), the devices with a share compute at the same time, and
+ *       every other participant sends its fp32 partial [tokens * D] back to it (one transfer each,
+ *       one after another: the devices share one link).  The input holder keeps the activations.
+ * A transfer of b bytes takes link_latency_s + b / link_bytes_per_s.  A device's compute time for
+ * its part of a block is max(bytes / rate[d], flops / flop_rate[d]) (flop_rate nullable: bytes
+ * only), where bytes are its fp16 weights plus, for ATTN, the K / V rows read at kv_len and
+ * written for the `tokens` new rows, and flops are 2 per weight per token plus the attention
+ * scores and weighted values over kv_len + tokens positions.  Memory (mem_bytes nullable: no
+ * limit) holds weights and the K / V cache at max_seq.  The input starts on device 0.
+ * plans[2 * n_layers] receives the plan of every block (ATTN of layer l at 2 l, FFN at 2 l + 1);
+ * total_s (nullable) the sum of the blocks' compute and transfer times.
+ * Errors: as vt_plan_tp_shares, plus VT_ERR_INVALID_ARG for tokens < 1, kv_len < 0 or
+ * kv_len + tokens > max_seq, or a link rate that is not finite and positive or a negative latency;
+ * VT_ERR_PLAN_MEMORY when a block fits under neither strategy. */
+typedef struct {
+    int32_t tp;                      /* 0: MP, 1: TP */
+    int32_t device;                  /* MP: the device; TP: the input holder, which gathers the partials */
+    vt_range ranges[VT_MAX_DEVICES]; /* query heads (ATTN) or FFN columns of each device */
+    double compute_s, comm_s;        /* slowest participant's compute; transfers */
+} vt_block_plan;
+VT_API vt_status vt_plan_layers(const vt_shapes* shapes, int32_t n_devices, const double* rate,
+                                const double* flop_rate, const double* mem_bytes, double link_bytes_per_s,
+                                double link_latency_s, int32_t tokens, int32_t kv_len, vt_block_plan* plans,
+                                double* total_s);
+
 /* ---------------------------------------------------------------- model ------------------------
  * vt_model_create: allocates device storage for every layer in the canonical (unpartitioned)
  * layout, the RoPE table for positions [0, max_seq) and, if vocab > 0, the embedding table, on

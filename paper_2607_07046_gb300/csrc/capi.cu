@@ -17,6 +17,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <limits>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -266,8 +267,83 @@ extern "C" vt_status vt_partition_validate(const vt_shapes* s, int32_t n, const 
 
 // ================================================================== planning
 
-// Heterogeneity-aware TP shares of one block (Voltron Section 4.2.1): equal units handed out one
-// at a time to the device that finishes soonest with one more, within the memory budgets.
+namespace {
+
+// A block cut into equal units (Voltron Section 4.2.1 assigns TP shards greedily by device
+// performance): KV groups for ATTN, `col_unit` FFN columns for FFN.
+struct BlockUnits {
+    int units, per_unit, total;  // units; heads or columns per unit; heads or columns of the block
+    double mem;                  // fp16 bytes a unit occupies (weights, and the K / V cache at max_seq)
+    double wbytes;               // weight bytes of a unit
+    int kv_heads;                // KV heads of a unit (ATTN: 1)
+};
+
+BlockUnits block_units(const vt_shapes& s, vt_block block, int col_unit) {
+    const double D = s.d_model, dh = s.d_head;
+    const int g = s.n_heads / s.n_kv_heads;
+    BlockUnits b{};
+    if (block == VT_BLOCK_ATTN) {
+        b.units = s.n_kv_heads;
+        b.per_unit = g;
+        b.total = s.n_heads;
+        b.wbytes = 2.0 * ((g + 2) * dh * D + D * g * dh);  // QKV rows and O columns
+        b.mem = b.wbytes + 2.0 * 2.0 * s.max_seq * dh;     // + its K and V cache
+        b.kv_heads = 1;
+    } else {
+        b.units = (s.d_ffn + col_unit - 1) / col_unit;
+        b.per_unit = col_unit;
+        b.total = s.d_ffn;
+        b.wbytes = 2.0 * 3.0 * D * col_unit;  // gate, up and down columns
+        b.mem = b.wbytes;
+        b.kv_heads = 0;
+    }
+    return b;
+}
+
+// Units one at a time to the device that finishes soonest with one more (unit time t[d]; ties:
+// the lower index), among those whose remaining memory still holds one more.  False if a unit fits
+// nowhere.  For equal units on devices of different speeds this minimises the largest time.
+bool greedy_shares(int units, double unit_mem, int n, const double* t, const double* mem_left, int* cnt) {
+    for (int d = 0; d < n; ++d) cnt[d] = 0;
+    for (int u = 0; u < units; ++u) {
+        int best = -1;
+        double best_t = 0.0;
+        for (int d = 0; d < n; ++d) {
+            if (mem_left && (cnt[d] + 1) * unit_mem > mem_left[d]) continue;
+            const double tt = (cnt[d] + 1) * t[d];
+            if (best < 0 || tt < best_t) {
+                best = d;
+                best_t = tt;
+            }
+        }
+        if (best < 0) return false;
+        ++cnt[best];
+    }
+    return true;
+}
+
+void shares_to_ranges(int n, const int* cnt, int per_unit, int total, vt_range* r) {
+    int at = 0;
+    for (int d = 0; d < n; ++d) {
+        const int e = std::min(total, at + cnt[d] * per_unit);
+        r[d].begin = at;
+        r[d].end = e;
+        at = e;
+    }
+}
+
+vt_status check_rates(int n, const double* rate, const double* mem) {
+    for (int d = 0; d < n; ++d) {
+        if (!(rate[d] > 0.0) || !std::isfinite(rate[d]))
+            return fail(VT_ERR_INVALID_ARG, "rate[%d] must be finite and positive", d);
+        if (mem && !(mem[d] >= 0.0)) return fail(VT_ERR_INVALID_ARG, "mem_bytes[%d] must be >= 0", d);
+    }
+    return VT_OK;
+}
+
+}  // namespace
+
+// Heterogeneity-aware TP shares of one block (Voltron Section 4.2.1).
 extern "C" vt_status vt_plan_tp_shares(const vt_shapes* s, vt_block block, int32_t n, const double* rate,
                                        const double* mem, int32_t col_unit, vt_range* ranges,
                                        double* makespan) {
@@ -275,52 +351,113 @@ extern "C" vt_status vt_plan_tp_shares(const vt_shapes* s, vt_block block, int32
     VT_TRY(vt_shapes_validate(s));
     if (n < 1 || n > VT_MAX_DEVICES) return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
     if (block != VT_BLOCK_ATTN && block != VT_BLOCK_FFN) return fail(VT_ERR_INVALID_ARG, "unknown block %d", (int)block);
-    for (int d = 0; d < n; ++d) {
-        if (!(rate[d] > 0.0) || !std::isfinite(rate[d]))
-            return fail(VT_ERR_INVALID_ARG, "rate[%d] must be finite and positive", d);
-        if (mem && !(mem[d] >= 0.0)) return fail(VT_ERR_INVALID_ARG, "mem_bytes[%d] must be >= 0", d);
-    }
-    const double D = s->d_model, dh = s->d_head;
-    const int g = s->n_heads / s->n_kv_heads;
-    int units, per_unit;   // units, and heads or columns per unit
-    double unit_bytes;
-    if (block == VT_BLOCK_ATTN) {
-        units = s->n_kv_heads;
-        per_unit = g;
-        // QKV rows (g query heads, one K and one V head), O columns, and the K / V cache
-        unit_bytes = 2.0 * ((g + 2) * dh * D + D * g * dh) + 2.0 * 2.0 * s->max_seq * dh;
-    } else {
-        if (col_unit < 1) return fail(VT_ERR_INVALID_ARG, "col_unit must be >= 1");
-        per_unit = col_unit;
-        units = (s->d_ffn + col_unit - 1) / col_unit;
-        unit_bytes = 2.0 * 3.0 * D * col_unit;  // gate, up and down columns
-    }
-    std::vector<int> cnt(n, 0);
-    for (int u = 0; u < units; ++u) {
-        int best = -1;
-        double best_t = 0.0;
-        for (int d = 0; d < n; ++d) {
-            if (mem && (cnt[d] + 1) * unit_bytes > mem[d]) continue;
-            const double t = (cnt[d] + 1) * unit_bytes / rate[d];
-            if (best < 0 || t < best_t) {
-                best = d;
-                best_t = t;
-            }
-        }
-        if (best < 0) return fail(VT_ERR_PLAN_MEMORY, "unit %d of %d fits on no device", u, units);
-        ++cnt[best];
-    }
-    const int total = block == VT_BLOCK_ATTN ? s->n_heads : s->d_ffn;
-    int at = 0;
+    VT_TRY(check_rates(n, rate, mem));
+    if (block == VT_BLOCK_FFN && col_unit < 1) return fail(VT_ERR_INVALID_ARG, "col_unit must be >= 1");
+    const BlockUnits b = block_units(*s, block, block == VT_BLOCK_FFN ? col_unit : 1);
+    double t[VT_MAX_DEVICES];
+    for (int d = 0; d < n; ++d) t[d] = b.mem / rate[d];
+    int cnt[VT_MAX_DEVICES];
+    if (!greedy_shares(b.units, b.mem, n, t, mem, cnt))
+        return fail(VT_ERR_PLAN_MEMORY, "the block's %d units do not fit the memory budgets", b.units);
+    shares_to_ranges(n, cnt, b.per_unit, b.total, ranges);
     double worst = 0.0;
-    for (int d = 0; d < n; ++d) {
-        const int e = std::min(total, at + cnt[d] * per_unit);
-        ranges[d].begin = at;
-        ranges[d].end = e;
-        at = e;
-        worst = std::max(worst, cnt[d] * unit_bytes / rate[d]);
-    }
+    for (int d = 0; d < n; ++d) worst = std::max(worst, cnt[d] * t[d]);
     if (makespan) *makespan = worst;
+    return ok();
+}
+
+// Layer-wise hybrid parallelism plan (Voltron Section 4.2.1, with the communication pattern of
+// MP and TP in Section 3.2.1).
+extern "C" vt_status vt_plan_layers(const vt_shapes* s, int32_t n, const double* rate, const double* frate,
+                                    const double* mem, double link_bps, double link_lat, int32_t tokens,
+                                    int32_t kv_len, vt_block_plan* plans, double* total_s) {
+    if (!s || !rate || !plans) return fail(VT_ERR_INVALID_ARG, "shapes, rate and plans must not be NULL");
+    VT_TRY(vt_shapes_validate(s));
+    if (n < 1 || n > VT_MAX_DEVICES) return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
+    VT_TRY(check_rates(n, rate, mem));
+    if (frate)
+        for (int d = 0; d < n; ++d)
+            if (!(frate[d] > 0.0) || !std::isfinite(frate[d]))
+                return fail(VT_ERR_INVALID_ARG, "flop_rate[%d] must be finite and positive", d);
+    if (!(link_bps > 0.0) || !std::isfinite(link_bps) || !(link_lat >= 0.0) || !std::isfinite(link_lat))
+        return fail(VT_ERR_INVALID_ARG, "the link needs a finite positive rate and a finite latency >= 0");
+    if (tokens < 1 || kv_len < 0 || (int64_t)kv_len + tokens > s->max_seq)
+        return fail(VT_ERR_INVALID_ARG, "tokens %d at kv_len %d do not fit max_seq %d", tokens, kv_len, s->max_seq);
+    const double D = s->d_model, dh = s->d_head, T = tokens, Lkv = kv_len;
+    const double act = T * D * 2.0, part = T * D * 4.0;  // fp16 activations, fp32 partials
+    auto xfer = [&](double bytes) { return link_lat + bytes / link_bps; };
+    std::vector<double> left(n, 0.0);
+    for (int d = 0; d < n; ++d) left[d] = mem ? mem[d] : std::numeric_limits<double>::infinity();
+    // devices by rate, fastest first (ties: lower index): the order MP tries them in
+    std::vector<int> by_rate(n);
+    for (int d = 0; d < n; ++d) by_rate[d] = d;
+    std::stable_sort(by_rate.begin(), by_rate.end(), [&](int a, int b) { return rate[a] > rate[b]; });
+    int holder = 0;
+    double total = 0.0;
+    for (int bi = 0; bi < 2 * s->n_layers; ++bi) {
+        const vt_block blk = (bi & 1) ? VT_BLOCK_FFN : VT_BLOCK_ATTN;
+        const BlockUnits b = block_units(*s, blk, 1);
+        // per unit: bytes streamed (weights, K / V rows read at kv_len and written for the new rows)
+        // and flops over all tokens (2 per weight per token; ATTN also 4 dh per query head and
+        // visible position: scores and weighted values)
+        double ubytes = b.wbytes, uflops = T * b.wbytes;  // 2 flops per fp16 weight (2 bytes) per token
+        if (blk == VT_BLOCK_ATTN) {
+            const double g = s->n_heads / s->n_kv_heads;
+            ubytes += 2.0 * 2.0 * dh * (Lkv + T);
+            uflops += g * 4.0 * dh * (T * Lkv + T * (T + 1) / 2.0);
+        }
+        double ut[VT_MAX_DEVICES];
+        for (int d = 0; d < n; ++d) ut[d] = std::max(ubytes / rate[d], frate ? uflops / frate[d] : 0.0);
+        // MP: the fastest device whose remaining memory holds the block
+        int mp = -1;
+        for (int d : by_rate)
+            if (b.units * b.mem <= left[d]) {
+                mp = d;
+                break;
+            }
+        const double inf = std::numeric_limits<double>::infinity();
+        double mp_comp = inf, mp_comm = 0.0;
+        if (mp >= 0) {
+            mp_comp = b.units * ut[mp];
+            mp_comm = mp != holder ? xfer(act) : 0.0;
+        }
+        // TP: greedy shares on the remaining memory
+        int cnt[VT_MAX_DEVICES];
+        const bool tp_ok = greedy_shares(b.units, b.mem, n, ut, left.data(), cnt);
+        double tp_comp = inf, tp_comm = 0.0;
+        if (tp_ok) {
+            tp_comp = 0.0;
+            int others = 0;
+            for (int d = 0; d < n; ++d) {
+                tp_comp = std::max(tp_comp, cnt[d] * ut[d]);
+                if (cnt[d] > 0 && d != holder) ++others;
+            }
+            if (others > 0) tp_comm = xfer(act) + others * xfer(part);
+        }
+        if (mp < 0 && !tp_ok)
+            return fail(VT_ERR_PLAN_MEMORY, "block %d of layer %d fits under neither MP nor TP", bi & 1, bi / 2);
+        vt_block_plan& pl = plans[bi];
+        pl = vt_block_plan{};
+        if (tp_ok && tp_comp + tp_comm < mp_comp + mp_comm) {
+            pl.tp = 1;
+            pl.device = holder;
+            shares_to_ranges(n, cnt, b.per_unit, b.total, pl.ranges);
+            pl.compute_s = tp_comp;
+            pl.comm_s = tp_comm;
+            for (int d = 0; d < n; ++d) left[d] -= cnt[d] * b.mem;
+        } else {
+            pl.tp = 0;
+            pl.device = mp;
+            // the whole block on mp: empty ranges before and after it, in device order
+            for (int d = 0; d < n; ++d) pl.ranges[d] = vt_range{d <= mp ? 0 : b.total, d < mp ? 0 : b.total};
+            pl.compute_s = mp_comp;
+            pl.comm_s = mp_comm;
+            left[mp] -= b.units * b.mem;
+            holder = mp;
+        }
+        total += pl.compute_s + pl.comm_s;
+    }
+    if (total_s) *total_s = total;
     return ok();
 }
 

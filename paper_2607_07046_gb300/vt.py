@@ -54,6 +54,11 @@ class vt_range(ctypes.Structure):
     _fields_ = [("begin", _I32), ("end", _I32)]
 
 
+class vt_block_plan(ctypes.Structure):
+    _fields_ = [("tp", _I32), ("device", _I32), ("ranges", vt_range * VT_MAX_DEVICES),
+                ("compute_s", ctypes.c_double), ("comm_s", ctypes.c_double)]
+
+
 ALLOC_FN = ctypes.CFUNCTYPE(_P, ctypes.c_size_t, _P)
 FREE_FN = ctypes.CFUNCTYPE(None, _P, _P)
 
@@ -92,6 +97,10 @@ def lib() -> ctypes.CDLL:
             "vt_plan_tp_shares": (S, [ctypes.POINTER(vt_shapes), _I32, _I32, ctypes.POINTER(ctypes.c_double),
                                       ctypes.POINTER(ctypes.c_double), _I32, ctypes.POINTER(vt_range),
                                       ctypes.POINTER(ctypes.c_double)]),
+            "vt_plan_layers": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(ctypes.c_double),
+                                   ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                                   ctypes.c_double, ctypes.c_double, _I32, _I32,
+                                   ctypes.POINTER(vt_block_plan), ctypes.POINTER(ctypes.c_double)]),
             "vt_model_create": (S, [ctypes.POINTER(vt_shapes), ctypes.POINTER(vt_layer_weights), _P,
                                     ctypes.POINTER(vt_allocator), _P, ctypes.POINTER(_P)]),
             "vt_model_load_layer": (S, [_P, _I32, ctypes.POINTER(vt_layer_weights), _P]),
@@ -229,6 +238,29 @@ def vt_plan_tp_shares(shapes: vt_shapes, block: int, rate, mem_bytes=None, col_u
     _check(lib().vt_plan_tp_shares(ctypes.byref(shapes), int(block), n, r, m, int(col_unit), out,
                                    ctypes.byref(ms)))
     return [(out[d].begin, out[d].end) for d in range(n)], ms.value
+
+
+def vt_plan_layers(shapes: vt_shapes, rate, flop_rate=None, mem_bytes=None, link_bytes_per_s=1e30,
+                   link_latency_s=0.0, tokens: int = 1, kv_len: int = 0):
+    """Layer-wise MP/TP plan of the stack: (list of per-block dicts, total seconds).  Blocks are
+    ATTN of layer 0, FFN of layer 0, ATTN of layer 1, ...  Raises VtError on a failed status."""
+    n = len(rate)
+
+    def arr(v):
+        if v is None:
+            return None
+        if len(v) != n:
+            raise ValueError("one value per device")
+        return (ctypes.c_double * max(1, n))(*[float(x) for x in v])
+
+    out = (vt_block_plan * (2 * shapes.n_layers))()
+    tot = ctypes.c_double(0.0)
+    _check(lib().vt_plan_layers(ctypes.byref(shapes), n, arr(rate), arr(flop_rate), arr(mem_bytes),
+                                float(link_bytes_per_s), float(link_latency_s), int(tokens), int(kv_len),
+                                out, ctypes.byref(tot)))
+    plans = [dict(tp=bool(p.tp), device=p.device, ranges=[(p.ranges[d].begin, p.ranges[d].end) for d in range(n)],
+                  compute_s=p.compute_s, comm_s=p.comm_s) for p in out]
+    return plans, tot.value
 
 
 # ------------------------------------------------------------------ model

@@ -7,6 +7,7 @@ devices; KV-group alignment under GQA; the minimum makespan over every split, by
 small blocks; the block's bytes from the layer definition; memory budgets."""
 from __future__ import annotations
 
+import dataclasses
 import itertools
 import math
 
@@ -161,4 +162,128 @@ def test_invalid_arguments(vtlib, rates, kw):
     s = vtlib.make_shapes(1, 256, 4, 4, 64, 100, 0, 64)
     with pytest.raises(vtlib.VtError) as e:
         vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates, **kw)
+    assert e.value.status == vtlib.VT_ERR_INVALID_ARG
+
+
+# ------------------------------------------------------------------ layer-wise MP / TP plan
+
+def block_time_bytes(wl, block, kv_len, tokens):
+    """Bytes a whole block streams for `tokens` new rows: fp16 weights, plus for ATTN the K and V
+    rows read at kv_len and written for the new rows."""
+    D, H, Hk, dh, F = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn
+    if block == 0:
+        return 2 * ((H + 2 * Hk) * dh * D + D * H * dh) + 2 * 2 * Hk * dh * (kv_len + tokens)
+    return 2 * 3 * D * F
+
+
+def block_flops(wl, block, kv_len, tokens):
+    """Multiply-adds x 2 of a block over `tokens` rows: projections, and for ATTN the scores and the
+    weighted values over the causally visible positions (row i sees kv_len + i + 1)."""
+    D, H, Hk, dh, F = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn
+    if block == 0:
+        proj = 2 * tokens * ((H + 2 * Hk) * dh * D + D * H * dh)
+        visible = sum(kv_len + i + 1 for i in range(tokens))
+        return proj + 2 * 2 * H * dh * visible
+    return 2 * tokens * 3 * D * F
+
+
+def plan_shapes(vt, wl, max_seq):
+    return vt.make_shapes(wl.n_layers, wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, 0, max_seq,
+                          wl.rms_eps, wl.rope_theta)
+
+
+def test_one_device_runs_every_block_without_transfers(vtlib):
+    wl = synthetic.WORKLOADS[2]
+    s = plan_shapes(vtlib, wl, 2048)
+    plans, total = vtlib.vt_plan_layers(s, [3e12], link_bytes_per_s=1e9, link_latency_s=1e-3, kv_len=1024)
+    assert len(plans) == 2 * wl.n_layers
+    for i, p in enumerate(plans):
+        assert not p["tp"] and p["device"] == 0 and p["comm_s"] == 0.0
+        assert p["compute_s"] == pytest.approx(block_time_bytes(wl, i % 2, 1024, 1) / 3e12, rel=1e-12)
+    want = wl.n_layers * (block_time_bytes(wl, 0, 1024, 1) + block_time_bytes(wl, 1, 1024, 1)) / 3e12
+    assert total == pytest.approx(want, rel=1e-12)
+
+
+def test_free_link_splits_every_block_evenly(vtlib):
+    """Two equal devices and a link that costs nothing: TP halves every block's time."""
+    wl = synthetic.WORKLOADS[2]
+    s = plan_shapes(vtlib, wl, 2048)
+    one, t1 = vtlib.vt_plan_layers(s, [1e12], kv_len=1024)
+    two, t2 = vtlib.vt_plan_layers(s, [1e12, 1e12], link_bytes_per_s=1e30, link_latency_s=0.0, kv_len=1024)
+    for i, p in enumerate(two):
+        assert p["tp"] and p["device"] == 0
+        assert p["ranges"] == ([(0, 16), (16, 32)] if i % 2 == 0 else [(0, 5504), (5504, 11008)])
+    assert t2 == pytest.approx(t1 / 2, rel=1e-9)
+
+
+def test_slow_link_keeps_the_stack_on_the_fastest_device(vtlib):
+    """A link too slow for TP: every block on the fastest device (device 1); the input moves there
+    once, before the first block."""
+    wl = synthetic.WORKLOADS[2]
+    s = plan_shapes(vtlib, wl, 2048)
+    bps, lat = 1e6, 2e-3
+    plans, total = vtlib.vt_plan_layers(s, [1e12, 2e12], link_bytes_per_s=bps, link_latency_s=lat, kv_len=1024)
+    assert all(not p["tp"] and p["device"] == 1 for p in plans)
+    assert plans[0]["comm_s"] == pytest.approx(lat + wl.d_model * 2 / bps, rel=1e-12)
+    assert all(p["comm_s"] == 0.0 for p in plans[1:])
+    assert plans[0]["ranges"][1] == (0, wl.n_heads) and plans[1]["ranges"][1] == (0, wl.d_ffn)
+
+
+def test_memory_moves_the_rest_of_the_stack_once(vtlib):
+    """The fastest device holds 3 blocks: blocks 0-2 run there, the rest on device 0, with one
+    transfer when the activations change device (slow link, so TP never pays)."""
+    wl = dataclasses.replace(synthetic.WORKLOADS[2], n_layers=4)
+    max_seq = 2048
+    s = plan_shapes(vtlib, wl, max_seq)
+    D, H, Hk, dh, F = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn
+    attn_mem = 2 * ((H + 2 * Hk) * dh * D + D * H * dh) + 2 * 2 * Hk * dh * max_seq
+    ffn_mem = 2 * 3 * D * F
+    budget1 = 2 * attn_mem + ffn_mem + 1.0   # ATTN 0, FFN 0, ATTN 1
+    bps, lat = 1e6, 1e-3
+    plans, _ = vtlib.vt_plan_layers(s, [1e12, 4e12], mem_bytes=[1e30, budget1], link_bytes_per_s=bps,
+                                    link_latency_s=lat, kv_len=1024)
+    assert [p["device"] for p in plans] == [1, 1, 1, 0, 0, 0, 0, 0]
+    assert not any(p["tp"] for p in plans)
+    hop = lat + D * 2 / bps
+    assert [p["comm_s"] for p in plans] == pytest.approx([hop, 0, 0, hop, 0, 0, 0, 0])
+
+
+def test_prefill_time_is_the_flop_bound_when_the_flop_rate_is_low(vtlib):
+    wl = dataclasses.replace(synthetic.WORKLOADS[4], n_layers=1)
+    s = plan_shapes(vtlib, wl, 1024)
+    plans, _ = vtlib.vt_plan_layers(s, [1e12], flop_rate=[1e9], tokens=512, kv_len=0)
+    for b in (0, 1):
+        assert plans[b]["compute_s"] == pytest.approx(block_flops(wl, b, 0, 512) / 1e9, rel=1e-12)
+    plans, _ = vtlib.vt_plan_layers(s, [1e6], flop_rate=[1e30], tokens=512, kv_len=0)
+    for b in (0, 1):
+        assert plans[b]["compute_s"] == pytest.approx(block_time_bytes(wl, b, 0, 512) / 1e6, rel=1e-12)
+
+
+def test_heterogeneous_devices_on_a_fast_link_get_their_rate_shares(vtlib):
+    wl = synthetic.WORKLOADS[3]
+    s = plan_shapes(vtlib, wl, 2056)
+    plans, _ = vtlib.vt_plan_layers(s, [5e11, 3e11, 2e11], link_bytes_per_s=1e30, kv_len=2048)
+    assert all(p["tp"] for p in plans)
+    assert plans[1]["ranges"] == list(wl.ffn_ranges)
+
+
+def test_no_device_can_hold_a_block(vtlib):
+    wl = dataclasses.replace(synthetic.WORKLOADS[2], n_layers=2)
+    s = plan_shapes(vtlib, wl, 2048)
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_layers(s, [1e12, 1e12], mem_bytes=[1e6, 1e6], kv_len=0)
+    assert e.value.status == vtlib.VT_ERR_PLAN_MEMORY
+
+
+@pytest.mark.parametrize("kw", [
+    dict(tokens=0), dict(kv_len=-1), dict(kv_len=2048, tokens=1), dict(link_bytes_per_s=0.0),
+    dict(link_latency_s=-1.0), dict(link_bytes_per_s=float("nan")), dict(flop_rate=[0.0, 1.0]),
+])
+def test_plan_layers_invalid_arguments(vtlib, kw):
+    wl = dataclasses.replace(synthetic.WORKLOADS[2], n_layers=1)
+    s = plan_shapes(vtlib, wl, 2048)
+    args = dict(rate=[1e12, 1e12], kv_len=0)
+    args.update(kw)
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_layers(s, **args)
     assert e.value.status == vtlib.VT_ERR_INVALID_ARG
