@@ -136,29 +136,64 @@ def kernels_per_token(wl):
     return wl.n_layers * (n + 2) + 1
 
 
-def cpu_baseline_decode(wl, layers=4, budget_s=12.0, max_tokens=512):
+def cpu_baseline_decode(wl, layers=4, budget_s=12.0, max_tokens=512, budget_1thread_s=4.0, max_tokens_1thread=32):
     """The oracle (as it stands) on `layers` layers, decoding teacher-forced tokens from KV 1024
-    until about `budget_s` seconds of CPU time have passed; tok/s is extrapolated to the full
-    stack by the layer ratio."""
+    until about `budget_s` seconds have passed on all host threads, then about `budget_1thread_s`
+    seconds on one thread (continuing the same caches); tok/s is extrapolated to the full stack by
+    the layer ratio."""
     import oracle
-    oracle.num_threads()
+    threads = oracle.num_threads()
     L0 = wl.kv_len
     ws = [wl.layer_weights(l) for l in range(layers)]
-    caches = [wl.kv_fill(l, L0, L0 + max_tokens + 1) for l in range(layers)]
-    t0 = time.perf_counter()
+    caches = [wl.kv_fill(l, L0, L0 + max_tokens + max_tokens_1thread + 1) for l in range(layers)]
     tokens = 0
-    while tokens < max_tokens and (tokens < 2 or time.perf_counter() - t0 < budget_s):
-        x = wl.hidden(1, stream=500 + tokens)
-        for l in range(layers):
-            _, x, _, _ = oracle.tp_layer(wl, ws[l], x, L0 + tokens, *caches[l])
-        tokens += 1
-    dt = time.perf_counter() - t0
-    per_token = dt / tokens * (wl.n_layers / layers)
-    return {"value": round(1.0 / per_token, 4), "unit": "tok/s", "cores": oracle.num_threads(),
+
+    def run(budget, limit):
+        nonlocal tokens
+        t0 = time.perf_counter()
+        done = 0
+        while done < limit and (done < 1 or time.perf_counter() - t0 < budget):
+            x = wl.hidden(1, stream=500 + tokens)
+            for l in range(layers):
+                _, x, _, _ = oracle.tp_layer(wl, ws[l], x, L0 + tokens, *caches[l])
+            tokens += 1
+            done += 1
+        return done, time.perf_counter() - t0
+
+    n_all, dt = run(budget_s, max_tokens)
+    oracle.set_threads(1)
+    try:
+        n_one, dt1 = run(budget_1thread_s, max_tokens_1thread)
+    finally:
+        oracle.set_threads(threads)
+    scale = wl.n_layers / layers
+    return {"value": round(n_all / (dt * scale), 4), "unit": "tok/s", "cores": threads,
             "kind": "oracle",
-            "sample": f"{tokens} teacher-forced decode tokens through layers 0-{layers - 1} of "
+            "sample": f"{n_all} teacher-forced decode tokens through layers 0-{layers - 1} of "
                       f"{wl.n_layers} from KV {L0}, 4-way TP shards, fp64 oracle; tok/s "
-                      f"extrapolated x{wl.n_layers / layers:g} by layers",
+                      f"extrapolated x{scale:g} by layers",
+            "seconds": round(dt, 2),
+            "value_1thread": round(n_one / (dt1 * scale), 4),
+            "sample_1thread": f"{n_one} further tokens on 1 thread (same layers and extrapolation)",
+            "seconds_1thread": round(dt1, 2)}
+
+
+def cpu_baseline_prefill(wl, layers=1):
+    """The oracle (as it stands) on the whole prompt of the prefill workload through `layers`
+    layers on all host threads; tok/s is extrapolated to the full stack by the layer ratio."""
+    import oracle
+    n = wl.prompt_len
+    x = wl.hidden(n, stream=600)
+    t0 = time.perf_counter()
+    for l in range(layers):
+        kc, vc = oracle.new_cache(wl, n)
+        _, x, _, _ = oracle.tp_layer(wl, wl.layer_weights(l), x, 0, kc, vc)
+    dt = time.perf_counter() - t0
+    scale = wl.n_layers / layers
+    return {"value": round(n / (dt * scale), 2), "unit": "tok/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"the {n}-token prompt through layer(s) 0-{layers - 1} of {wl.n_layers}, 4-way TP "
+                      f"shards, fp64 oracle; tok/s extrapolated x{scale:g} by layers",
             "seconds": round(dt, 2)}
 
 
@@ -556,6 +591,8 @@ def main():
         line["other_workloads"] = [run_decode_workload(cid, args.other_steps, 8) for cid in (3, 5)]
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_decode(synthetic.WORKLOADS[2])
+        if "prefill" in line:
+            line["prefill"]["cpu_baseline"] = cpu_baseline_prefill(synthetic.WORKLOADS[4])
     if world > 1:
         import torch
         torch.distributed.barrier()
