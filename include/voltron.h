@@ -196,6 +196,18 @@ VT_API vt_status vt_plan_layers(const vt_shapes* shapes, int32_t n_devices, cons
                                 double link_latency_s, int32_t tokens, int32_t kv_len, vt_block_plan* plans,
                                 double* total_s);
 
+/* vt_quantize_rows (host only): block quantization of fp16 weight rows for mixed-precision shards
+ * (Voltron Section 3.2.2 and Section 4.2.2, precision heterogeneity; Section 5.1 names k-quant
+ * formats without defining them).  Each row of w (host fp16 [rows][k], row-major) is cut into
+ * blocks of `block` consecutive weights (the last one may be shorter); a block gets the fp16
+ * scale d = fp16(amax / qmax) (amax: its largest |w|; qmax: 127 for bits = 8, 7 for bits = 4) and
+ * every weight the code q = round-half-even(w / d) clamped to [-qmax, qmax] (0 when d = 0), both
+ * divisions in fp32.  Outputs (host, caller-owned): q int8 [rows][k]; scales fp16
+ * [rows][ceil(k / block)].  The dequantized weight is q * d.
+ * Errors: VT_ERR_INVALID_ARG (NULL pointer, rows or k < 0, block < 1, bits not 8 or 4). */
+VT_API vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, int32_t bits, int32_t block, int8_t* q,
+                                  void* scales);
+
 /* ---------------------------------------------------------------- model ------------------------
  * vt_model_create: allocates device storage for every layer in the canonical (unpartitioned)
  * layout, the RoPE table for positions [0, max_seq) and, if vocab > 0, the embedding table, on

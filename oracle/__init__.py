@@ -59,6 +59,9 @@ def lib():
                                      _I32, _P, _I32, _P]
         L.or_ffn_partial.restype = _I32
         L.or_combine.argtypes = [ctypes.POINTER(_P), _I32, _I64, _P, _P]
+        L.or_quantize_rows.argtypes = [_P, _I64, _I64, _I32, _I32, _P, _P]
+        L.or_quantize_rows.restype = _I32
+        L.or_gemv_blockq.argtypes = [_P, _P, _I64, _I64, _I32, _P, _P]
         _lib = L
     return _lib
 
@@ -225,3 +228,31 @@ def tp_layer(wl, weights, x: np.ndarray, pos0: int, kcache, vcache, head_ranges=
     h, ap = tp_attention(wl, weights, x, pos0, kcache, vcache, head_ranges)
     xn, fp = tp_ffn(wl, weights, h, ffn_ranges)
     return h, xn, ap, fp
+
+
+def quantize_rows(w: np.ndarray, bits: int, block: int = 32) -> Tuple[np.ndarray, np.ndarray]:
+    """Block quantization of binary16 weight rows [rows, k] (format in oracle.c): int8 codes
+    [rows, k] and binary16 scales [rows, ceil(k / block)]."""
+    w = _f16(w)
+    if w.ndim != 2:
+        raise ValueError("expected [rows, k]")
+    rows, k = w.shape
+    q = np.zeros((rows, k), np.int8)
+    sc = np.zeros((rows, (k + block - 1) // block), np.float16)
+    st = lib().or_quantize_rows(w.ctypes.data, rows, k, bits, block, q.ctypes.data, sc.ctypes.data)
+    if st != 0:
+        raise ValueError(f"or_quantize_rows failed ({st})")
+    return q, sc
+
+
+def gemv_blockq(q: np.ndarray, scales: np.ndarray, x, block: int = 32) -> np.ndarray:
+    """Dequantized W . x in binary64."""
+    q = np.ascontiguousarray(q, np.int8)
+    sc = _f16(scales)
+    xx = _f64(x).reshape(-1)
+    rows, k = q.shape
+    if xx.size != k or sc.shape != (rows, (k + block - 1) // block):
+        raise ValueError("shape mismatch")
+    y = np.zeros(rows, np.float64)
+    lib().or_gemv_blockq(q.ctypes.data, sc.ctypes.data, rows, k, block, xx.ctypes.data, y.ctypes.data)
+    return y

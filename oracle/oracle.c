@@ -278,3 +278,57 @@ void or_combine(const double* const* partials, int32_t n, int64_t count, const u
         out[e] = or_f64_to_f16(acc);
     }
 }
+
+/* ---------------------------------------------------------------- block quantization ------ */
+/* Mixed-precision weight shards (Voltron Section 3.2.2, precision heterogeneity; Section 4.2.2;
+ * Section 5.1 adopts k-quant formats without defining them).  Reading: each row of a weight
+ * matrix is cut into blocks of `block` consecutive weights along the input dimension; a block
+ * keeps one binary16 scale d = binary16(amax / qmax), amax the largest |w| of the block, qmax 127
+ * (8 bits) or 7 (4 bits), and one signed code per weight, q = round-half-even(w / d) clamped to
+ * [-qmax, qmax] (q = 0 when d = 0).  The decision is taken in binary32 arithmetic (the division
+ * amax / qmax and w / d), the precision the library's quantizer uses, so both give the same codes.
+ * The dequantized weight is q * d. */
+
+int32_t or_quantize_rows(const uint16_t* w, int64_t rows, int64_t k, int32_t bits, int32_t block, int8_t* q,
+                         uint16_t* scales) {
+    if (!w || !q || !scales || rows < 0 || k < 0 || block < 1 || (bits != 8 && bits != 4)) return OR_ERR_ARG;
+    const int32_t qmax = bits == 8 ? 127 : 7;
+    const int64_t nb = (k + block - 1) / block;
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) {
+        for (int64_t b = 0; b < nb; ++b) {
+            const int64_t e0 = b * block, e1 = e0 + block < k ? e0 + block : k;
+            float amax = 0.0f;
+            for (int64_t e = e0; e < e1; ++e) {
+                const float v = fabsf((float)or_f16_to_f64(w[r * k + e]));
+                if (v > amax) amax = v;
+            }
+            const float t = amax / (float)qmax;            /* binary32 division */
+            const uint16_t d16 = or_f64_to_f16((double)t);  /* exact widening, then round to binary16 */
+            const float d = (float)or_f16_to_f64(d16);
+            scales[r * nb + b] = d16;
+            for (int64_t e = e0; e < e1; ++e) {
+                int32_t c = 0;
+                if (d != 0.0f) {
+                    const float x = (float)or_f16_to_f64(w[r * k + e]) / d;  /* binary32 division */
+                    const float rx = nearbyintf(x);                          /* ties to even */
+                    c = rx > (float)qmax ? qmax : (rx < (float)-qmax ? -qmax : (int32_t)rx);
+                }
+                q[r * k + e] = (int8_t)c;
+            }
+        }
+    }
+    return OR_OK;
+}
+
+/* y[r] = sum_e (q[r][e] * d[r][e / block]) * x[e] in binary64, e in index order. */
+void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64_t k, int32_t block,
+                    const double* x, double* y) {
+    const int64_t nb = (k + block - 1) / block;
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) {
+        double acc = 0.0;
+        for (int64_t e = 0; e < k; ++e) acc += (double)q[r * k + e] * or_f16_to_f64(scales[r * nb + e / block]) * x[e];
+        y[r] = acc;
+    }
+}

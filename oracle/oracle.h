@@ -96,4 +96,13 @@ int32_t or_ffn_partial(const or_shapes* s, const or_layer* w, int32_t c0, int32_
 void or_combine(const double* const* partials, int32_t n, int64_t count, const uint16_t* residual,
                 uint16_t* out);
 
+/* Block quantization of binary16 weight rows [rows, k] (Section 3.2.2 / 4.2.2 precision
+ * heterogeneity; format reading in oracle.c): codes q [rows, k] (one int8 per weight, in
+ * [-127, 127] for bits = 8, [-7, 7] for bits = 4) and binary16 scales [rows, ceil(k / block)]. */
+int32_t or_quantize_rows(const uint16_t* w, int64_t rows, int64_t k, int32_t bits, int32_t block, int8_t* q,
+                         uint16_t* scales);
+/* y = dequantized W . x in binary64 (rows of q, scales as above). */
+void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64_t k, int32_t block,
+                    const double* x, double* y);
+
 #endif

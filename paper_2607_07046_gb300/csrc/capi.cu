@@ -461,6 +461,39 @@ extern "C" vt_status vt_plan_layers(const vt_shapes* s, int32_t n, const double*
     return ok();
 }
 
+// ================================================================== quantization (host)
+
+// Block quantization of fp16 weight rows (Voltron Sections 3.2.2 / 4.2.2): fp16 scale per block,
+// int8 code per weight, every decision in fp32.
+extern "C" vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, int32_t bits, int32_t block, int8_t* q,
+                                      void* scales) {
+    if (!w || !q || !scales) return fail(VT_ERR_INVALID_ARG, "w, q and scales must not be NULL");
+    if (rows < 0 || k < 0 || block < 1 || (bits != 8 && bits != 4))
+        return fail(VT_ERR_INVALID_ARG, "rows %lld, k %lld, block %d, bits %d", (long long)rows, (long long)k, block, bits);
+    const __half* src = static_cast<const __half*>(w);
+    __half* sc = static_cast<__half*>(scales);
+    const int qmax = bits == 8 ? 127 : 7;
+    const int64_t nb = (k + block - 1) / block;
+    for (int64_t r = 0; r < rows; ++r)
+        for (int64_t b = 0; b < nb; ++b) {
+            const int64_t e0 = b * block, e1 = std::min(k, e0 + block);
+            float amax = 0.0f;
+            for (int64_t e = e0; e < e1; ++e) amax = std::max(amax, std::fabs(__half2float(src[r * k + e])));
+            const __half d16 = __float2half_rn(amax / (float)qmax);
+            const float d = __half2float(d16);
+            sc[r * nb + b] = d16;
+            for (int64_t e = e0; e < e1; ++e) {
+                int c = 0;
+                if (d != 0.0f) {
+                    const float x = std::nearbyint(__half2float(src[r * k + e]) / d);  // ties to even
+                    c = x > (float)qmax ? qmax : (x < (float)-qmax ? -qmax : (int)x);
+                }
+                q[r * k + e] = (int8_t)c;
+            }
+        }
+    return ok();
+}
+
 // ================================================================== model
 
 static vt_status upload(void* dst, const void* src, size_t bytes, cudaStream_t st) {

@@ -97,6 +97,7 @@ def lib() -> ctypes.CDLL:
             "vt_plan_tp_shares": (S, [ctypes.POINTER(vt_shapes), _I32, _I32, ctypes.POINTER(ctypes.c_double),
                                       ctypes.POINTER(ctypes.c_double), _I32, ctypes.POINTER(vt_range),
                                       ctypes.POINTER(ctypes.c_double)]),
+            "vt_quantize_rows": (S, [_P, ctypes.c_int64, ctypes.c_int64, _I32, _I32, _P, _P]),
             "vt_plan_layers": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
                                    ctypes.c_double, ctypes.c_double, _I32, _I32,
@@ -238,6 +239,20 @@ def vt_plan_tp_shares(shapes: vt_shapes, block: int, rate, mem_bytes=None, col_u
     _check(lib().vt_plan_tp_shares(ctypes.byref(shapes), int(block), n, r, m, int(col_unit), out,
                                    ctypes.byref(ms)))
     return [(out[d].begin, out[d].end) for d in range(n)], ms.value
+
+
+def vt_quantize_rows(w, bits: int, block: int = 32):
+    """Host block quantization of fp16 weight rows [rows, k]: (int8 codes [rows, k], fp16 scales
+    [rows, ceil(k / block)]).  Raises VtError on a failed status."""
+    import numpy as np
+    w = np.ascontiguousarray(w, dtype=np.float16)
+    if w.ndim != 2:
+        raise ValueError("expected [rows, k]")
+    rows, k = w.shape
+    q = np.zeros((rows, k), np.int8)
+    sc = np.zeros((rows, (k + block - 1) // block if block > 0 else 1), np.float16)  # the library checks block
+    _check(lib().vt_quantize_rows(w.ctypes.data, rows, k, int(bits), int(block), q.ctypes.data, sc.ctypes.data))
+    return q, sc
 
 
 def vt_plan_layers(shapes: vt_shapes, rate, flop_rate=None, mem_bytes=None, link_bytes_per_s=1e30,

@@ -1,0 +1,117 @@
+"""Block quantization of weight shards (Voltron Sections 3.2.2 and 4.2.2, precision heterogeneity;
+Section 5.1 uses k-quant formats without defining them).  Reading: per row, blocks of 32 weights,
+fp16 scale d = fp16(amax / qmax) (qmax 127 for INT8, 7 for INT4), codes round-half-even(w / d)
+clamped to [-qmax, qmax], decisions in fp32.
+
+The oracle's quantizer is pinned to closed forms of that definition (exact power-of-two grids,
+ties to even, the zero block, a subnormal scale that needs the clamp, the d / 2 error bound), its
+dequantized matrix-vector product to numpy, and the library's own quantizer must give the same
+codes and scales bit for bit.  CPU only."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+
+import oracle
+
+
+def f16(a):
+    return np.asarray(a, dtype=np.float16)
+
+
+@pytest.mark.parametrize("bits,qmax", [(8, 127), (4, 7)])
+def test_power_of_two_grid_returns_its_integers(bits, qmax):
+    """Weights i * 2^-8 for i in [-qmax, qmax]: amax / qmax = 2^-8 exactly, so d = 2^-8 and every
+    code is i."""
+    i = np.arange(-qmax, qmax + 1)
+    w = f16(i * 2.0 ** -8)[None, :]
+    q, d = oracle.quantize_rows(w, bits, block=w.shape[1])
+    assert d[0, 0] == np.float16(2.0 ** -8)
+    assert np.array_equal(q[0], i.astype(np.int8))
+
+
+def test_ties_round_to_even():
+    """d = 2^-8 (the block's max is 127 * 2^-8); w = +-2.5 d, +-3.5 d, +-0.5 d sit exactly halfway."""
+    d = 2.0 ** -8
+    w = f16([127 * d, 2.5 * d, -2.5 * d, 3.5 * d, -3.5 * d, 0.5 * d, -0.5 * d, 1.5 * d])[None, :]
+    q, sc = oracle.quantize_rows(w, 8, block=8)
+    assert sc[0, 0] == np.float16(d)
+    assert q[0].tolist() == [127, 2, -2, 4, -4, 0, 0, 2]
+
+
+def test_zero_block_and_vanishing_scale():
+    """A zero block has d = 0 and codes 0; so does a block whose scale rounds to zero in fp16
+    (amax = 2^-20: amax / 127 is below half the smallest subnormal)."""
+    w = f16([[0.0] * 32 + [2.0 ** -20, -2.0 ** -21] + [0.0] * 30])
+    q, sc = oracle.quantize_rows(w, 8, block=32)
+    assert sc[0].tolist() == [0.0, 0.0]
+    assert not q.any()
+
+
+def test_subnormal_scale_needs_the_clamp():
+    """amax = 2^-15: amax / 127 = 2.40e-7 rounds to the subnormal 4 * 2^-24, so amax / d = 128,
+    clamped to 127; 2^-16 gives 64."""
+    w = f16([[2.0 ** -15, -(2.0 ** -15), 2.0 ** -16, 0.0]])
+    q, sc = oracle.quantize_rows(w, 8, block=4)
+    assert sc[0, 0] == np.float16(4 * 2.0 ** -24)
+    assert q[0].tolist() == [127, -127, 64, 0]
+
+
+@pytest.mark.parametrize("bits,qmax", [(8, 127), (4, 7)])
+def test_error_bound_and_extremes(bits, qmax):
+    """|w - q d| <= d / 2 for every weight (the scales here are normal fp16, so no clamp acts), the
+    block maximum maps to +-qmax, and negating the weights negates the codes."""
+    rng = np.random.default_rng(3 + bits)
+    w = f16(rng.standard_normal((64, 96)) * np.exp(rng.uniform(-3, 3, (64, 1))))
+    q, sc = oracle.quantize_rows(w, bits, block=32)
+    d = np.repeat(sc.astype(np.float64), 32, axis=1)
+    err = np.abs(w.astype(np.float64) - q.astype(np.float64) * d)
+    assert np.all(err <= d / 2 * (1 + 1e-6) + 1e-30)
+    blocks = np.abs(w.astype(np.float64)).reshape(64, 3, 32)
+    arg = blocks.argmax(axis=2)
+    for r in range(64):
+        for b in range(3):
+            assert abs(int(q[r, b * 32 + arg[r, b]])) == qmax
+    qn, scn = oracle.quantize_rows(-w, bits, block=32)
+    assert np.array_equal(qn, -q) and np.array_equal(scn, sc)
+
+
+def test_ragged_last_block():
+    w = f16(np.linspace(-1, 1, 70))[None, :]
+    q, sc = oracle.quantize_rows(w, 8, block=32)
+    assert sc.shape == (1, 3)
+    q6, sc6 = oracle.quantize_rows(w[:, 64:], 8, block=32)
+    assert np.array_equal(q[:, 64:], q6) and sc[0, 2] == sc6[0, 0]
+
+
+def test_dequantized_gemv_equals_numpy():
+    rng = np.random.default_rng(11)
+    w = f16(rng.standard_normal((33, 200)) * 0.02)
+    x = rng.standard_normal(200)
+    for bits in (8, 4):
+        q, sc = oracle.quantize_rows(w, bits, block=32)
+        deq = q.astype(np.float64) * np.repeat(sc.astype(np.float64), 32, axis=1)[:, :200]
+        assert np.allclose(oracle.gemv_blockq(q, sc, x), deq @ x, rtol=1e-13, atol=1e-15)
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("shape,block", [((37, 1000), 32), ((5, 31), 32), ((3, 4096), 32), ((9, 100), 16)])
+def test_library_quantizer_matches_the_oracle_bit_for_bit(vtlib, bits, shape, block):
+    rng = np.random.default_rng(sum(shape) + bits)
+    w = rng.standard_normal(shape) * np.exp(rng.uniform(-8, 8, (shape[0], 1)))
+    w = np.clip(w, -65504, 65504).astype(np.float16)
+    w[0, : min(8, shape[1])] = 0.0                      # part of a zero block
+    if shape[0] > 1:
+        w[1] = f16(rng.standard_normal(shape[1]) * 2.0 ** -16)   # subnormal scales
+    q1, s1 = oracle.quantize_rows(w, bits, block)
+    q2, s2 = vtlib.vt_quantize_rows(w, bits, block)
+    assert np.array_equal(q1, q2)
+    assert np.array_equal(s1.view(np.uint16), s2.view(np.uint16))
+
+
+def test_library_quantizer_rejects_bad_arguments(vtlib):
+    w = np.zeros((2, 8), np.float16)
+    for bits, block in ((5, 32), (8, 0), (0, 32)):
+        with pytest.raises(vtlib.VtError) as e:
+            vtlib.vt_quantize_rows(w, bits, block)
+        assert e.value.status == vtlib.VT_ERR_INVALID_ARG
