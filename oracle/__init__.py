@@ -62,6 +62,9 @@ def lib():
         L.or_quantize_rows.argtypes = [_P, _I64, _I64, _I32, _I32, _P, _P]
         L.or_quantize_rows.restype = _I32
         L.or_gemv_blockq.argtypes = [_P, _P, _I64, _I64, _I32, _P, _P]
+        L.or_quantize_vec.argtypes = [_P, _I64, _I32, _I32, _P, _P]
+        L.or_quantize_vec.restype = _I32
+        L.or_combine_q.argtypes = [ctypes.POINTER(_P), ctypes.POINTER(_P), _I32, _I64, _I32, _P, _P]
         _lib = L
     return _lib
 
@@ -256,3 +259,27 @@ def gemv_blockq(q: np.ndarray, scales: np.ndarray, x, block: int = 32) -> np.nda
     y = np.zeros(rows, np.float64)
     lib().or_gemv_blockq(q.ctypes.data, sc.ctypes.data, rows, k, block, xx.ctypes.data, y.ctypes.data)
     return y
+
+
+def quantize_vec(x, bits: int, block: int = 32) -> Tuple[np.ndarray, np.ndarray]:
+    """Block quantization of a binary32 vector (a shard partial): int8 codes, binary16 scales."""
+    xx = np.ascontiguousarray(x, np.float32).reshape(-1)
+    q = np.zeros(xx.size, np.int8)
+    sc = np.zeros((xx.size + block - 1) // block, np.float16)
+    st = lib().or_quantize_vec(xx.ctypes.data, xx.size, bits, block, q.ctypes.data, sc.ctypes.data)
+    if st != 0:
+        raise ValueError(f"or_quantize_vec failed ({st})")
+    return q, sc
+
+
+def combine_q(parts: Sequence[Tuple[np.ndarray, np.ndarray]], residual: Optional[np.ndarray], block: int = 32) -> np.ndarray:
+    """binary16(residual + sum of the dequantized partials), shards in order."""
+    qs = [np.ascontiguousarray(q, np.int8) for q, _ in parts]
+    ss = [_f16(s) for _, s in parts]
+    count = qs[0].size
+    qp = (_P * len(qs))(*[q.ctypes.data for q in qs])
+    sp = (_P * len(ss))(*[s.ctypes.data for s in ss])
+    out = np.zeros(count, np.float16)
+    res = _f16(residual).reshape(-1) if residual is not None else None
+    lib().or_combine_q(qp, sp, len(qs), count, block, res.ctypes.data if res is not None else None, out.ctypes.data)
+    return out

@@ -332,3 +332,47 @@ void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64
         y[r] = acc;
     }
 }
+
+/* ---------------------------------------------------------------- quantized partials ------ */
+/* Communication scaling (Voltron Section 4.3.2): activations sent between devices are lowered to
+ * INT8 or INT4.  Under tensor parallelism those are the shard partials sent to the main device.
+ * Reading: the same block format as the weights (blocks of `block` values, fp16 scale
+ * d = fp16(amax / qmax), codes round-half-even(x / d) clamped to [-qmax, qmax], binary32
+ * decisions), applied to the binary32 partial as it leaves the device; the main device adds the
+ * dequantized partials to the residual. */
+
+int32_t or_quantize_vec(const float* x, int64_t n, int32_t bits, int32_t block, int8_t* q, uint16_t* scales) {
+    if (!x || !q || !scales || n < 0 || block < 1 || (bits != 8 && bits != 4)) return OR_ERR_ARG;
+    const int32_t qmax = bits == 8 ? 127 : 7;
+    const int64_t nb = (n + block - 1) / block;
+    for (int64_t b = 0; b < nb; ++b) {
+        const int64_t e0 = b * block, e1 = e0 + block < n ? e0 + block : n;
+        float amax = 0.0f;
+        for (int64_t e = e0; e < e1; ++e)
+            if (fabsf(x[e]) > amax) amax = fabsf(x[e]);
+        const uint16_t d16 = or_f64_to_f16((double)(amax / (float)qmax));
+        const float d = (float)or_f16_to_f64(d16);
+        scales[b] = d16;
+        for (int64_t e = e0; e < e1; ++e) {
+            int32_t c = 0;
+            if (d != 0.0f) {
+                const float rx = nearbyintf(x[e] / d);
+                c = rx > (float)qmax ? qmax : (rx < (float)-qmax ? -qmax : (int32_t)rx);
+            }
+            q[e] = (int8_t)c;
+        }
+    }
+    return OR_OK;
+}
+
+/* out = binary16(residual + sum_s q_s * d_s) elementwise, shards in order s = 0..n-1, binary64
+ * sums; q[s] / scales[s] as written by or_quantize_vec for `count` values. */
+void or_combine_q(const int8_t* const* q, const uint16_t* const* scales, int32_t n, int64_t count, int32_t block,
+                  const uint16_t* residual, uint16_t* out) {
+#pragma omp parallel for schedule(static)
+    for (int64_t e = 0; e < count; ++e) {
+        double acc = residual ? HALF(residual[e]) : 0.0;
+        for (int32_t s = 0; s < n; ++s) acc += (double)q[s][e] * or_f16_to_f64(scales[s][e / block]);
+        out[e] = or_f64_to_f16(acc);
+    }
+}

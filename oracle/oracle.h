@@ -105,4 +105,11 @@ int32_t or_quantize_rows(const uint16_t* w, int64_t rows, int64_t k, int32_t bit
 void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64_t k, int32_t block,
                     const double* x, double* y);
 
+/* Quantized shard partials (Section 4.3.2, communication scaling; reading in oracle.c):
+ * codes q [n] and binary16 scales [ceil(n / block)] of a binary32 vector, and the combine of
+ * n quantized partials with a binary16 residual (NULL: zero) into binary16 out [count]. */
+int32_t or_quantize_vec(const float* x, int64_t n, int32_t bits, int32_t block, int8_t* q, uint16_t* scales);
+void or_combine_q(const int8_t* const* q, const uint16_t* const* scales, int32_t n, int64_t count, int32_t block,
+                  const uint16_t* residual, uint16_t* out);
+
 #endif

@@ -115,3 +115,52 @@ def test_library_quantizer_rejects_bad_arguments(vtlib):
         with pytest.raises(vtlib.VtError) as e:
             vtlib.vt_quantize_rows(w, bits, block)
         assert e.value.status == vtlib.VT_ERR_INVALID_ARG
+
+
+# ------------------------------------------------------------------ quantized partials (Section 4.3.2)
+
+@pytest.mark.parametrize("bits,qmax", [(8, 127), (4, 7)])
+def test_partial_grid_and_ties(bits, qmax):
+    """fp32 partials on the grid i * 2^-6 return their integers; halfway values round to even."""
+    i = np.arange(-qmax, qmax + 1)
+    q, sc = oracle.quantize_vec((i * 2.0 ** -6).astype(np.float32), bits, block=i.size)
+    assert sc[0] == np.float16(2.0 ** -6) and np.array_equal(q, i.astype(np.int8))
+    d = 2.0 ** -6
+    x = np.array([qmax * d, 2.5 * d, -2.5 * d, 1.5 * d, -0.5 * d], np.float32)
+    q, _ = oracle.quantize_vec(x, bits, block=5)
+    assert q.tolist() == [qmax, 2, -2, 2, 0]
+
+
+def test_partial_error_bound_and_zero_partial():
+    rng = np.random.default_rng(21)
+    x = (rng.standard_normal(4096) * 3.0).astype(np.float32)
+    for bits in (8, 4):
+        q, sc = oracle.quantize_vec(x, bits, block=32)
+        d = np.repeat(sc.astype(np.float64), 32)
+        assert np.all(np.abs(x.astype(np.float64) - q * d) <= d / 2 * (1 + 1e-6))
+    q, sc = oracle.quantize_vec(np.zeros(70, np.float32), 8, block=32)
+    assert not q.any() and not sc.astype(np.float64).any()
+
+
+def test_quantized_combine_equals_numpy_and_stays_within_the_bound():
+    """The combine of quantized partials is binary16(residual + sum of q * d) (numpy, fp64 sums,
+    round to nearest even), and differs from the unquantized combine by at most the partials'
+    half-steps plus the output's rounding."""
+    rng = np.random.default_rng(22)
+    D, n = 512, 3
+    parts = [(rng.standard_normal(D) * 0.5).astype(np.float32) for _ in range(n)]
+    res = rng.standard_normal(D).astype(np.float16)
+    for bits in (8, 4):
+        qp = [oracle.quantize_vec(p, bits) for p in parts]
+        got = oracle.combine_q(qp, res)
+        deq = [q.astype(np.float64) * np.repeat(s.astype(np.float64), 32) for q, s in qp]
+        want = (res.astype(np.float64) + sum(deq)).astype(np.float16)
+        assert np.array_equal(got.view(np.uint16), want.view(np.uint16))
+        exact = res.astype(np.float64) + sum(p.astype(np.float64) for p in parts)
+        half_steps = sum(np.repeat(s.astype(np.float64), 32) / 2 for _, s in qp)
+        ulp = np.abs(exact) * 2.0 ** -10 + 2.0 ** -24
+        assert np.all(np.abs(got.astype(np.float64) - exact) <= half_steps * (1 + 1e-6) + ulp)
+    # no residual and one zero partial: the other partial alone
+    z = oracle.quantize_vec(np.zeros(D, np.float32), 8)
+    one = oracle.quantize_vec(parts[0], 8)
+    assert np.array_equal(oracle.combine_q([z, one], None), oracle.combine_q([one], None))
