@@ -55,6 +55,9 @@ def lib():
         L.or_attn_partial.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32,
                                       _I32, _P, _I32, _P, _P, _P, _I64, _P]
         L.or_attn_partial.restype = _I32
+        L.or_attn_partial_window.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32,
+                                             _I32, _P, _I32, _P, _P, _P, _I64, _I64, _P]
+        L.or_attn_partial_window.restype = _I32
         L.or_ffn_partial.argtypes = [ctypes.POINTER(OrShapes), ctypes.POINTER(OrLayer), _I32,
                                      _I32, _P, _I32, _P]
         L.or_ffn_partial.restype = _I32
@@ -153,16 +156,18 @@ def kv_append(wl, weights, kv_heads: Tuple[int, int], x: np.ndarray, pos0: int,
 
 
 def attn_partial(wl, weights, heads: Tuple[int, int], x: np.ndarray, pos: Sequence[int],
-                 kcache: np.ndarray, vcache: np.ndarray) -> np.ndarray:
+                 kcache: np.ndarray, vcache: np.ndarray, window: int = 0) -> np.ndarray:
+    """ATTN partial of query heads `heads`; window > 0: sliding-window attention over the last
+    `window` positions (up to and including the row's own)."""
     x = _f16(x).reshape(-1, wl.d_model)
     p = np.ascontiguousarray(pos, dtype=np.int64)
     assert p.size == x.shape[0]
     out = np.empty((x.shape[0], wl.d_model), np.float64)
     s = shapes_of(wl)
     L, keep = layer_of(weights)
-    rc = lib().or_attn_partial(ctypes.byref(s), ctypes.byref(L), heads[0], heads[1],
-                               x.ctypes.data, x.shape[0], p.ctypes.data, _f16(kcache).ctypes.data,
-                               _f16(vcache).ctypes.data, kcache.shape[1], out.ctypes.data)
+    rc = lib().or_attn_partial_window(ctypes.byref(s), ctypes.byref(L), heads[0], heads[1],
+                                      x.ctypes.data, x.shape[0], p.ctypes.data, _f16(kcache).ctypes.data,
+                                      _f16(vcache).ctypes.data, kcache.shape[1], int(window), out.ctypes.data)
     if rc != 0:
         raise ValueError("or_attn_partial rejected its arguments")
     return out

@@ -202,6 +202,16 @@ int32_t or_attn_partial(const or_shapes* s, const or_layer* w, int32_t h0, int32
                         const uint16_t* x, int32_t rows, const int64_t* pos,
                         const uint16_t* kcache, const uint16_t* vcache, int64_t cap,
                         double* partial) {
+    return or_attn_partial_window(s, w, h0, h1, x, rows, pos, kcache, vcache, cap, 0, partial);
+}
+
+/* Sliding-window attention (Voltron Section 2.1 names it among the attention variants of the
+ * evaluated models): row i attends to cache positions [max(0, pos - window + 1), pos]; window <= 0
+ * means every position 0..pos. */
+int32_t or_attn_partial_window(const or_shapes* s, const or_layer* w, int32_t h0, int32_t h1,
+                               const uint16_t* x, int32_t rows, const int64_t* pos,
+                               const uint16_t* kcache, const uint16_t* vcache, int64_t cap,
+                               int64_t window, double* partial) {
     if (!shapes_ok(s) || !w || h0 < 0 || h1 < h0 || h1 > s->n_heads || rows < 0) return OR_ERR_ARG;
     for (int32_t i = 0; i < rows; ++i)
         if (pos[i] < 0 || pos[i] >= cap) return OR_ERR_ARG;
@@ -221,11 +231,13 @@ int32_t or_attn_partial(const or_shapes* s, const or_layer* w, int32_t h0, int32
         or_rmsnorm(xin, w->attn_norm, D, s->rms_eps, xh);
         matvec(w->wq + (int64_t)h0 * dh * D, D, (int64_t)nh * dh, xh, D, q);
         for (int32_t h = 0; h < nh; ++h) or_rope(q + (int64_t)h * dh, dh, pos[i], s->rope_theta);
+        const int64_t first = window > 0 && pos[i] + 1 > window ? pos[i] + 1 - window : 0;
 #pragma omp parallel for schedule(static)
         for (int32_t h = 0; h < nh; ++h) {
             const int32_t j = (h0 + h) / group;
-            or_attend(q + (int64_t)h * dh, kcache + (int64_t)j * cap * dh,
-                      vcache + (int64_t)j * cap * dh, pos[i] + 1, dh, NULL, o + (int64_t)h * dh);
+            or_attend(q + (int64_t)h * dh, kcache + ((int64_t)j * cap + first) * dh,
+                      vcache + ((int64_t)j * cap + first) * dh, pos[i] + 1 - first, dh, NULL,
+                      o + (int64_t)h * dh);
         }
         /* partial[d] = sum over the range's columns of Wo[d][h0*dh + k] * o[k] */
         matvec(w->wo + (int64_t)h0 * dh, (int64_t)H * dh, D, o, (int64_t)nh * dh, out);

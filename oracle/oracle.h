@@ -86,6 +86,13 @@ int32_t or_attn_partial(const or_shapes* s, const or_layer* w, int32_t h0, int32
                         const uint16_t* kcache, const uint16_t* vcache, int64_t cap,
                         double* partial);
 
+/* The same with a sliding window: row i attends to positions [max(0, pos[i] - window + 1), pos[i]]
+ * (window <= 0: all of 0..pos[i]). */
+int32_t or_attn_partial_window(const or_shapes* s, const or_layer* w, int32_t h0, int32_t h1,
+                               const uint16_t* x, int32_t rows, const int64_t* pos,
+                               const uint16_t* kcache, const uint16_t* vcache, int64_t cap,
+                               int64_t window, double* partial);
+
 /* FFN-block partial output of intermediate columns [c0, c1) for `rows` rows of h (binary16):
  * RMSNorm, a_j = silu(Wg[j] h^) * (Wu[j] h^), partial = Wd[:, c0:c1] . a (fp64 [rows, D]). */
 int32_t or_ffn_partial(const or_shapes* s, const or_layer* w, int32_t c0, int32_t c1,

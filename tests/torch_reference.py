@@ -33,8 +33,10 @@ def _rope_complex(t: torch.Tensor, pos: torch.Tensor, theta: float) -> torch.Ten
     return torch.cat([z.real, z.imag], dim=-1)
 
 
-def layer(wl, w, x: np.ndarray, pos0: int, k_prefix: np.ndarray | None, v_prefix: np.ndarray | None):
-    """Full (unpartitioned) decoder layer on rows at positions pos0..pos0+rows-1.
+def layer(wl, w, x: np.ndarray, pos0: int, k_prefix: np.ndarray | None, v_prefix: np.ndarray | None,
+          window: int = 0):
+    """Full (unpartitioned) decoder layer on rows at positions pos0..pos0+rows-1; window > 0 bands
+    the causal mask to the last `window` positions of each row (sliding-window attention).
 
     k_prefix / v_prefix: fp16 [Hk, pos0, dh] cache content before the call (or None when pos0 = 0).
     Returns a dict with attn_out, h (fp16), ffn_out, x_next (fp16), k_new / v_new (fp16 [Hk, rows, dh]).
@@ -62,6 +64,8 @@ def layer(wl, w, x: np.ndarray, pos0: int, k_prefix: np.ndarray | None, v_prefix
     Vt = _t(V).repeat_interleave(g, dim=0)[None]
     L = pos0 + rows
     mask = torch.arange(L)[None, :] <= (pos0 + torch.arange(rows))[:, None]
+    if window > 0:
+        mask &= torch.arange(L)[None, :] > (pos0 + torch.arange(rows))[:, None] - window
     o = F.scaled_dot_product_attention(q.permute(1, 0, 2)[None], Kt, Vt, attn_mask=mask)
     attn = o[0].permute(1, 0, 2).reshape(rows, H * dh)
     attn_out = F.linear(attn, _t(w["wo"]))
