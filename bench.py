@@ -34,6 +34,9 @@ import numpy as np  # noqa: E402
 import synthetic  # noqa: E402
 
 METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline"
+WORKLOAD = ("llama2-7b-shaped batch-1 decode: 32 layers, D 4096, 32 heads x 128 (MHA), "
+            "FFN 11008 SwiGLU; even 4-way TP (8 heads, 2752 FFN columns per shard), "
+            "shards run one after another on 1 GPU; KV 1024 -> 1151 (128-step schedule)")
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
@@ -428,9 +431,7 @@ def run_decode(args, rank, world):
         "dtype": "fp16",
         "data": "synthetic (seeded N(0,0.02) fp16 weights, seeded N(0,(0.02*sqrt(D))^2) KV cache)",
         "config": {
-            "workload": "llama2-7b-shaped batch-1 decode: 32 layers, D 4096, 32 heads x 128 (MHA), "
-                        "FFN 11008 SwiGLU; even 4-way TP (8 heads, 2752 FFN columns per shard), "
-                        "shards run one after another on 1 GPU; KV 1024 -> 1151 (128-step schedule)",
+            "workload": WORKLOAD,
             "kv_len_start": wl.kv_len,
             "kv_schedule_steps": sched,
             "partition": "heads 8/8/8/8, ffn 2752 x 4",
@@ -551,7 +552,8 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(per_token * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": "llama2-7b-shaped batch-1 decode, 4-way TP, KV 1024 (CPU oracle)"},
+            "config": {"workload": WORKLOAD, "kv_len_start": L0, "partition": "heads 8/8/8/8, ffn 2752 x 4",
+                       "implementation": "CPU oracle (fp64), one layer per step, x32 by layers"},
             "cpu_baseline": {"value": round(value, 4), "unit": "tok/s", "cores": oracle.num_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 4), "unit": "tok/s", "h2d_bytes_per_step": 0,
