@@ -16,7 +16,7 @@ def declared_symbols():
     return sorted(set(re.findall(r"^VT_API\s+[^;(]*?\b(vt_[a-z0-9_]+)\s*\(", text, flags=re.M)))
 
 
-def test_header_declares_the_north_star_calls():
+def test_header_declares_the_core_calls():
     names = declared_symbols()
     for must in ("vt_model_create", "vt_partition_create", "vt_prefill", "vt_decode_step",
                  "vt_combine", "vt_kv_create", "vt_decode_token", "vt_prefill_tokens"):
