@@ -287,3 +287,29 @@ def test_plan_layers_invalid_arguments(vtlib, kw):
     with pytest.raises(vtlib.VtError) as e:
         vtlib.vt_plan_layers(s, **args)
     assert e.value.status == vtlib.VT_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_plans_are_always_valid_partitions(vtlib, seed):
+    """Random shapes, device counts, rates and budgets: the share balancer's and the layer plan's
+    ranges always pass vt_partition_validate (whole KV groups, full coverage, device order)."""
+    rng = np.random.default_rng(900 + seed)
+    H = int(rng.choice([4, 8, 16, 32, 40]))
+    Hk = int(rng.choice([g for g in (1, 2, 4, 8, 16, 32, 40) if H % g == 0 and H // g in (1, 2, 4, 8)]))
+    F = int(rng.integers(1, 3000))
+    s = vtlib.make_shapes(2, 256, H, Hk, 64, F, 0, 128)
+    n = int(rng.integers(1, 9))
+    rates = [float(x) for x in rng.uniform(0.1, 10.0, n)]
+    heads, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_ATTN, rates)
+    cols, _ = vtlib.vt_plan_tp_shares(s, vtlib.VT_BLOCK_FFN, rates, col_unit=int(rng.choice([1, 8, 64])))
+    assert vtlib.vt_partition_validate(s, heads, cols) == vtlib.VT_OK
+    plans, total = vtlib.vt_plan_layers(s, rates, link_bytes_per_s=float(10 ** rng.uniform(5, 12)),
+                                        link_latency_s=float(rng.uniform(0, 1e-2)), tokens=int(rng.integers(1, 64)),
+                                        kv_len=int(rng.integers(0, 64)))
+    assert total > 0
+    for i in range(0, len(plans), 2):
+        assert vtlib.vt_partition_validate(s, plans[i]["ranges"], plans[i + 1]["ranges"]) == vtlib.VT_OK
+        for p in plans[i:i + 2]:
+            if not p["tp"]:
+                sizes_ = [b - a for a, b in p["ranges"]]
+                assert sum(1 for x in sizes_ if x) == 1 and sizes_[p["device"]] > 0
