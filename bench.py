@@ -9,8 +9,10 @@ Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs r
 `e2e` is the same metric through the C ABI with host buffers (token id H2D, hidden state D2H,
 synchronised every step); `roofline` is the token kernel's achieved HBM bandwidth (algorithmic
 bytes of the step over its time); `sharded_token` times the same token as per-shard kernels;
-`cpu_baseline` is the CPU oracle timed on a bounded sample; `prefill` is the 512-token prompt of the
-7B prefill workload through the same stack (tok/s and tensor-core rate); `other_workloads` are the
+`cpu_baseline` is the CPU oracle timed on a bounded sample (all host threads, and one thread in
+`value_1thread`); `prefill` is the 512-token prompt of the 7B prefill workload through the same
+stack (tok/s and tensor-core rate, with the oracle's prefill in `prefill.cpu_baseline`);
+`other_workloads` are the
 13B (uneven 3-way, KV 2048) and 8B GQA (4-way, KV 4096) decode shapes timed the same way.
 `--impl reference` times the CPU oracle alone.
 """
