@@ -12,8 +12,8 @@ bytes of the step over its time); `sharded_token` times the same token as per-sh
 `cpu_baseline` is the CPU oracle timed on a bounded sample (all host threads, and one thread in
 `value_1thread`); `prefill` is the 512-token prompt of the 7B prefill workload through the same
 stack (tok/s and tensor-core rate, with the oracle's prefill in `prefill.cpu_baseline`);
-`other_workloads` are the
-13B (uneven 3-way, KV 2048) and 8B GQA (4-way, KV 4096) decode shapes timed the same way.
+`other_workloads` are the 13B (uneven 3-way, KV 2048) and 8B GQA (4-way, KV 4096) decode shapes
+timed the same way.
 `--impl reference` times the CPU oracle alone.
 """
 from __future__ import annotations
