@@ -2,8 +2,11 @@
 
 One step = one decode token through all 32 layers: for each layer every ATTN shard (4 of them),
 the on-device combine, every FFN shard, the combine; then the KV lengths advance.  The token step
-is one CUDA graph of vt_decode_token (one fused cooperative kernel) replayed K times; the KV length
-runs 1024 -> 1151 and rewinds to 1024 every 128 steps (the 128-step schedule of the workload).
+is one CUDA graph of vt_decode_token (one fused cooperative kernel, in which the shards of a block
+run side by side, each with its own fp32 partial, and the combines add them in shard order)
+replayed K times; the KV length runs 1024 -> 1151 and rewinds to 1024 every 128 steps (the
+128-step schedule of the workload).  The K-step timed region is repeated until it covers
+--min-timed-s seconds, so the clock sampler sees enough samples; ms_per_step is the median.
 
 Printed: one JSON line (rank 0).  `value` is device-timed tokens/s with inputs resident in HBM;
 `e2e` is the same metric through the C ABI with host buffers (token id H2D, hidden state D2H,
@@ -37,8 +40,9 @@ import synthetic  # noqa: E402
 
 METRIC = "batch-1 decode tok/s (7B fp16, all shards on 1 GPU); % of HBM roofline"
 WORKLOAD = ("llama2-7b-shaped batch-1 decode: 32 layers, D 4096, 32 heads x 128 (MHA), "
-            "FFN 11008 SwiGLU; even 4-way TP (8 heads, 2752 FFN columns per shard), "
-            "shards run one after another on 1 GPU; KV 1024 -> 1151 (128-step schedule)")
+            "FFN 11008 SwiGLU; even 4-way TP (8 heads, 2752 FFN columns per shard), all shards on "
+            "1 GPU: the shards of a block run side by side inside one launch, each keeping its own "
+            "fp32 partial, combined in shard order; KV 1024 -> 1151 (128-step schedule)")
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
@@ -76,7 +80,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "25"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
             time.sleep(0.3)
         except FileNotFoundError:
@@ -250,7 +254,8 @@ def run_prefill(vt, st, wl, stream, steps, warmup):
     launches = 2 + wl.n_layers * (3 * n_dev + 1 + 2 * n_dev + 1) + 2
     return {
         "workload": f"llama2-7b-shaped prefill: {n}-token prompt (seeded ids, embedding gather), "
-                    f"{wl.n_layers} layers, even {n_dev}-way TP, shards one after another on 1 GPU",
+                    f"{wl.n_layers} layers, even {n_dev}-way TP on 1 GPU (one grouped GEMM launch per "
+                    f"projection covers every shard, each with its own fp32 partial)",
         "value": round(n / (ms * 1e-3), 1), "unit": "tok/s", "ms_per_prompt": round(ms, 4),
         "steps": steps, "warmup": warmup,
         "gemm_tflop_per_prompt": round(gemm / 1e12, 4),
@@ -282,7 +287,8 @@ class TokenSchedule:
         self.reset()
 
     def reset(self):
-        # the captures moved the host-side length mirror; put device and host back at kv_len
+        # replays advance the device lengths (captures leave them and the host mirror alone):
+        # put both back at kv_len
         self.vt.vt_kv_set_length(self.st.kv, -1, self.kv_len, self.stream)
         self.pos = 0
 
@@ -349,24 +355,39 @@ def run_decode(args, rank, world):
         stream.synchronize()
         sch = TokenSchedule(vt, st, vt.vt_decode_token, xin, xout, stream, sched, wl.kv_len)
 
+        # warm-up steps, timed once to size the measurement: the timed region is exactly K steps,
+        # repeated R times (R from the warm-up rate, the same on every rank) so that the clock
+        # sampler sees at least ~10 samples at 25 ms; ms_per_step is the median repeat
+        w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
+            w0.record(stream)
             for _ in range(args.warmup):
                 sch.step()
-        stream.synchronize()
-        sch.reset()
+            w1.record(stream)
+        w1.synchronize()
+        est_ms = w0.elapsed_time(w1) / max(args.warmup, 1)
+        repeats = int(min(64, max(1, np.ceil(args.min_timed_s * 1e3 / max(est_ms * args.steps, 1e-3)))))
         if world > 1:
-            torch.distributed.barrier()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t = torch.tensor([repeats], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            repeats = int(t.item())
+        sch.reset()
+        rep_ms = []
         with ClockSampler(torch.cuda.current_device()) as clk:
-            with torch.cuda.stream(stream):
-                e0.record(stream)
-                for _ in range(args.steps):
-                    sch.step()
-                e1.record(stream)
-            e1.synchronize()
-        torch.cuda.synchronize()
-        ms = e0.elapsed_time(e1)
+            for _ in range(repeats):
+                if world > 1:
+                    torch.distributed.barrier()
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with torch.cuda.stream(stream):
+                    e0.record(stream)
+                    for _ in range(args.steps):
+                        sch.step()
+                    e1.record(stream)
+                e1.synchronize()
+                torch.cuda.synchronize()
+                rep_ms.append(e0.elapsed_time(e1))
+        ms = float(np.median(rep_ms))
         if world > 1:
             t = torch.tensor([ms], device="cuda")
             torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -460,6 +481,8 @@ def run_decode(args, rank, world):
         },
         "e2e": {"value": round(world / e2e_s, 3), "unit": "tok/s", "h2d_bytes_per_step": 4,
                 "d2h_bytes_per_step": 2 * D, "finite": e2e_finite},
+        "timed_repeats": repeats,
+        "ms_per_step_repeats": [round(r / args.steps, 5) for r in rep_ms],
         "gpu_launches": launches_per_token * args.steps + (args.steps // sched),
         "device_status": {"kv": kv_status, "partition": part_status},
         "setup_s": round(setup_s, 1),
@@ -548,14 +571,16 @@ def run_reference(args):
     dt = (time.perf_counter() - t0) / max(args.steps, 1)
     per_token = dt * wl.n_layers
     value = 1.0 / per_token
-    sample = (f"each step: one decode token through layer 0 of 32 (4-way TP shards, KV from {L0}); "
-              f"tok/s = 1 / (32 x layer time)")
+    sample = (f"each step: one decode token through layer 0 of 32 (4-way TP shards, KV from {L0}), "
+              f"timed; tok/s = 1 / (32 x step time), the x32 by layers stated in ms_per_token_extrapolated")
     return {"metric": METRIC, "value": round(value, 4), "unit": "tok/s", "n_gpus": 1,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(per_token * 1e3, 3),
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3),
+            "ms_per_token_extrapolated": round(per_token * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
             "config": {"workload": WORKLOAD, "kv_len_start": L0, "partition": "heads 8/8/8/8, ffn 2752 x 4",
-                       "implementation": "CPU oracle (fp64), one layer per step, x32 by layers"},
+                       "implementation": "CPU oracle (fp64); a step is one layer of the token (timed), "
+                                         "value extrapolated x32 by layers"},
             "cpu_baseline": {"value": round(value, 4), "unit": "tok/s", "cores": oracle.num_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 4), "unit": "tok/s", "h2d_bytes_per_step": 0,
@@ -575,6 +600,8 @@ def main():
                     help="timed tokens of the per-shard entry point, for context (0: skip)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: only the first N layers of the stack")
+    ap.add_argument("--min-timed-s", type=float, default=0.3,
+                    help="repeat the K-step timed region until it covers this many seconds in total")
     ap.add_argument("--other-steps", type=int, default=64,
                     help="timed tokens of the 13B and 8B decode workloads, 1 GPU only (0: skip)")
     args = ap.parse_args()

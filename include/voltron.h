@@ -35,7 +35,12 @@
  *  - Threads: objects are not internally locked; use one object from one host thread at a time.
  *  - Streams and graphs: every compute call except vt_decode_step_static can be captured into a
  *    CUDA graph; positions come from device-resident KV lengths, so a replayed graph appends at
- *    the right place.  (No claim is made for vt_decode_step_static.)
+ *    the right place.  (No claim is made for vt_decode_step_static.)  While the stream is being
+ *    captured, calls record device work only and leave the host-side mirror of the KV lengths
+ *    unchanged; replays advance the device lengths alone, and vt_kv_length refreshes the mirror.
+ *    vt_kv_set_length and the synchronous test hooks cannot be captured.
+ *  - Citations: each declaration names the section of Voltron that defines its operation; calls
+ *    that are library plumbing (object lifetime, status words, test hooks) say so.
  */
 #ifndef VOLTRON_H
 #define VOLTRON_H
@@ -72,6 +77,7 @@ typedef int32_t vt_status;
 /* Bits of the device status word. */
 #define VT_DEV_KV_OVERFLOW 1u     /* a kernel saw a KV length at or past capacity and skipped */
 #define VT_DEV_WAIT_TIMEOUT 2u    /* a kernel gave up waiting on an asynchronous copy */
+#define VT_DEV_BAD_TOKEN 4u       /* the embedding gather saw a token id outside [0, vocab) */
 
 typedef void* vt_stream; /* a cudaStream_t; NULL is the legacy default stream */
 
@@ -127,14 +133,17 @@ typedef struct vt_model vt_model;
 typedef struct vt_partition vt_partition;
 typedef struct vt_kv vt_kv;
 
-/* Text of the last error on the calling thread ("" if none).  Valid until the next call. */
+/* Library plumbing (no paper counterpart).  Text of the last error on the calling thread ("" if
+ * none).  Valid until the next call. */
 VT_API const char* vt_last_error(void);
 
-/* Library version, "major.minor.patch". */
+/* Library plumbing.  Library version, "major.minor.patch". */
 VT_API const char* vt_version(void);
 
-/* Host-only checks (no GPU needed).  vt_shapes_validate returns VT_OK or VT_ERR_SHAPE.
- * vt_partition_validate applies the partition rules of vt_partition below. */
+/* Host-only checks (no GPU needed).  vt_shapes_validate returns VT_OK or VT_ERR_SHAPE: the
+ * decoder-layer shapes of Section 2.1 ("LLM Architecture": attention heads, GQA groups, FFN) that
+ * the kernels support.  vt_partition_validate applies the partition rules of vt_partition below
+ * (Section 3.2.1 head/column shards, Section 4.2.1 uneven shares). */
 VT_API vt_status vt_shapes_validate(const vt_shapes* shapes);
 VT_API vt_status vt_partition_validate(const vt_shapes* shapes, int32_t n_devices,
                                 const vt_range* head_ranges, const vt_range* ffn_col_ranges);
@@ -209,7 +218,8 @@ VT_API vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, int32_
                                   void* scales);
 
 /* ---------------------------------------------------------------- model ------------------------
- * vt_model_create: allocates device storage for every layer in the canonical (unpartitioned)
+ * vt_model_create (Section 2.1, "LLM Architecture": the decoder layers the shards are cut from;
+ * the weights are the unpartitioned layer before Section 3.2.1 splits it): allocates device storage for every layer in the canonical (unpartitioned)
  * layout, the RoPE table for positions [0, max_seq) and, if vocab > 0, the embedding table, on
  * the current CUDA device.  per_layer (nullable) holds n_layers host weight sets, copied now;
  * embed (nullable) is the host fp16 table [vocab, D].  Layers not given here are loaded later
@@ -218,14 +228,22 @@ VT_API vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, int32_
 VT_API vt_status vt_model_create(const vt_shapes* shapes, const vt_layer_weights* per_layer,
                           const void* embed, const vt_allocator* allocator, vt_stream stream,
                           vt_model** out);
+/* Library plumbing for vt_model_create: load one layer's weights (copied now, synchronizes the
+ * stream), load the embedding table, read the shapes back, free everything. */
 VT_API vt_status vt_model_load_layer(vt_model* model, int32_t layer, const vt_layer_weights* weights,
                               vt_stream stream);
 VT_API vt_status vt_model_load_embedding(vt_model* model, const void* embed, vt_stream stream);
 VT_API vt_status vt_model_shapes(const vt_model* model, vt_shapes* out);
 VT_API void vt_model_destroy(vt_model* model);
+/* Library plumbing.  Reads the model's device status word (VT_DEV_BAD_TOKEN from vt_embed),
+ * synchronizing the device; clear != 0 resets it. */
+VT_API vt_status vt_model_status(vt_model* model, uint32_t* flags, int32_t clear);
 
-/* Embedding gather: out[i, :] = E[ids[i], :] for i < n.  ids: device int32 [n] (values outside
- * [0, vocab) give a zero row and set no error); out: device fp16 [n, D]. */
+/* Embedding gather (Section 2.1, "LLM Architecture": token ids enter the stack as embedding
+ * rows): out[i, :] = E[ids[i], :] for i < n, copied bit for bit.  ids: device int32 [n]; out:
+ * device fp16 [n, D], 16-byte aligned.  An id outside [0, vocab) gives a zero row and sets
+ * VT_DEV_BAD_TOKEN in the model's status word (vt_model_status); the call itself still returns
+ * VT_OK, since the ids are only seen on the device.  VT_ERR_STATE without a loaded table. */
 VT_API vt_status vt_embed(const vt_model* model, const int32_t* ids, int32_t n, void* out,
                    vt_stream stream);
 
@@ -243,13 +261,15 @@ VT_API vt_status vt_embed(const vt_model* model, const int32_t* ids, int32_t n, 
 VT_API vt_status vt_partition_create(vt_model* model, int32_t n_devices, const vt_range* head_ranges,
                               const vt_range* ffn_col_ranges, vt_stream stream,
                               vt_partition** out);
+/* Library plumbing: the partition's device count; its device status word (VT_DEV_* bits of
+ * kernels that have no KV cache; synchronizes the device; clear != 0 resets it and re-arms the
+ * fused decode kernel's grid barrier); destruction (the model must still exist). */
 VT_API int32_t vt_partition_devices(const vt_partition* part);
-/* Reads the device status word (VT_DEV_* bits) of kernels that have no KV cache, synchronizing
- * the device; clear != 0 resets it. */
 VT_API vt_status vt_partition_status(vt_partition* part, uint32_t* flags, int32_t clear);
 VT_API void vt_partition_destroy(vt_partition* part);
 
-/* Test hook: copies one tensor of a shard's sliced weights to host memory.  which: 0 = attention
+/* Test hook (library plumbing; the slicing itself is Section 3.2.1's head/column split): copies
+ * one tensor of a shard's sliced weights to host memory.  which: 0 = attention
  * RMSNorm gain, 1 = fused QKV rows, 2 = O columns, 3 = FFN RMSNorm gain, 4 = fused gate/up rows,
  * 5 = down columns.  Copies min(bytes, size) bytes; *size_out (nullable) receives the size.
  * Layouts are documented beside vt_shard_weight_layout.  Synchronous. */
@@ -267,22 +287,29 @@ VT_API vt_status vt_shard_weight_layout(const vt_partition* part, vt_shard shard
                                  int64_t* rows, int64_t* row_stride);
 
 /* ---------------------------------------------------------------- KV cache ---------------------
- * vt_kv_create: per (layer, device) fp16 caches K and V, each [hk_s][capacity][dh] for that
+ * vt_kv_create (Section 2.1, "LLM Inference": the KV cache that prefill fills and every decode
+ * step appends to; split by KV head among the devices as tensor parallelism splits the heads,
+ * Section 3.2.1): per (layer, device) fp16 caches K and V, each [hk_s][capacity][dh] for that
  * device's KV heads (tensor parallelism splits the cache by head), plus one device-resident length
  * per layer (initially 0) and a host mirror of it.  capacity <= max_seq.  Contents start zeroed.
  */
 VT_API vt_status vt_kv_create(const vt_partition* part, int32_t capacity, vt_stream stream, vt_kv** out);
+/* Library plumbing: destruction and the capacity given at creation. */
 VT_API void vt_kv_destroy(vt_kv* kv);
 VT_API int32_t vt_kv_capacity(const vt_kv* kv);
-/* Adds n to the length of `layer` (or of every layer when layer == -1), on the device (in stream
+/* Cache bookkeeping (Section 2.1: each decode step appends one position, a prefill n).  Adds n
+ * to the length of `layer` (or of every layer when layer == -1), on the device (in stream
  * order) and in the host mirror.  Decode and prefill append at the current length without
  * advancing it: advance once per layer after all of that layer's attention shards ran. */
 VT_API vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_stream stream);
-/* Sets the length of `layer` (or all when -1) to len, device and host mirror. */
+/* Cache bookkeeping: sets the length of `layer` (or all when -1) to len, device and host
+ * mirror; synchronizes the stream (not capturable). */
 VT_API vt_status vt_kv_set_length(vt_kv* kv, int32_t layer, int32_t len, vt_stream stream);
-/* Reads the device length of `layer` (synchronizes the stream) and refreshes the host mirror. */
+/* Cache bookkeeping: reads the device length of `layer` (synchronizes the stream) and refreshes
+ * the host mirror. */
 VT_API vt_status vt_kv_length(vt_kv* kv, int32_t layer, vt_stream stream, int32_t* len);
-/* Reads (and with clear != 0 resets) the device status word of kernels that used this cache. */
+/* Library plumbing: reads (and with clear != 0 resets) the device status word of kernels that
+ * used this cache. */
 VT_API vt_status vt_kv_status(vt_kv* kv, uint32_t* flags, int32_t clear);
 /* Test hooks, synchronous: copy positions [0, n_pos) of the (layer, device) cache between device
  * and host.  Host layout [hk_s][n_pos][dh] fp16 for K and for V. */
@@ -292,7 +319,9 @@ VT_API vt_status vt_kv_write_raw(vt_kv* kv, int32_t layer, int32_t device, int32
                           const void* k_host, const void* v_host);
 
 /* ---------------------------------------------------------------- shard compute ----------------
- * vt_decode_step: one decode token through one shard.
+ * vt_decode_step (Section 2.1, decode phase; Section 3.2.1, one device's shard of a tensor-
+ * parallel layer, the ATTN and FFN blocks being separate layers as in Section 4.2.1): one decode
+ * token through one shard.
  *   ATTN shard (kv required): x^ = RMSNorm(x); q, k, v of the shard's heads; RoPE on q and k at
  *   position p = current length of the layer; k, v appended at p; attention of each query head
  *   over positions 0..p (split-K flash decoding); out_partial = Wo[:, shard cols] . attn.
@@ -331,7 +360,8 @@ VT_API vt_status vt_decode_step(const vt_partition* part, vt_shard shard, const 
 VT_API vt_status vt_decode_step_static(const vt_partition* part, vt_shard shard, const void* x, vt_kv* kv,
                                 float* out_partial, vt_stream stream);
 
-/* vt_prefill: n prompt rows through one shard (n >= 1).
+/* vt_prefill (Section 2.1, prefill phase: the prompt in parallel, K/V written to the cache;
+ * Section 3.2.1 shard): n prompt rows through one shard (n >= 1).
  *   ATTN shard: rows sit at positions p0..p0+n-1 with p0 = current length of the layer; row i
  *   attends causally to positions 0..p0+i (earlier turns' cache included).  K and V of all rows
  *   are appended.  FFN shard: as decode, row by row.
@@ -340,7 +370,7 @@ VT_API vt_status vt_decode_step_static(const vt_partition* part, vt_shard shard,
 VT_API vt_status vt_prefill(const vt_partition* part, vt_shard shard, const void* x, int32_t n,
                      vt_kv* kv, float* out_partial, vt_stream stream);
 
-/* vt_combine: the aggregation on the main device.
+/* vt_combine (Section 3.2.1: the shard results are aggregated on the main device): the sum.
  *   out[e] = fp16(residual[e] + sum_{s=0}^{n-1} partials[s][e]), e < rows*d, summed in fp32 in
  *   the order s = 0..n-1.  partials: host array of n device pointers to fp32 [rows, d];
  *   residual: device fp16 [rows, d] or NULL; out: device fp16 [rows, d] (may alias residual).
@@ -370,18 +400,29 @@ VT_API vt_status vt_combine(const float* const* partials, int32_t n, int32_t row
  */
 VT_API vt_status vt_decode_token(const vt_partition* part, vt_kv* kv, const void* x_in, void* x_out,
                           vt_stream stream);
-/* The same token as a sequence of per-shard kernels (3 per ATTN shard, 1 per FFN shard, one
- * combine per block, one length update), linked by programmatic dependent launch. */
+/* The same token (Sections 2.1 and 3.2.1, as vt_decode_token) as a sequence of per-shard
+ * kernels (3 per ATTN shard, 1 per FFN shard, one combine per block, one length update), linked
+ * by programmatic dependent launch: vt_decode_step for every shard, one after another, and
+ * vt_combine per block. */
 VT_API vt_status vt_decode_token_sharded(const vt_partition* part, vt_kv* kv, const void* x_in,
                                          void* x_out, vt_stream stream);
-/* 1 if vt_decode_token runs as one fused kernel for this partition, else 0; *why (optional)
+/* Library plumbing: 1 if vt_decode_token runs as one fused kernel for this partition, else 0; *why (optional)
  * receives the reason when it does not (valid while the partition lives).  Fused needs a
  * device with cooperative launch, d_model a multiple of 8 and at most 6144, d_head 64 or 128,
  * 1, 2 or 4 query heads per KV head, at most as many KV heads as SMs, at most 256 layers, and
  * at most 256 QKV rows per SM. */
 VT_API int32_t vt_decode_token_fused_available(const vt_partition* part, const char** why);
-/* vt_prefill_tokens: n prompt rows through every layer (same order as vt_decode_token), then
- * every layer's KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same. */
+/* Test hook (library plumbing): copies the fp32 shard partials [n_devices][D] of the last layer
+ * that the fused decode-token kernel computed (block VT_BLOCK_ATTN: the O-projection partials;
+ * VT_BLOCK_FFN: the down-projection partials) to host memory, after synchronizing the device.
+ * Valid after a vt_decode_token that ran fused; VT_ERR_STATE when the partition has no fused
+ * kernel. */
+VT_API vt_status vt_token_partials_read(const vt_partition* part, int32_t block, float* host_dst);
+/* vt_prefill_tokens (Section 2.1, prefill phase, through the tensor-parallel layers of Section
+ * 3.2.1): n prompt rows through every layer (same order as vt_decode_token), then every layer's
+ * KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same.  The shards of a
+ * block run together: one tensor-core GEMM launch per projection covers every shard (each with
+ * its own partial), then the combine adds them in shard order. */
 VT_API vt_status vt_prefill_tokens(const vt_partition* part, vt_kv* kv, const void* x_in, int32_t n,
                             void* x_out, vt_stream stream);
 

@@ -62,6 +62,17 @@ vt_status ok() {
     } while (0)
 
 inline size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+inline bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
+// True while `st` is being captured into a CUDA graph: calls then record device work only and
+// leave the host-side mirror of the KV lengths alone (replays advance the device lengths).
+inline bool capturing(cudaStream_t st) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return cs == cudaStreamCaptureStatusActive;
+}
 inline int round_up8(int k) { return (k + 7) & ~7; }
 
 // ------------------------------------------------------------------ allocator
@@ -128,6 +139,7 @@ struct vt_model {
     __half* embed = nullptr;
     bool embed_loaded = false;
     float2* rope = nullptr;
+    uint32_t* status = nullptr;  // device status word of the embedding gather
 };
 
 struct AttnShard {
@@ -496,6 +508,21 @@ extern "C" vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, in
 
 // ================================================================== model
 
+// With `clear`, also re-arms the decode-token kernel's grid barrier and abort word: a token that
+// gave up on a wait leaves them in an unknown state (the call that read the flags synchronised the
+// device, so no kernel is using them).
+static vt_status read_status(uint32_t* dev, uint32_t* flags, int32_t clear, uint32_t* tok_sync) {
+    if (!flags) return fail(VT_ERR_INVALID_ARG, "flags is NULL");
+    VT_CUDA(cudaDeviceSynchronize());
+    VT_CUDA(cudaMemcpy(flags, dev, 4, cudaMemcpyDeviceToHost));
+    if (clear) {
+        VT_CUDA(cudaMemset(dev, 0, 4));
+        if (tok_sync) VT_CUDA(cudaMemset(tok_sync, 0, (size_t)kTokSyncWords * sizeof(uint32_t)));
+    }
+    return ok();
+}
+
+
 static vt_status upload(void* dst, const void* src, size_t bytes, cudaStream_t st) {
     if (!src) return fail(VT_ERR_INVALID_ARG, "a weight pointer is NULL");
     VT_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st));
@@ -541,6 +568,7 @@ extern "C" void vt_model_destroy(vt_model* m) {
     for (void* p : m->layer_base) m->alloc.put(p);
     m->alloc.put(m->embed);
     m->alloc.put(m->rope);
+    m->alloc.put(m->status);
     delete m;
 }
 
@@ -592,6 +620,15 @@ extern "C" vt_status vt_model_create(const vt_shapes* shapes, const vt_layer_wei
             return fail(VT_ERR_ALLOC, "allocating the embedding table failed");
         }
     }
+    m->status = static_cast<uint32_t*>(m->alloc.get(256));
+    if (!m->status) {
+        vt_model_destroy(m);
+        return fail(VT_ERR_ALLOC, "allocating the model status word failed");
+    }
+    if (cudaMemsetAsync(m->status, 0, 256, st) != cudaSuccess) {
+        vt_model_destroy(m);
+        return fail(VT_ERR_CUDA, "clearing the model status word failed");
+    }
     const size_t rope_bytes = (size_t)s.max_seq * (s.d_head / 2) * sizeof(float2);
     m->rope = static_cast<float2*>(m->alloc.get(rope_bytes));
     if (!m->rope) {
@@ -638,12 +675,18 @@ extern "C" vt_status vt_model_shapes(const vt_model* m, vt_shapes* out) {
     return ok();
 }
 
+extern "C" vt_status vt_model_status(vt_model* m, uint32_t* flags, int32_t clear) {
+    if (!m) return fail(VT_ERR_INVALID_ARG, "model is NULL");
+    return read_status(m->status, flags, clear, nullptr);
+}
+
 extern "C" vt_status vt_embed(const vt_model* m, const int32_t* ids, int32_t n, void* out,
                               vt_stream stream) {
     if (!m || (!ids && n > 0) || (!out && n > 0) || n < 0)
         return fail(VT_ERR_INVALID_ARG, "bad vt_embed arguments");
     if (!m->embed || !m->embed_loaded) return fail(VT_ERR_STATE, "no embedding table loaded");
-    VT_CUDA(launch_embed(m->embed, ids, n, m->s.d_model, m->s.vocab, static_cast<__half*>(out),
+    if (n > 0 && !aligned16(out)) return fail(VT_ERR_INVALID_ARG, "out must be 16-byte aligned");
+    VT_CUDA(launch_embed(m->embed, ids, n, m->s.d_model, m->s.vocab, static_cast<__half*>(out), m->status,
                          (cudaStream_t)stream));
     return ok();
 }
@@ -883,26 +926,10 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
 
 extern "C" int32_t vt_partition_devices(const vt_partition* p) { return p ? p->n_dev : 0; }
 
-// With `clear`, also re-arms the decode-token kernel's grid barrier and abort word: a token that
-// gave up on a wait leaves them in an unknown state (the call that read the flags synchronised the
-// device, so no kernel is using them).
-static vt_status read_status(uint32_t* dev, uint32_t* flags, int32_t clear, uint32_t* tok_sync) {
-    if (!flags) return fail(VT_ERR_INVALID_ARG, "flags is NULL");
-    VT_CUDA(cudaDeviceSynchronize());
-    VT_CUDA(cudaMemcpy(flags, dev, 4, cudaMemcpyDeviceToHost));
-    if (clear) {
-        VT_CUDA(cudaMemset(dev, 0, 4));
-        if (tok_sync) VT_CUDA(cudaMemset(tok_sync, 0, (size_t)kTokSyncWords * sizeof(uint32_t)));
-    }
-    return ok();
-}
-
 extern "C" vt_status vt_partition_status(vt_partition* p, uint32_t* flags, int32_t clear) {
     if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
     return read_status(p->status, flags, clear, p->tok_base.sync);
 }
-
-static bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
 static vt_status check_shard(const vt_partition* p, vt_shard sh) {
     if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
@@ -1070,7 +1097,8 @@ extern "C" vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_strea
             return fail(VT_ERR_KV_CAPACITY, "advancing layer %d from %d by %d leaves [0, %d]", l,
                         kv->h_len[l], n, kv->cap);
     VT_CUDA(launch_kv_advance(kv->len, first, count, n, (cudaStream_t)stream));
-    for (int l = first; l < first + count; ++l) kv->h_len[l] += n;
+    if (!capturing((cudaStream_t)stream))
+        for (int l = first; l < first + count; ++l) kv->h_len[l] += n;
     return ok();
 }
 
@@ -1498,6 +1526,16 @@ extern "C" int32_t vt_decode_token_fused_available(const vt_partition* p, const 
     return p && p->tok_ok ? 1 : 0;
 }
 
+extern "C" vt_status vt_token_partials_read(const vt_partition* p, int32_t block, float* host_dst) {
+    if (!p || !host_dst || (block != VT_BLOCK_ATTN && block != VT_BLOCK_FFN))
+        return fail(VT_ERR_INVALID_ARG, "bad vt_token_partials_read arguments");
+    if (!p->tok_ok) return fail(VT_ERR_STATE, "the partition has no fused decode-token kernel: %s", p->tok_why.c_str());
+    const float* src = block == VT_BLOCK_ATTN ? p->tok_base.attn_part : p->tok_base.ffn_part;
+    VT_CUDA(cudaDeviceSynchronize());
+    VT_CUDA(cudaMemcpy(host_dst, src, (size_t)p->n_dev * p->m->s.d_model * 4, cudaMemcpyDeviceToHost));
+    return ok();
+}
+
 extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
                                      vt_stream stream) {
     VT_TRY(check_token_args(p, kv, x_in, x_out));
@@ -1513,7 +1551,8 @@ extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const voi
     t.x_out = static_cast<__half*>(x_out);
     t.status = kv->status;
     VT_CUDA(launch_decode_token(t, p->tok_plan, (cudaStream_t)stream));
-    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
+    if (!capturing((cudaStream_t)stream))
+        for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
     return ok();
 }
 
@@ -1559,7 +1598,8 @@ extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, c
         cur = dst;
     }
     VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, 1, st));
-    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
+    if (!capturing(st))
+        for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
     return ok();
 }
 
@@ -1602,6 +1642,7 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
         }
     }
     VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, n, st));
-    for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += n;
+    if (!capturing(st))
+        for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += n;
     return ok();
 }

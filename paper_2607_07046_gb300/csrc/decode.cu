@@ -939,22 +939,27 @@ cudaError_t launch_rope_table(float2* tab, int max_seq, int dh, double theta, cu
                     dh, theta);
 }
 
-__global__ void k_embed(const __half* table, const int32_t* ids, int n, int d, int vocab,
-                        __half* out) {
+// One CTA per row: 16-byte chunks of the table row (d is a multiple of 8, out 16-byte aligned).
+// An id outside [0, vocab) gives a zero row and sets VT_DEV_BAD_TOKEN.
+__global__ void k_embed(const __half* table, const int32_t* ids, int n, int d, int vocab, __half* out,
+                        uint32_t* status) {
     pdl_wait();
     pdl_launch_dependents();
     const int row = blockIdx.x;
     if (row >= n) return;
     const int id = ids[row];
     const bool ok = id >= 0 && id < vocab;
-    for (int c = threadIdx.x; c < d; c += blockDim.x)
-        out[(int64_t)row * d + c] = ok ? table[(int64_t)id * d + c] : __float2half(0.f);
+    if (!ok && threadIdx.x == 0) set_status(status, VT_DEV_BAD_TOKEN);
+    const uint4* src = reinterpret_cast<const uint4*>(table + (int64_t)(ok ? id : 0) * d);
+    uint4* dst = reinterpret_cast<uint4*>(out + (int64_t)row * d);
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) dst[c] = ok ? src[c] : make_uint4(0u, 0u, 0u, 0u);
 }
 
-cudaError_t launch_embed(const __half* table, const int32_t* ids, int n, int d, int vocab,
-                         __half* out, cudaStream_t st) {
+cudaError_t launch_embed(const __half* table, const int32_t* ids, int n, int d, int vocab, __half* out,
+                         uint32_t* status, cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    return launch_k(k_embed, dim3(n), dim3(256), 0, st, table, ids, n, d, vocab, out);
+    if (d % 8 != 0) return cudaErrorInvalidValue;
+    return launch_k(k_embed, dim3(n), dim3(256), 0, st, table, ids, n, d, vocab, out, status);
 }
 
 // dst[c][r] = src[r][c] for r < rows, c < cols (32 x 32 tiles through shared memory)

@@ -124,7 +124,7 @@ cudaError_t launch_fill_zero_f32(float* p, int64_t n, cudaStream_t st);
 cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, cudaStream_t st);
 cudaError_t launch_rope_table(float2* tab, int max_seq, int dh, double theta, cudaStream_t st);
 cudaError_t launch_embed(const __half* table, const int32_t* ids, int n, int d, int vocab,
-                         __half* out, cudaStream_t st);
+                         __half* out, uint32_t* status, cudaStream_t st);
 cudaError_t launch_gather_rows(const __half* const* src_rows, __half* dst, int n_rows,
                                int64_t row_len, int64_t dst_stride, cudaStream_t st);
 

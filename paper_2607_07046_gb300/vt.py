@@ -31,6 +31,7 @@ VT_ERR_PLAN_MEMORY = 11
 VT_MAX_DEVICES = 16
 VT_DEV_KV_OVERFLOW = 1
 VT_DEV_WAIT_TIMEOUT = 2
+VT_DEV_BAD_TOKEN = 4
 VT_BLOCK_ATTN = 0
 VT_BLOCK_FFN = 1
 
@@ -108,6 +109,7 @@ def lib() -> ctypes.CDLL:
             "vt_model_load_embedding": (S, [_P, _P, _P]),
             "vt_model_shapes": (S, [_P, ctypes.POINTER(vt_shapes)]),
             "vt_model_destroy": (None, [_P]),
+            "vt_model_status": (S, [_P, ctypes.POINTER(ctypes.c_uint32), _I32]),
             "vt_embed": (S, [_P, _P, _I32, _P, _P]),
             "vt_partition_create": (S, [_P, _I32, ctypes.POINTER(vt_range), ctypes.POINTER(vt_range),
                                         _P, ctypes.POINTER(_P)]),
@@ -135,6 +137,7 @@ def lib() -> ctypes.CDLL:
             "vt_decode_token_sharded": (S, [_P, _P, _P, _P, _P]),
             "vt_decode_token_fused_available": (_I32, [_P, ctypes.POINTER(ctypes.c_char_p)]),
             "vt_prefill_tokens": (S, [_P, _P, _P, _I32, _P, _P]),
+            "vt_token_partials_read": (S, [_P, _I32, _P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -323,6 +326,12 @@ def vt_model_destroy(model: int) -> None:
         lib().vt_model_destroy(model)
 
 
+def vt_model_status(model: int, clear: bool = False) -> int:
+    f = ctypes.c_uint32()
+    _check(lib().vt_model_status(model, ctypes.byref(f), int(clear)))
+    return int(f.value)
+
+
 def vt_embed(model: int, ids, out, stream=None) -> None:
     import torch
     _check(lib().vt_embed(model, _ptr(ids, torch.int32), ids.numel(), _ptr(out, torch.float16),
@@ -474,6 +483,14 @@ def vt_decode_token_fused_available(part: int):
     why = ctypes.c_char_p()
     ok = lib().vt_decode_token_fused_available(part, ctypes.byref(why))
     return bool(ok), (why.value or b"").decode()
+
+
+def vt_token_partials_read(part: int, block: int, n_devices: int, d_model: int) -> np.ndarray:
+    """The fused decode-token kernel's fp32 shard partials [n_devices, d_model] of the last layer
+    (block VT_BLOCK_ATTN or VT_BLOCK_FFN); test hook, synchronous."""
+    out = np.empty((n_devices, d_model), np.float32)
+    _check(lib().vt_token_partials_read(part, int(block), out.ctypes.data))
+    return out
 
 
 def vt_prefill_tokens(part: int, kv: int, x_in, n: int, x_out, stream=None) -> None:

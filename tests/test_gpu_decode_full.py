@@ -79,8 +79,8 @@ def test_7b_decode_token_graph_two_layer_stack(vtlib):
             with torch.cuda.graph(g, stream=s):
                 vtlib.vt_decode_token(st.part, st.kv, xin, xout, stream=s)
         torch.cuda.current_stream().wait_stream(s)
-        # the capture moved the host-side length mirror; restore it
-        vtlib.vt_kv_set_length(st.kv, -1, L0)
+        # the capture recorded device work only: the device lengths and the host mirror are still L0
+        assert vtlib.vt_kv_length(st.kv, 0) == L0
         for t in range(steps):
             x = wl.hidden(1, stream=60 + t)
             xin.copy_(dev(x.reshape(-1)))

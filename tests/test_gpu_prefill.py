@@ -280,3 +280,81 @@ def test_decode_after_prefill_equals_longer_prefill(vtlib):
         vt.vt_prefill_tokens(b.part, b.kv, dev(X), M + 1, out_b)
         assert_close(host(y), host(out_b)[M], "decode vs prefill row")
         assert_close(host(out_a), host(out_b)[:M], "shorter prefill rows")
+
+
+# ------------------------------------------------------------------ the timed path at full width
+
+def _stack_layer_reference(wl, w, X, rows, cap):
+    """The oracle's one-layer prefill of X from position 0: every KV head's K/V rows for all of X,
+    the layer output on `rows` (attention over the causal set of each row)."""
+    kc, vc = oracle.new_cache(wl, cap)
+    n = X.shape[0]
+    for hr in wl.head_ranges:
+        k0, k1 = oracle.kv_heads_of(wl, hr)
+        if k1 > k0:
+            oracle.kv_append(wl, w, (k0, k1), X, 0, kc, vc)
+    rows = np.asarray(rows)
+    ap = [oracle.attn_partial(wl, w, hr, X[rows], rows, kc, vc) for hr in wl.head_ranges]
+    h = oracle.combine(ap, X[rows])
+    fp = [oracle.ffn_partial(wl, w, cr, h) for cr in wl.ffn_ranges]
+    return oracle.combine(fp, h), kc, vc
+
+
+def _check_cache(vt, st, wl, layer, n, kc, vc, tag):
+    for d, hr in enumerate(wl.head_ranges):
+        k0, k1 = kv_range(wl, hr)
+        if k1 == k0:
+            continue
+        kg, vg = vt.vt_kv_read(st.kv, layer, d, n, k1 - k0, wl.d_head)
+        assert_close(kg, kc[k0:k1, :n], f"{tag} layer {layer} k dev {d}")
+        assert_close(vg, vc[k0:k1, :n], f"{tag} layer {layer} v dev {d}")
+
+
+FULL_WIDTH = {
+    # config: (prompt rows, sampled rows spanning 128-row tiles and the ragged tail)
+    4: (512, [0, 1, 127, 128, 255, 256, 300, 383, 384, 510, 511]),   # 7B, even 4-way (the bench's shape)
+    3: (300, [0, 63, 127, 128, 200, 256, 299]),                      # 13B, heads 20/12/8, FFN 6912/4147/2765
+    5: (260, [0, 1, 127, 128, 255, 259]),                           # 8B GQA, 2 KV heads per shard
+}
+
+
+@pytest.mark.parametrize("cid", list(FULL_WIDTH))
+def test_prefill_tokens_full_width_one_layer(vtlib, cid):
+    """vt_prefill_tokens (one grouped tensor-core GEMM launch per projection for all shards, split-K
+    chosen by the time model) on one full-width layer, against the oracle.  The prompt's residual is
+    scaled down (x ~ N(0, 0.01^2)), so the output is dominated by the shard partials and an error in
+    any of them shows; every appended K/V row is compared too."""
+    vt = vtlib
+    n, rows = FULL_WIDTH[cid]
+    wl = dataclasses.replace(synthetic.WORKLOADS[cid], n_layers=1)
+    w = wl.layer_weights(0)
+    X = (wl.hidden(n, stream=160 + cid).astype(np.float32) * 0.01).astype(np.float16)
+    ref, kc, vc = _stack_layer_reference(wl, w, X, rows, n)
+    assert np.sqrt(np.mean(X.astype(np.float64) ** 2)) < 0.05 * np.sqrt(np.mean(ref.astype(np.float64) ** 2))
+    with build(vt, wl, n) as st:
+        out = torch.empty((n, wl.d_model), dtype=torch.float16, device="cuda")
+        vt.vt_prefill_tokens(st.part, st.kv, dev(X), n, out)
+        assert_close(host(out)[rows], ref, f"{wl.name} prefill_tokens x_out")
+        _check_cache(vt, st, wl, 0, n, kc, vc, wl.name)
+        assert vt.vt_kv_length(st.kv, 0) == n
+        assert vt.vt_kv_status(st.kv) == 0 and vt.vt_partition_status(st.part) == 0
+
+
+def test_prefill_tokens_7b_two_layers_512_rows(vtlib):
+    """The benchmarked prompt shape (512 rows, 7B width, even 4-way) through two layers of the
+    stack: layer 0 in full on the oracle (its output feeds layer 1's K/V), layer 1 on sampled rows."""
+    vt = vtlib
+    n, rows = FULL_WIDTH[4]
+    wl = dataclasses.replace(synthetic.WORKLOADS[4], n_layers=2)
+    X = wl.hidden(n, stream=170)
+    w0, w1 = wl.layer_weights(0), wl.layer_weights(1)
+    kc0, vc0 = oracle.new_cache(wl, n)
+    _, x1, _, _ = oracle.tp_layer(wl, w0, X, 0, kc0, vc0)
+    ref, kc1, vc1 = _stack_layer_reference(wl, w1, x1, rows, n)
+    with build(vt, wl, n) as st:
+        out = torch.empty((n, wl.d_model), dtype=torch.float16, device="cuda")
+        vt.vt_prefill_tokens(st.part, st.kv, dev(X), n, out)
+        assert_close(host(out)[rows], ref, "7b two-layer prefill_tokens x_out")
+        _check_cache(vt, st, wl, 0, n, kc0, vc0, "7b")
+        _check_cache(vt, st, wl, 1, n, kc1, vc1, "7b")
+        assert vt.vt_kv_status(st.kv) == 0 and vt.vt_partition_status(st.part) == 0

@@ -45,7 +45,6 @@ def run_tokens(vt, wl, layers, L0, steps, entry, graph=True, stream_id=70):
                 with torch.cuda.graph(g, stream=s):
                     entry(st.part, st.kv, xin, xout, stream=s)
             torch.cuda.current_stream().wait_stream(s)
-            vt.vt_kv_set_length(st.kv, -1, L0)
         for t in range(steps):
             x = wl.hidden(1, stream=stream_id + t)
             xin.copy_(dev(x.reshape(-1)))
@@ -146,3 +145,101 @@ def test_fused_and_sharded_agree_and_repeat(vtlib):
         assert_close(a[t], b[t], f"fused vs sharded token {t}")
         d = np.abs(a[t].astype(np.float64) - c[t].astype(np.float64))
         assert d.max() <= 2e-3, f"fused run-to-run difference {d.max():.3e}"
+
+
+# ------------------------------------------------------------------ partials of the fused kernel
+
+def _one_layer_token_with_small_residual(vt, wl, layer, L0, scale=1e-2, stream_id=130):
+    """One token through one layer with the input residual scaled down (x ~ N(0, scale^2)): the
+    RMSNorm undoes the scale, so the partials keep their size while the residual they are added to
+    becomes small, and an error in a partial is no longer hidden by the fp16 rounding of the
+    residual.  Returns the GPU's x_out and fp32 partials of both blocks, and the oracle's."""
+    from tests.test_gpu_decode import build as build_stack, write_cache
+    cap = L0 + 8
+    w = wl.layer_weights(layer)
+    kc, vc = wl.kv_fill(layer, L0, cap) if L0 > 0 else oracle.new_cache(wl, cap)
+    x = (wl.hidden(1, stream=stream_id).astype(np.float32) * scale).astype(np.float16)
+    n = len(wl.head_ranges)
+    with build_stack(vt, wl, layer_ids=[layer], capacity=cap) as st:
+        write_cache(vt, st, 0, wl, kc, vc, L0, wl.head_ranges)
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        fused = vt.vt_decode_token_fused_available(st.part)
+        assert fused[0], fused[1]
+        xout = torch.empty(wl.d_model, dtype=torch.float16, device="cuda")
+        vt.vt_decode_token(st.part, st.kv, dev(x.reshape(-1)), xout)
+        got_attn = vt.vt_token_partials_read(st.part, vt.VT_BLOCK_ATTN, n, wl.d_model)
+        got_ffn = vt.vt_token_partials_read(st.part, vt.VT_BLOCK_FFN, n, wl.d_model)
+        got_out = host(xout)
+        assert vt.vt_kv_status(st.kv) == 0
+    h_ref, ap = oracle.tp_attention(wl, w, x.reshape(1, -1), L0, kc, vc)
+    xn_ref, fp = oracle.tp_ffn(wl, w, h_ref)
+    return x, got_out, got_attn, got_ffn, h_ref, xn_ref, ap, fp
+
+
+def _check_partials(wl, got_out, got_attn, got_ffn, x, h_ref, xn_ref, ap, fp, tag):
+    n = len(wl.head_ranges)
+    for d in range(n):
+        h0, h1 = wl.head_ranges[d]
+        if h1 > h0:
+            assert_close(got_attn[d], ap[d].reshape(-1), f"{tag} fused ATTN partial dev {d}")
+        c0, c1 = wl.ffn_ranges[d]
+        if c1 > c0:
+            assert_close(got_ffn[d], fp[d].reshape(-1), f"{tag} fused FFN partial dev {d}")
+    # h from the kernel's own ATTN partials (the combine it performs: residual + partials in
+    # shard order, one fp16 rounding) against the oracle's h
+    used = [got_attn[d].astype(np.float64) for d in range(n) if wl.head_ranges[d][1] > wl.head_ranges[d][0]]
+    h_gpu = oracle.combine(used, x.reshape(1, -1))
+    assert_close(h_gpu, h_ref, f"{tag} h")
+    # with the residual scaled down, x_out is dominated by the partials
+    resid = np.sqrt(np.mean(x.astype(np.float64) ** 2))
+    assert resid < 0.05 * np.sqrt(np.mean(xn_ref.astype(np.float64) ** 2))
+    assert_close(got_out, xn_ref.reshape(-1), f"{tag} x_out")
+
+
+@pytest.mark.parametrize("name", list(SHAPES))
+def test_fused_token_partials_with_small_residual(vtlib, name):
+    kw, layers, L0, steps = SHAPES[name]
+    wl = synthetic.small(name, kv_len=L0, decode_steps=steps, prompt_len=0, **kw)
+    r = _one_layer_token_with_small_residual(vtlib, wl, layers[-1], L0)
+    x, got_out, got_attn, got_ffn, h_ref, xn_ref, ap, fp = r
+    _check_partials(wl, got_out, got_attn, got_ffn, x, h_ref, xn_ref, ap, fp, name)
+
+
+@pytest.mark.parametrize("cid", [2, 3, 5])
+def test_fused_token_partials_full_size_layer(vtlib, cid):
+    """The benchmarked kernel's fp32 shard partials at full width (7B 4-way, 13B uneven 3-way,
+    8B GQA 4-way, at the workloads' KV lengths), with a small residual so x_out shows them."""
+    wl = synthetic.WORKLOADS[cid]
+    r = _one_layer_token_with_small_residual(vtlib, wl, wl.n_layers - 1, wl.kv_len, stream_id=140 + cid)
+    x, got_out, got_attn, got_ffn, h_ref, xn_ref, ap, fp = r
+    _check_partials(wl, got_out, got_attn, got_ffn, x, h_ref, xn_ref, ap, fp, wl.name)
+
+
+def test_capture_leaves_the_host_length_mirror(vtlib):
+    """Capturing vt_decode_token records device work only: with room for exactly one more token,
+    an eager token after the capture is accepted (a capture that had advanced the host mirror would
+    make it fail the capacity check), and the next one is refused before any launch."""
+    vt = vtlib
+    kw, layers, L0, steps = SHAPES["mha-dh64-uneven-empty"]
+    wl = synthetic.small("capture", kv_len=L0, decode_steps=1, prompt_len=0, **kw)
+    cap = L0 + 1
+    with build(vt, wl, layer_ids=[0], capacity=cap) as st:
+        kc, vc = wl.kv_fill(0, L0, cap)
+        write_cache(vt, st, 0, wl, kc, vc, L0, wl.head_ranges)
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        xin = dev(wl.hidden(1, stream=150).reshape(-1))
+        xout = torch.empty_like(xin)
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            with torch.cuda.graph(g, stream=s):
+                vt.vt_decode_token(st.part, st.kv, xin, xout, stream=s)
+        torch.cuda.current_stream().wait_stream(s)
+        vt.vt_decode_token(st.part, st.kv, xin, xout)
+        with pytest.raises(vt.VtError) as e:
+            vt.vt_decode_token(st.part, st.kv, xin, xout)
+        assert e.value.status == vt.VT_ERR_KV_CAPACITY
+        assert vt.vt_kv_length(st.kv, 0) == L0 + 1
+        assert vt.vt_kv_status(st.kv) == 0
+        del g
