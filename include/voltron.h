@@ -235,6 +235,16 @@ VT_API vt_status vt_model_load_layer(vt_model* model, int32_t layer, const vt_la
 VT_API vt_status vt_model_load_embedding(vt_model* model, const void* embed, vt_stream stream);
 VT_API vt_status vt_model_shapes(const vt_model* model, vt_shapes* out);
 VT_API void vt_model_destroy(vt_model* model);
+/* vt_model_set_window (Section 2.1, "LLM Architecture": sliding-window attention is one of the
+ * attention variants of the evaluated models; gemma-3 uses a window of 1024 on most layers):
+ * layer `layer` (or every layer when -1) attends, for a row at position p, only to positions
+ * [max(0, p - window + 1), p] (window = 0, the default: every position 0..p).  Applies to every
+ * decode and prefill entry point.  Windows are fixed while a partition of the model exists:
+ * set them before vt_partition_create (VT_ERR_STATE otherwise).  VT_ERR_INVALID_ARG for a
+ * negative window or a layer out of range.  Host only.
+ * vt_model_window reads one layer's window back. */
+VT_API vt_status vt_model_set_window(vt_model* model, int32_t layer, int32_t window);
+VT_API vt_status vt_model_window(const vt_model* model, int32_t layer, int32_t* window);
 /* Library plumbing.  Reads the model's device status word (VT_DEV_BAD_TOKEN from vt_embed),
  * synchronizing the device; clear != 0 resets it. */
 VT_API vt_status vt_model_status(vt_model* model, uint32_t* flags, int32_t clear);

@@ -210,16 +210,17 @@ def new_cache(wl, cap: int) -> Tuple[np.ndarray, np.ndarray]:
 
 
 def tp_attention(wl, weights, x: np.ndarray, pos0: int, kcache, vcache,
-                 head_ranges=None) -> Tuple[np.ndarray, List[np.ndarray]]:
+                 head_ranges=None, window: int = 0) -> Tuple[np.ndarray, List[np.ndarray]]:
     """One ATTN block under tensor parallelism: every shard appends its KV heads for all rows,
-    then computes its partial; returns (h = binary16(x + sum partials), partials)."""
+    then computes its partial; returns (h = binary16(x + sum partials), partials).  window > 0:
+    sliding-window attention (see attn_partial)."""
     head_ranges = wl.head_ranges if head_ranges is None else head_ranges
     x = _f16(x).reshape(-1, wl.d_model)
     rows = x.shape[0]
     for hr in head_ranges:
         kv_append(wl, weights, kv_heads_of(wl, hr), x, pos0, kcache, vcache)
     pos = np.arange(pos0, pos0 + rows)
-    parts = [attn_partial(wl, weights, hr, x, pos, kcache, vcache) for hr in head_ranges]
+    parts = [attn_partial(wl, weights, hr, x, pos, kcache, vcache, window) for hr in head_ranges]
     return combine(parts, x), parts
 
 
@@ -231,9 +232,9 @@ def tp_ffn(wl, weights, h: np.ndarray, ffn_ranges=None) -> Tuple[np.ndarray, Lis
 
 
 def tp_layer(wl, weights, x: np.ndarray, pos0: int, kcache, vcache, head_ranges=None,
-             ffn_ranges=None):
+             ffn_ranges=None, window: int = 0):
     """Whole decoder layer: returns (h, x_next, attn_partials, ffn_partials)."""
-    h, ap = tp_attention(wl, weights, x, pos0, kcache, vcache, head_ranges)
+    h, ap = tp_attention(wl, weights, x, pos0, kcache, vcache, head_ranges, window)
     xn, fp = tp_ffn(wl, weights, h, ffn_ranges)
     return h, xn, ap, fp
 

@@ -140,6 +140,8 @@ struct vt_model {
     bool embed_loaded = false;
     float2* rope = nullptr;
     uint32_t* status = nullptr;  // device status word of the embedding gather
+    std::vector<int32_t> window;  // per layer: sliding attention window (0: all cached positions)
+    int n_partitions = 0;         // live partitions (windows are fixed while any exists)
 };
 
 struct AttnShard {
@@ -174,6 +176,7 @@ struct vt_partition {
     std::vector<FfnShard> ffn;
     std::vector<DecodeScratch> dec;
     std::vector<void*> owned;  // every allocation besides the shard bases
+    bool counted = false;      // counted in the model's n_partitions
     uint32_t* status = nullptr;
     // whole-stack buffers
     float* dpart = nullptr;     // [n_dev][D] decode partials (kept zero between blocks)
@@ -181,7 +184,7 @@ struct vt_partition {
     __half* hbuf = nullptr;     // [kPrefillChunk][D]
     __half* xbuf = nullptr;     // [kPrefillChunk][D]
     // prefill scratch
-    __half* p_xhat = nullptr;   // [kPrefillChunk][D]
+    __half* p_xhat = nullptr;   // [kPrefillChunk][2 D]: ATTN input as fp16 hi / lo halves (FFN: [.][D])
     __half* p_q = nullptr;      // [n_dev] slots of [kPrefillChunk][max_hq][dh], q_slot halves apart
     __half* p_attn = nullptr;   // [n_dev] slots of [kPrefillChunk][max_hq dh]
     __half* p_u = nullptr;      // [n_dev] slots of [kPrefillChunk][max_ld], u_slot halves apart
@@ -597,6 +600,7 @@ extern "C" vt_status vt_model_create(const vt_shapes* shapes, const vt_layer_wei
     for (size_t b : sizes) total += align256(b);
     m->layer.resize(s.n_layers);
     m->loaded.assign(s.n_layers, 0);
+    m->window.assign(s.n_layers, 0);
     for (int l = 0; l < s.n_layers; ++l) {
         uint8_t* base = static_cast<uint8_t*>(m->alloc.get(total));
         if (!base) {
@@ -675,6 +679,23 @@ extern "C" vt_status vt_model_shapes(const vt_model* m, vt_shapes* out) {
     return ok();
 }
 
+extern "C" vt_status vt_model_set_window(vt_model* m, int32_t layer, int32_t window) {
+    if (!m) return fail(VT_ERR_INVALID_ARG, "model is NULL");
+    if (layer < -1 || layer >= m->s.n_layers) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
+    if (window < 0) return fail(VT_ERR_INVALID_ARG, "window %d is negative", window);
+    if (m->n_partitions > 0)
+        return fail(VT_ERR_STATE, "attention windows are fixed while a partition of the model exists");
+    for (int l = layer < 0 ? 0 : layer; l < (layer < 0 ? m->s.n_layers : layer + 1); ++l) m->window[l] = window;
+    return ok();
+}
+
+extern "C" vt_status vt_model_window(const vt_model* m, int32_t layer, int32_t* window) {
+    if (!m || !window) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    if (layer < 0 || layer >= m->s.n_layers) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
+    *window = m->window[layer];
+    return ok();
+}
+
 extern "C" vt_status vt_model_status(vt_model* m, uint32_t* flags, int32_t clear) {
     if (!m) return fail(VT_ERR_INVALID_ARG, "model is NULL");
     return read_status(m->status, flags, clear, nullptr);
@@ -700,6 +721,7 @@ extern "C" void vt_partition_destroy(vt_partition* p) {
     for (auto& s : p->attn) A.put(s.base);
     for (auto& s : p->ffn) A.put(s.base);
     for (void* q : p->owned) A.put(q);
+    if (p->counted) --p->m->n_partitions;
     delete p;
 }
 
@@ -741,6 +763,8 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     vt_partition* p = new vt_partition();
     p->m = m;
     p->n_dev = n;
+    p->counted = true;
+    ++m->n_partitions;
     p->heads.assign(heads, heads + n);
     p->cols.assign(cols, cols + n);
     p->attn.resize((size_t)s.n_layers * n);
@@ -867,7 +891,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         p->q_slot = align256(R * std::max(p->max_hq, 1) * dh * 2) / 2;
         p->u_slot = align256(R * std::max(p->max_ld, 8) * 2) / 2;
         const size_t bytes = align256(4) + align256((size_t)n * D * 4) + align256((size_t)n * R * D * 4) + 2 * align256(R * D * 2) +
-                             align256(R * D * 2) + 2 * (size_t)n * p->q_slot * 2 + (size_t)n * p->u_slot * 2;
+                             align256(R * 2 * D * 2) + 2 * (size_t)n * p->q_slot * 2 + (size_t)n * p->u_slot * 2;
         void* q;
         if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
         Bump b{static_cast<uint8_t*>(q)};
@@ -876,7 +900,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         p->partials = b.take<float>((size_t)n * R * D);
         p->hbuf = b.take<__half>(R * D);
         p->xbuf = b.take<__half>(R * D);
-        p->p_xhat = b.take<__half>(R * D);
+        p->p_xhat = b.take<__half>(R * 2 * D);
         p->p_q = b.take<__half>((size_t)n * p->q_slot);
         p->p_attn = b.take<__half>((size_t)n * p->q_slot);
         p->p_u = b.take<__half>((size_t)n * p->u_slot);
@@ -1047,6 +1071,7 @@ extern "C" vt_status vt_kv_create(const vt_partition* p, int32_t cap, vt_stream 
         for (int l = 0; l < L; ++l) {
             tly[l].attn_norm = p->m->layer[l].attn_norm;
             tly[l].ffn_norm = p->m->layer[l].ffn_norm;
+            tly[l].window = p->m->window[l];
             for (int d = 0; d < n; ++d) {
                 const AttnShard& a = p->a(l, d);
                 const FfnShard& f = p->f(l, d);
@@ -1212,6 +1237,7 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
     t.dh = dh;
     t.stages = attn_stages(kv->cap, attn_cluster_size(hk));
     t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    t.window = p->m->window[l];
     t.out = ds.attn;
     t.status = kv->status;
     VT_CUDA(launch_attn_decode(t, st));
@@ -1335,6 +1361,7 @@ extern "C" vt_status vt_decode_step_static(const vt_partition* p, vt_shard sh, c
     t.group = s.n_heads / s.n_kv_heads;
     t.dh = dh;
     t.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    t.window = p->m->window[l];
     t.part_ml = reinterpret_cast<float*>(b + lay.part_ml);
     t.part_o = reinterpret_cast<float*>(b + lay.part_o);
     t.counters = reinterpret_cast<uint32_t*>(b + lay.counters);
@@ -1396,6 +1423,7 @@ static void attn_args(const vt_partition* p, vt_shard sh, const __half* x, int n
     t->cap = kv->cap;
     t->len = kv->len + sh.layer;
     t->row_offset = row_offset;
+    t->window = p->m->window[sh.layer];
     t->rope = p->m->rope;
     t->xhat = p->p_xhat;
     t->xhat_ready = xhat_ready;
@@ -1625,19 +1653,19 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
         const __half* cur = static_cast<const __half*>(x_in) + (size_t)r0 * D;
         // Every shard of a block normalises the same input with the same gain: the norm runs once
         // per block, fused into the combine that produced the block's input.
-        VT_CUDA(launch_rmsnorm_rows(cur, p->m->layer[0].attn_norm, s.rms_eps, rows, D, p->p_xhat, st));
+        VT_CUDA(launch_rmsnorm_rows(cur, p->m->layer[0].attn_norm, s.rms_eps, rows, D, p->p_xhat, 1, st));
         for (int l = 0; l < s.n_layers; ++l) {
             VT_TRY(prefill_block(p, l, VT_BLOCK_ATTN, cur, rows, kv, r0, st));
             c.residual = cur;
             c.out = p->hbuf;
-            VT_CUDA(launch_combine_norm(c, rows, D, p->m->layer[l].ffn_norm, s.rms_eps, p->p_xhat, st));
+            VT_CUDA(launch_combine_norm(c, rows, D, p->m->layer[l].ffn_norm, s.rms_eps, p->p_xhat, 0, st));
             VT_TRY(prefill_block(p, l, VT_BLOCK_FFN, p->hbuf, rows, kv, r0, st));
             const bool last = l == s.n_layers - 1;
             __half* dst = last ? static_cast<__half*>(x_out) + (size_t)r0 * D : p->xbuf;
             c.residual = p->hbuf;
             c.out = dst;
             VT_CUDA(launch_combine_norm(c, rows, D, last ? nullptr : p->m->layer[l + 1].attn_norm, s.rms_eps,
-                                        p->p_xhat, st));
+                                        p->p_xhat, 1, st));
             cur = dst;
         }
     }

@@ -577,8 +577,11 @@ __global__ void __launch_bounds__(kAttnThreads) k_attn_decode(const __grid_const
     const bool ok = len >= 0 && len < a.cap;
     const int n_pos = ok ? len + 1 : min(max(len, 0), a.cap);
     const int pnew = ok ? len : -1;
-    const int chunk = (n_pos + csize - 1) / csize;
-    const int t0 = min(rank * chunk, n_pos), t1 = min(n_pos, t0 + chunk);
+    // sliding window: only the last `window` positions (ending at the new token) are attended
+    const int t_lo = (a.window > 0 && n_pos > a.window) ? n_pos - a.window : 0;
+    const int n_att = n_pos - t_lo;
+    const int chunk = (n_att + csize - 1) / csize;
+    const int t0 = t_lo + min(rank * chunk, n_att), t1 = min(n_pos, t0 + chunk);
     const int old_end = pnew >= 0 ? min(t1, pnew) : t1;
     const int n_old = max(old_end - t0, 0);
     const int ntiles = (n_old + kAttnTilePos - 1) / kAttnTilePos;

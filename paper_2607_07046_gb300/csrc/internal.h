@@ -77,6 +77,7 @@ struct AttnDecodeArgs {
     int dh;
     int stages;            // K/V tiles in flight per CTA (attn_stages)
     float scale_log2;      // log2(e) / sqrt(dh)
+    int window;            // > 0: attend to the last `window` positions only (sliding window)
     float* out;            // [h_s][dh] attention output of the shard's query heads
     uint32_t* status;
 };
@@ -149,9 +150,10 @@ struct PrefillAttnArgs {
     int cap;
     const int32_t* len;     // device length: rows sit at positions len + row_offset + i
     int row_offset;         // rows already processed by earlier chunks of the same call
+    int window;             // > 0: row at position p attends to [p - window + 1, p] only
     const float2* rope;     // [max_seq][dh/2]
     // scratch
-    __half* xhat;           // [n][d]
+    __half* xhat;           // [n][2d]: fp16 RMSNorm(x) * gain, then the fp16 rounding of its remainder
     int xhat_ready;         // 1: xhat already holds RMSNorm(x) with this gain (skip the norm)
     __half* q;              // [n][hq][dh]
     __half* attn;           // [n][hq * dh]
@@ -183,11 +185,12 @@ vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::str
 // GEMM of the block for every shard
 vt_status prefill_attn_group(const PrefillAttnArgs* a, int n, cudaStream_t st, std::string* err);
 vt_status prefill_ffn_group(const PrefillFfnArgs* a, int n, cudaStream_t st, std::string* err);
-// rows x d: out = fp16(residual + sum of partials); with gain, also xhat = RMSNorm(out) * gain
+// rows x d: out = fp16(residual + sum of partials); with gain, also xhat = RMSNorm(out) * gain.
+// split != 0: xhat rows are 2d long, the fp16 value then the fp16 rounding of the remainder.
 cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __half* gain, float eps, __half* xhat,
-                                cudaStream_t st);
+                                int split, cudaStream_t st);
 cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
-                                cudaStream_t st);
+                                int split, cudaStream_t st);
 
 // ------------------------------------------------------------------ static-scratch decode attention
 // (static_scratch.cu) split-K decode attention whose scratch is one file-scope __device__ array.
@@ -209,6 +212,7 @@ struct StaticAttnArgs {
     const int32_t* len;
     int cap, hk, group, dh;
     float scale_log2;
+    int window;            // > 0: sliding window over the last `window` positions
     float* part_ml;        // [hk][kStaticSplits][group][2] (max, sum) of each slice
     float* part_o;         // [hk][kStaticSplits][group][dh] weighted V of each slice
     uint32_t* counters;    // [hk] slices finished; zero between calls
@@ -253,6 +257,7 @@ struct TokShardPtrs {  // one (layer, device) shard; null weights for an empty b
 struct TokLayerPtrs {
     const __half* attn_norm;  // [D]
     const __half* ffn_norm;   // [D]
+    int window;               // > 0: sliding attention window of the layer
 };
 
 struct TokArgs {

@@ -117,12 +117,29 @@ __host__ __device__ constexpr uint32_t idesc_f16(int m, int n) {
 
 // ================================================================== RMSNorm rows
 
+// One CTA per row: y = fp16(RMSNorm(x) * gain).  split != 0: the row of y is 2d long and holds
+// the fp16 value in [0, d) and the fp16 rounding of the remainder in [d, 2d), so that a GEMM over
+// the 2d columns (the weights read twice) multiplies the normalised input at fp32 precision.
+__device__ __forceinline__ void store_hl8(__half* row, int d, int c, const float (&v)[8], bool split) {
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const __half2 h = __floats2half2_rn(v[2 * e], v[2 * e + 1]);
+        hi[e] = *reinterpret_cast<const uint32_t*>(&h);
+        const float2 hf = __half22float2(h);
+        const __half2 l = __floats2half2_rn(v[2 * e] - hf.x, v[2 * e + 1] - hf.y);
+        lo[e] = *reinterpret_cast<const uint32_t*>(&l);
+    }
+    *reinterpret_cast<uint4*>(row + (size_t)c * 8) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    if (split) *reinterpret_cast<uint4*>(row + d + (size_t)c * 8) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+}
+
 __global__ void __launch_bounds__(256) k_rmsnorm_rows(const __half* __restrict__ x, const __half* __restrict__ gain,
-                                                      float eps, int d, __half* __restrict__ y) {
+                                                      float eps, int d, __half* __restrict__ y, int split) {
     __shared__ float red[8];
     pdl_wait();
     const __half* xr = x + (size_t)blockIdx.x * d;
-    __half* yr = y + (size_t)blockIdx.x * d;
+    __half* yr = y + (size_t)blockIdx.x * d * (split ? 2 : 1);
     float ss = 0.f;
     for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
         const uint4 v = *reinterpret_cast<const uint4*>(xr + c * 8);
@@ -144,14 +161,14 @@ __global__ void __launch_bounds__(256) k_rmsnorm_rows(const __half* __restrict__
         const uint4 v = *reinterpret_cast<const uint4*>(xr + c * 8);
         const uint4 g = *reinterpret_cast<const uint4*>(gain + c * 8);
         const uint32_t w[4] = {v.x, v.y, v.z, v.w}, gw[4] = {g.x, g.y, g.z, g.w};
-        uint32_t o[4];
+        float o[8];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float2 f = h2_to_f2(w[e]), gg = h2_to_f2(gw[e]);
-            const __half2 h = __floats2half2_rn(f.x * r * gg.x, f.y * r * gg.y);
-            o[e] = *reinterpret_cast<const uint32_t*>(&h);
+            o[2 * e] = f.x * r * gg.x;
+            o[2 * e + 1] = f.y * r * gg.y;
         }
-        *reinterpret_cast<uint4*>(yr + c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+        store_hl8(yr, d, c, o, split != 0);
     }
 }
 
@@ -162,7 +179,7 @@ __global__ void __launch_bounds__(256) k_rmsnorm_rows(const __half* __restrict__
 // every shard of the next block would normalise for itself.
 __global__ void __launch_bounds__(256) k_combine_norm(const __grid_constant__ CombineArgs a, int d,
                                                       const __half* __restrict__ gain, float eps,
-                                                      __half* __restrict__ xhat) {
+                                                      __half* __restrict__ xhat, int split) {
     __shared__ float red[8];
     pdl_wait();
     const size_t row = blockIdx.x;
@@ -213,27 +230,24 @@ __global__ void __launch_bounds__(256) k_combine_norm(const __grid_constant__ Co
         const uint4 hv = *reinterpret_cast<const uint4*>(a.out + row * d + (size_t)c * 8);
         const uint4 g = *reinterpret_cast<const uint4*>(gain + c * 8);
         const uint32_t w[4] = {hv.x, hv.y, hv.z, hv.w}, gw[4] = {g.x, g.y, g.z, g.w};
-        uint32_t o[4];
+        float o[8];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const float2 f = h2_to_f2(w[j]), gg = h2_to_f2(gw[j]);
-            const __half2 h = __floats2half2_rn(f.x * r * gg.x, f.y * r * gg.y);
-            o[j] = *reinterpret_cast<const uint32_t*>(&h);
+            o[2 * j] = f.x * r * gg.x;
+            o[2 * j + 1] = f.y * r * gg.y;
         }
-        *reinterpret_cast<uint4*>(xhat + row * d + (size_t)c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+        store_hl8(xhat + row * d * (split ? 2 : 1), d, c, o, split != 0);
     }
 }
 
 cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __half* gain, float eps, __half* xhat,
-                                cudaStream_t st) {
+                                int split, cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
     if (d % 8 != 0 || d > 16384) return cudaErrorInvalidValue;
-    k_combine_norm<<<rows, 256, 0, st>>>(a, d, gain, eps, xhat);
+    k_combine_norm<<<rows, 256, 0, st>>>(a, d, gain, eps, xhat, split);
     return cudaGetLastError();
 }
-
-cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
-                                cudaStream_t st);
 
 // ================================================================== tensor-core GEMM
 
@@ -246,6 +260,7 @@ enum GemmEpi : int { kGemmF32 = 0, kGemmQkv = 1, kGemmSwiglu = 2 };
 
 struct GemmArgs {
     int m, n, k_tiles;
+    int kb_wrap;  // > 0: A's k-tile kt multiplies B's k-tile kt mod kb_wrap (B read twice: hi / lo A halves)
     const __half* b;  // B [n][ldb] (prefetched into L2 by the epilogue warps while they wait)
     int64_t ldb;
     // kGemmF32: c[row][col], row stride ldc
@@ -281,6 +296,11 @@ struct GemmGroup {
 // permutation keeps those 8 threads on distinct banks both for the writer (8 consecutive rows, one
 // chunk) and for the reader (one row, 8 consecutive chunks).
 __device__ __forceinline__ int recv_slot(int chunk, int e, int lr) { return chunk * 8 + (e ^ ((chunk + lr) & 7)); }
+
+// B's k-tile for A's k-tile kt.
+__device__ __forceinline__ int bk_tile(const GemmArgs& a, int kt) {
+    return a.kb_wrap > 0 && kt >= a.kb_wrap ? kt - a.kb_wrap : kt;
+}
 
 // Epilogue of 4 consecutive columns [col, col + 4) of one output row (col a multiple of 4).
 template <int EPI>
@@ -381,14 +401,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
     if (warp == 0 && lane == 0) {
         for (int i = 0; i < pre; ++i) {
             mbar_arrive_expect_tx(&full[i], kStageBytes);
-            tc::tma_load_2d(smem + i * kStageBytes + kABytes, &tb, (kt0 + i) * kBK, n0, &full[i]);
+            tc::tma_load_2d(smem + i * kStageBytes + kABytes, &tb, bk_tile(a, kt0 + i) * kBK, n0, &full[i]);
         }
     } else if (warp >= 2) {
         const int t = threadIdx.x - 64;
-        for (int i = kt0 + pre; i < kt1; ++i)
+        for (int i = kt0 + pre; i < kt1; ++i) {
+            if (a.kb_wrap > 0 && i >= a.kb_wrap && kt0 < a.kb_wrap) break;  // the second pass reads the same B again
             for (int r = t; r < kBN; r += kGemmThreads - 64)
                 if (n0 + r < a.n)
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.b + (size_t)(n0 + r) * a.ldb + (size_t)i * kBK));
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.b + (size_t)(n0 + r) * a.ldb + (size_t)bk_tile(a, i) * kBK));
+        }
     }
     pdl_wait();  // A was written by the preceding kernel
 
@@ -410,7 +432,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
                 } else {
                     mbar_arrive_expect_tx(&full[s], kStageBytes);
                     tc::tma_load_2d(st, &ta, (kt0 + i) * kBK, m0, &full[s]);
-                    tc::tma_load_2d(st + kABytes, &tb, (kt0 + i) * kBK, n0, &full[s]);
+                    tc::tma_load_2d(st + kABytes, &tb, bk_tile(a, kt0 + i) * kBK, n0, &full[s]);
                 }
                 issued = i + 1;
             }
@@ -535,6 +557,7 @@ struct PrefillAttnKArgs {
     const __half* vcache;
     const int32_t* len;
     int row_offset, n, hq, group, cap;
+    int window;  // > 0: row at position p sees positions [p - window + 1, p]
     float scale_log2;
     __half* out;  // [n][hq * dh]
 };
@@ -588,8 +611,11 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
     pdl_wait();
     const int P0 = *a.len + a.row_offset;
     const int rlast = min(r0 + kAttnRows - 1, a.n - 1);
-    const int kend = min(P0 + rlast + 1, a.cap);  // positions [0, kend) are needed
+    const int kend = min(P0 + rlast + 1, a.cap);  // positions [kbeg, kend) are needed
     const int nkb = (kend + kAttnKeys - 1) / kAttnKeys;
+    // with a sliding window the first row of the CTA sees nothing before P0 + r0 - window + 1
+    const int kbeg = a.window > 0 ? max(0, P0 + r0 - a.window + 1) : 0;
+    const int kb0 = kbeg / kAttnKeys;
     const __half* kbase = a.kcache + (size_t)j * a.cap * DH;
     const __half* vbase = a.vcache + (size_t)j * a.cap * DH;
 
@@ -625,9 +651,13 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
     float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
     const int qpos[2] = {P0 + qr0 + g, P0 + qr0 + g + 8};
     const int warp_last = P0 + qr0 + 15;
+    // first position any row of this warp sees (sliding window), and the window's lower bound
+    // of each of the lane's two rows
+    const int warp_first = a.window > 0 ? P0 + qr0 - a.window + 1 : 0;
+    const int qlo[2] = {a.window > 0 ? qpos[0] - a.window + 1 : 0, a.window > 0 ? qpos[1] - a.window + 1 : 0};
 
-    load_tile(0, 0);
-    for (int kb = 0; kb < nkb; ++kb) {
+    if (kb0 < nkb) load_tile(kb0, kb0 & 1);
+    for (int kb = kb0; kb < nkb; ++kb) {
         const int buf = kb & 1;
         if (kb + 1 < nkb) {
             load_tile(kb + 1, buf ^ 1);
@@ -636,7 +666,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
             cp_async_wait<0>();
         }
         __syncthreads();
-        if (kb * kAttnKeys <= warp_last) {
+        if (kb * kAttnKeys <= warp_last && (kb + 1) * kAttnKeys - 1 >= warp_first) {
             const __half* kt = Ks + buf * kAttnKeys * LDS;
             float s[8][4];
 #pragma unroll
@@ -656,7 +686,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const int pos = kb * kAttnKeys + nt * 8 + 2 * t + (e & 1);
-                    const float v = pos <= qpos[e >> 1] ? s[nt][e] * a.scale_log2 : -INFINITY;
+                    const float v = (pos <= qpos[e >> 1] && pos >= qlo[e >> 1]) ? s[nt][e] * a.scale_log2 : -INFINITY;
                     s[nt][e] = v;
                     mx[e >> 1] = fmaxf(mx[e >> 1], v);
                 }
@@ -829,6 +859,7 @@ struct GemmSpec {
     int64_t ldb;
     int n, k;
     GemmArgs base;
+    int kb = 0;  // > 0: B has kb columns and A's k = 2 kb columns hold the hi and lo halves of the input
 };
 
 // Launches the GEMMs of `specs` (all with m rows) kGemmGroups at a time, one CTA (or split-K
@@ -843,7 +874,12 @@ static vt_status run_gemm_group(const GemmSpec* specs, int n_specs, int m, cudaS
         int tiles_n = 0, max_k_tiles = 1, min_k_tiles = 1 << 30;
         for (int g = 0; g < ng; ++g) {
             const GemmSpec& sp = specs[g0 + g];
-            if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) || !make_map(&G.tb[g], sp.B, sp.k, sp.n, sp.ldb, kBN, err))
+            if (sp.kb > 0 && (sp.kb % kBK != 0 || sp.k != 2 * sp.kb)) {
+                *err = "a split GEMM needs k = 2 kb with kb a multiple of 64";
+                return VT_ERR_INVALID_ARG;
+            }
+            if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) ||
+                !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, kBN, err))
                 return VT_ERR_INVALID_ARG;
             GemmArgs& a = G.a[g];
             a = sp.base;
@@ -852,6 +888,7 @@ static vt_status run_gemm_group(const GemmSpec* specs, int n_specs, int m, cudaS
             a.b = static_cast<const __half*>(sp.B);
             a.ldb = sp.ldb;
             a.k_tiles = (sp.k + kBK - 1) / kBK;
+            a.kb_wrap = sp.kb > 0 ? sp.kb / kBK : 0;
             max_k_tiles = std::max(max_k_tiles, a.k_tiles);
             min_k_tiles = std::min(min_k_tiles, a.k_tiles);
             tiles_n += (sp.n + kBN - 1) / kBN;
@@ -888,15 +925,16 @@ static vt_status run_gemm(const void* A, int64_t lda, const void* B, int64_t ldb
 }
 
 cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
-                                cudaStream_t st) {
+                                int split, cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
-    k_rmsnorm_rows<<<rows, 256, 0, st>>>(x, gain, eps, d, y);
+    if (d % 8 != 0) return cudaErrorInvalidValue;
+    k_rmsnorm_rows<<<rows, 256, 0, st>>>(x, gain, eps, d, y, split);
     return cudaGetLastError();
 }
 
-static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int n, int d, __half* y, cudaStream_t st,
-                             std::string* err) {
-    const cudaError_t e = launch_rmsnorm_rows(x, gain, eps, n, d, y, st);
+static vt_status run_rmsnorm(const __half* x, const __half* gain, float eps, int n, int d, __half* y, int split,
+                             cudaStream_t st, std::string* err) {
+    const cudaError_t e = launch_rmsnorm_rows(x, gain, eps, n, d, y, split, st);
     if (e != cudaSuccess) {
         *err = std::string("RMSNorm launch failed: ") + cudaGetErrorString(e);
         return VT_ERR_CUDA;
@@ -917,7 +955,8 @@ static GemmSpec qkv_spec(const PrefillAttnArgs& a) {
     g.row_offset = a.row_offset;
     g.rope = a.rope;
     g.status = a.status;
-    return GemmSpec{a.xhat, a.d, a.wqkv, a.d, (a.hq + 2 * a.hk) * a.dh, a.d, g};
+    // A = [hi | lo] halves of the normalised input (2d columns), B = Wqkv read once per half
+    return GemmSpec{a.xhat, 2 * a.d, a.wqkv, a.d, (a.hq + 2 * a.hk) * a.dh, 2 * a.d, g, a.d};
 }
 
 static GemmSpec o_spec(const PrefillAttnArgs& a) {
@@ -940,6 +979,7 @@ static vt_status prefill_attention(const PrefillAttnArgs& a, cudaStream_t st, st
     t.hq = a.hq;
     t.group = a.hq / a.hk;
     t.cap = a.cap;
+    t.window = a.window;
     t.scale_log2 = a.scale_log2;
     t.out = a.attn;
     const dim3 grid((a.n + kAttnRows - 1) / kAttnRows, a.hq);
@@ -962,7 +1002,7 @@ vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::str
 vt_status prefill_attn_group(const PrefillAttnArgs* a, int n, cudaStream_t st, std::string* err) {
     if (n < 1) return VT_OK;
     vt_status r;
-    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, st, err)) != VT_OK)
+    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, 1, st, err)) != VT_OK)
         return r;
     GemmSpec specs[VT_MAX_DEVICES];
     for (int i = 0; i < n; ++i) specs[i] = qkv_spec(a[i]);
@@ -981,7 +1021,7 @@ vt_status prefill_ffn_shard(const PrefillFfnArgs& a, cudaStream_t st, std::strin
 vt_status prefill_ffn_group(const PrefillFfnArgs* a, int n, cudaStream_t st, std::string* err) {
     if (n < 1) return VT_OK;
     vt_status r;
-    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, st, err)) != VT_OK)
+    if (!a[0].xhat_ready && (r = run_rmsnorm(a[0].x, a[0].gain, a[0].eps, a[0].n, a[0].d, a[0].xhat, 0, st, err)) != VT_OK)
         return r;
     GemmSpec specs[VT_MAX_DEVICES];
     for (int i = 0; i < n; ++i) {

@@ -85,8 +85,10 @@ __global__ void __launch_bounds__(kSplitWarps * 32) k_attn_decode_split(const __
     const int len = *a.len;
     const bool ok = len >= 0 && len < a.cap;
     const int n_pos = ok ? len + 1 : min(max(len, 0), a.cap);
-    const int chunk = (n_pos + nsplit - 1) / nsplit;
-    const int t0 = min(split * chunk, n_pos), t1 = min(n_pos, t0 + chunk);
+    const int t_lo = (a.window > 0 && n_pos > a.window) ? n_pos - a.window : 0;  // sliding window
+    const int n_att = n_pos - t_lo;
+    const int chunk = (n_att + nsplit - 1) / nsplit;
+    const int t0 = t_lo + min(split * chunk, n_att), t1 = min(n_pos, t0 + chunk);
     const __half* kbase = a.kcache + (int64_t)j * a.cap * DH;
     const __half* vbase = a.vcache + (int64_t)j * a.cap * DH;
 

@@ -170,6 +170,8 @@ __device__ __forceinline__ void kv_geom(int len, int cap, int& n_pos, int& pnew,
     n_pos = ok ? len + 1 : min(max(len, 0), cap);
     pnew = ok ? len : -1;
 }
+// First attended position of a layer with sliding window `win` (0: every cached position).
+__device__ __forceinline__ int window_start(int n_pos, int win) { return (win > 0 && n_pos > win) ? n_pos - win : 0; }
 
 // ------------------------------------------------------------------ ring of stages
 
@@ -802,7 +804,10 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                         issue(w + (int64_t)r * D, (uint32_t)(min(rps_d, r1 - r) * D * 2), nullptr, 0);
                 });
                 const int np_stage = kTokStageBytes / (4 * dh);
-                for_kv_pieces(a, n_pos, c, NC, [&](int j, int t0, int t1, int) {
+                const int t_lo = window_start(n_pos, a.layer[l].window);
+                for_kv_pieces(a, n_pos - t_lo, c, NC, [&](int j, int t0, int t1, int) {
+                    t0 += t_lo;
+                    t1 += t_lo;
                     const int s = shard_of_kv(a, j), jl = j - a.kv0[s];
                     const __half* kb = sp[s].kc + (int64_t)jl * a.cap * dh;
                     const __half* vb = sp[s].vc + (int64_t)jl * a.cap * dh;
@@ -951,22 +956,24 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
         if (c == 0 && live)  // nobody reads the previous layer's FFN partials any more
             for (int i = tid; i < a.n_dev * D; i += kTokConsumers) __stcg(a.ffn_part + i, 0.f);
         ring.live = live;
-        for_kv_pieces(a, n_pos, c, NC, [&](int j, int t0, int t1, int seg) {
-            ring = attn_slice<dh / 32, G>(a, sp, ring, j, t0, t1, seg, pnew, uni, tid, warp, lane);
+        // sliding window: the layer attends to positions [t_lo, n_pos); slices are cut from those
+        const int t_lo = window_start(n_pos, a.layer[l].window), n_att = n_pos - t_lo;
+        for_kv_pieces(a, n_att, c, NC, [&](int j, int t0, int t1, int seg) {
+            ring = attn_slice<dh / 32, G>(a, sp, ring, j, t_lo + t0, t_lo + t1, seg, pnew, uni, tid, warp, lane);
         });
         live = ring.live;
         // Slice table of every KV head for the O phase: the state offset of each CTA slice of the
         // head (-1: none), mstride entries per head.  Every CTA builds the same table.
-        const int T = a.n_kv * n_pos;
+        const int T = a.n_kv * n_att;
         const int mstride = NC / a.n_kv + 3;
         int* mtab = reinterpret_cast<int*>(slots + a.slot_floats / 2);
         for (int idx = tid; idx < a.n_kv * mstride; idx += kTokConsumers) {
             const int j = idx / mstride, k = idx - j * mstride;
             int cf = 0, cl = -1, base = -1;
-            if (T > 0) head_ctas(T, j, n_pos, NC, cf, cl);
+            if (T > 0) head_ctas(T, j, n_att, NC, cf, cl);
             if (cf + k <= cl) {
                 const Span sx = cta_span(T, cf + k, NC);
-                if (sx.a < sx.b) base = (((cf + k) * kTokMaxSeg + (j - sx.a / n_pos)) * G) * (dh + 4);
+                if (sx.a < sx.b) base = (((cf + k) * kTokMaxSeg + (j - sx.a / n_att)) * G) * (dh + 4);
             }
             mtab[idx] = base;
         }

@@ -14,7 +14,8 @@ class Stack:
 
     def __init__(self, shapes: vt.vt_shapes, layer_fn: Callable[[int], Dict[str, np.ndarray]],
                  head_ranges: Sequence[Tuple[int, int]], ffn_ranges: Sequence[Tuple[int, int]],
-                 capacity: int, embed: Optional[np.ndarray] = None, stream=None):
+                 capacity: int, embed: Optional[np.ndarray] = None, stream=None, windows=None):
+        """windows: None, one sliding attention window for every layer, or one per layer (0: none)."""
         self.shapes = shapes
         self.model = self.part = self.kv = 0
         self.model = vt.vt_model_create(shapes, None, None, stream)
@@ -22,6 +23,10 @@ class Stack:
             vt.vt_model_load_layer(self.model, l, layer_fn(l), stream)
         if embed is not None:
             vt.vt_model_load_embedding(self.model, embed, stream)
+        if windows is not None:
+            ws = [windows] * shapes.n_layers if isinstance(windows, int) else list(windows)
+            for l, w in enumerate(ws):
+                vt.vt_model_set_window(self.model, l, w)
         self.part = vt.vt_partition_create(self.model, head_ranges, ffn_ranges, stream)
         self.kv = vt.vt_kv_create(self.part, capacity, stream) if capacity > 0 else 0
         self.head_ranges = list(head_ranges)

@@ -110,6 +110,8 @@ def lib() -> ctypes.CDLL:
             "vt_model_shapes": (S, [_P, ctypes.POINTER(vt_shapes)]),
             "vt_model_destroy": (None, [_P]),
             "vt_model_status": (S, [_P, ctypes.POINTER(ctypes.c_uint32), _I32]),
+            "vt_model_set_window": (S, [_P, _I32, _I32]),
+            "vt_model_window": (S, [_P, _I32, ctypes.POINTER(_I32)]),
             "vt_embed": (S, [_P, _P, _I32, _P, _P]),
             "vt_partition_create": (S, [_P, _I32, ctypes.POINTER(vt_range), ctypes.POINTER(vt_range),
                                         _P, ctypes.POINTER(_P)]),
@@ -324,6 +326,17 @@ def vt_model_load_embedding(model: int, embed: np.ndarray, stream=None) -> None:
 def vt_model_destroy(model: int) -> None:
     if model:
         lib().vt_model_destroy(model)
+
+
+def vt_model_set_window(model: int, layer: int, window: int) -> None:
+    """Sliding attention window of `layer` (-1: every layer); 0 attends to every position."""
+    _check(lib().vt_model_set_window(model, int(layer), int(window)))
+
+
+def vt_model_window(model: int, layer: int) -> int:
+    w = _I32()
+    _check(lib().vt_model_window(model, int(layer), ctypes.byref(w)))
+    return int(w.value)
 
 
 def vt_model_status(model: int, clear: bool = False) -> int:

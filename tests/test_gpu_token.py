@@ -149,7 +149,7 @@ def test_fused_and_sharded_agree_and_repeat(vtlib):
 
 # ------------------------------------------------------------------ partials of the fused kernel
 
-def _one_layer_token_with_small_residual(vt, wl, layer, L0, scale=1e-2, stream_id=130):
+def _one_layer_token_with_small_residual(vt, wl, layer, L0, scale=1e-3, stream_id=130):
     """One token through one layer with the input residual scaled down (x ~ N(0, scale^2)): the
     RMSNorm undoes the scale, so the partials keep their size while the residual they are added to
     becomes small, and an error in a partial is no longer hidden by the fp16 rounding of the
