@@ -310,7 +310,10 @@ VT_API int32_t vt_kv_capacity(const vt_kv* kv);
 /* Cache bookkeeping (Section 2.1: each decode step appends one position, a prefill n).  Adds n
  * to the length of `layer` (or of every layer when layer == -1), on the device (in stream
  * order) and in the host mirror.  Decode and prefill append at the current length without
- * advancing it: advance once per layer after all of that layer's attention shards ran. */
+ * advancing it: advance once per layer after all of that layer's attention shards ran.
+ * VT_ERR_KV_CAPACITY when the mirror says a length would leave [0, capacity].  While the stream
+ * is being captured the mirror is not consulted: the device clamps a length that would leave
+ * [0, capacity] into it and sets VT_DEV_KV_OVERFLOW. */
 VT_API vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_stream stream);
 /* Cache bookkeeping: sets the length of `layer` (or all when -1) to len, device and host
  * mirror; synchronizes the stream (not capturable). */

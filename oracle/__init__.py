@@ -29,6 +29,10 @@ class OrShapes(ctypes.Structure):
                 ("d_ffn", _I32), ("rms_eps", _F64), ("rope_theta", _F64)]
 
 
+class OrQMat(ctypes.Structure):
+    _fields_ = [("q", _P), ("scales", _P), ("rows", _I64), ("k", _I64), ("block", _I32)]
+
+
 class OrLayer(ctypes.Structure):
     _fields_ = [(n, _P) for n in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate",
                                   "w_up", "w_down")]
@@ -68,6 +72,14 @@ def lib():
         L.or_quantize_vec.argtypes = [_P, _I64, _I32, _I32, _P, _P]
         L.or_quantize_vec.restype = _I32
         L.or_combine_q.argtypes = [ctypes.POINTER(_P), ctypes.POINTER(_P), _I32, _I64, _I32, _P, _P]
+        QM = ctypes.POINTER(OrQMat)
+        L.or_kv_append_q.argtypes = [ctypes.POINTER(OrShapes), _P, QM, QM, _I32, _I32, _P, _I32, _I64, _P, _P, _I64]
+        L.or_kv_append_q.restype = _I32
+        L.or_attn_partial_q.argtypes = [ctypes.POINTER(OrShapes), _P, QM, QM, _I32, _I32, _P, _I32, _P, _P, _P,
+                                         _I64, _I64, _P]
+        L.or_attn_partial_q.restype = _I32
+        L.or_ffn_partial_q.argtypes = [ctypes.POINTER(OrShapes), _P, QM, QM, QM, _I32, _P, _I32, _P]
+        L.or_ffn_partial_q.restype = _I32
         _lib = L
     return _lib
 
@@ -289,3 +301,106 @@ def combine_q(parts: Sequence[Tuple[np.ndarray, np.ndarray]], residual: Optional
     res = _f16(residual).reshape(-1) if residual is not None else None
     lib().or_combine_q(qp, sp, len(qs), count, block, res.ctypes.data if res is not None else None, out.ctypes.data)
     return out
+
+
+# ------------------------------------------------------------------ quantized shards ---------
+
+def _qm(m):
+    """(codes int8 [rows, k], scales binary16 [rows, nb], block) -> OrQMat (arrays kept alive by the caller)."""
+    q, sc, block = m
+    q = np.ascontiguousarray(q, np.int8)
+    sc = _f16(sc)
+    return OrQMat(q.ctypes.data, sc.ctypes.data, q.shape[0], q.shape[1], int(block)), (q, sc)
+
+
+def shard_qweights(wl, weights, heads: Tuple[int, int], cols: Tuple[int, int], attn_bits: int, ffn_bits: int,
+                   block: int = 32) -> Dict[str, tuple]:
+    """The shard's projections quantized with quantize_rows (bits 16: left out): query rows of heads,
+    K / V rows of their KV heads, the heads' columns of Wo, gate / up rows of the columns and the
+    columns of W_down, each as (codes, scales, block) with blocks along its contraction axis."""
+    dh = wl.d_head
+    (h0, h1), (c0, c1) = heads, cols
+    k0, k1 = kv_heads_of(wl, heads)
+    out = {}
+    if attn_bits in (8, 4) and h1 > h0:
+        for name, m in (("wq", weights["wq"][h0 * dh:h1 * dh]), ("wk", weights["wk"][k0 * dh:k1 * dh]),
+                        ("wv", weights["wv"][k0 * dh:k1 * dh]), ("wo", weights["wo"][:, h0 * dh:h1 * dh])):
+            out[name] = quantize_rows(np.ascontiguousarray(m), attn_bits, block) + (block,)
+    if ffn_bits in (8, 4) and c1 > c0:
+        for name, m in (("w_gate", weights["w_gate"][c0:c1]), ("w_up", weights["w_up"][c0:c1]),
+                        ("w_down", weights["w_down"][:, c0:c1])):
+            out[name] = quantize_rows(np.ascontiguousarray(m), ffn_bits, block) + (block,)
+    return out
+
+
+def kv_append_q(wl, weights, kv_heads: Tuple[int, int], x, pos0: int, kcache, vcache, qw) -> None:
+    x = _f16(x).reshape(-1, wl.d_model)
+    s = shapes_of(wl)
+    mk, kk = _qm(qw["wk"])
+    mv, kv = _qm(qw["wv"])
+    g = _f16(weights["attn_norm"])
+    rc = lib().or_kv_append_q(ctypes.byref(s), g.ctypes.data, ctypes.byref(mk), ctypes.byref(mv), kv_heads[0],
+                              kv_heads[1], x.ctypes.data, x.shape[0], int(pos0), kcache.ctypes.data,
+                              vcache.ctypes.data, kcache.shape[1])
+    if rc != 0:
+        raise ValueError("or_kv_append_q rejected its arguments")
+
+
+def attn_partial_q(wl, weights, heads: Tuple[int, int], x, pos, kcache, vcache, qw, window: int = 0):
+    x = _f16(x).reshape(-1, wl.d_model)
+    p = np.ascontiguousarray(pos, dtype=np.int64)
+    out = np.empty((x.shape[0], wl.d_model), np.float64)
+    s = shapes_of(wl)
+    empty = (np.zeros((0, 0), np.int8), np.zeros((0, 0), np.float16), 32)
+    mq, k1 = _qm(qw.get("wq", empty))
+    mo, k2 = _qm(qw.get("wo", empty))
+    g = _f16(weights["attn_norm"])
+    rc = lib().or_attn_partial_q(ctypes.byref(s), g.ctypes.data, ctypes.byref(mq), ctypes.byref(mo), heads[0],
+                                 heads[1], x.ctypes.data, x.shape[0], p.ctypes.data, _f16(kcache).ctypes.data,
+                                 _f16(vcache).ctypes.data, kcache.shape[1], int(window), out.ctypes.data)
+    if rc != 0:
+        raise ValueError("or_attn_partial_q rejected its arguments")
+    return out
+
+
+def ffn_partial_q(wl, weights, cols: Tuple[int, int], h, qw):
+    h = _f16(h).reshape(-1, wl.d_model)
+    out = np.empty((h.shape[0], wl.d_model), np.float64)
+    s = shapes_of(wl)
+    empty = (np.zeros((0, 0), np.int8), np.zeros((0, 0), np.float16), 32)
+    mg, k1 = _qm(qw.get("w_gate", empty))
+    mu, k2 = _qm(qw.get("w_up", empty))
+    md, k3 = _qm(qw.get("w_down", empty))
+    g = _f16(weights["ffn_norm"])
+    rc = lib().or_ffn_partial_q(ctypes.byref(s), g.ctypes.data, ctypes.byref(mg), ctypes.byref(mu), ctypes.byref(md),
+                                cols[1] - cols[0], h.ctypes.data, h.shape[0], out.ctypes.data)
+    if rc != 0:
+        raise ValueError("or_ffn_partial_q rejected its arguments")
+    return out
+
+
+def tp_layer_mixed(wl, weights, x, pos0: int, kcache, vcache, attn_bits, ffn_bits, window: int = 0,
+                   head_ranges=None, ffn_ranges=None):
+    """A decoder layer whose shards each run at their own precision (16: binary16 weights; 8 / 4:
+    block-quantized by quantize_rows): returns (h, x_next, attn_partials, ffn_partials)."""
+    head_ranges = wl.head_ranges if head_ranges is None else head_ranges
+    ffn_ranges = wl.ffn_ranges if ffn_ranges is None else ffn_ranges
+    x = _f16(x).reshape(-1, wl.d_model)
+    rows = x.shape[0]
+    qws = [shard_qweights(wl, weights, hr, cr, ab, fb)
+           for hr, cr, ab, fb in zip(head_ranges, ffn_ranges, attn_bits, ffn_bits)]
+    for hr, ab, qw in zip(head_ranges, attn_bits, qws):
+        kvh = kv_heads_of(wl, hr)
+        if kvh[1] > kvh[0]:
+            if ab == 16:
+                kv_append(wl, weights, kvh, x, pos0, kcache, vcache)
+            else:
+                kv_append_q(wl, weights, kvh, x, pos0, kcache, vcache, qw)
+    pos = np.arange(pos0, pos0 + rows)
+    ap = [attn_partial(wl, weights, hr, x, pos, kcache, vcache, window) if ab == 16 or hr[1] == hr[0]
+          else attn_partial_q(wl, weights, hr, x, pos, kcache, vcache, qw, window)
+          for hr, ab, qw in zip(head_ranges, attn_bits, qws)]
+    h = combine(ap, x)
+    fp = [ffn_partial(wl, weights, cr, h) if fb == 16 or cr[1] == cr[0] else ffn_partial_q(wl, weights, cr, h, qw)
+          for cr, fb, qw in zip(ffn_ranges, ffn_bits, qws)]
+    return h, combine(fp, h), ap, fp

@@ -345,6 +345,118 @@ void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64
     }
 }
 
+/* ---------------------------------------------------------------- quantized shards -------- */
+/* The layer steps of the attention and FFN blocks with every projection by a dequantized,
+ * block-quantized matrix (or_gemv_blockq); everything else is as in the binary16 functions above. */
+
+static int qmat_ok(const or_qmat* m, int64_t rows, int64_t k) {
+    return m && m->q && m->scales && m->block >= 1 && m->rows == rows && m->k == k;
+}
+
+int32_t or_kv_append_q(const or_shapes* s, const uint16_t* attn_norm, const or_qmat* wk, const or_qmat* wv,
+                       int32_t kvh0, int32_t kvh1, const uint16_t* x, int32_t rows, int64_t pos0, uint16_t* kcache,
+                       uint16_t* vcache, int64_t cap) {
+    if (!shapes_ok(s) || !attn_norm || kvh0 < 0 || kvh1 < kvh0 || kvh1 > s->n_kv_heads || rows < 0 || pos0 < 0 ||
+        pos0 + rows > cap)
+        return OR_ERR_ARG;
+    const int32_t D = s->d_model, dh = s->d_head, nk = kvh1 - kvh0;
+    if (!qmat_ok(wk, (int64_t)nk * dh, D) || !qmat_ok(wv, (int64_t)nk * dh, D)) return OR_ERR_ARG;
+    double* xin = (double*)malloc(sizeof(double) * D);
+    double* xh = (double*)malloc(sizeof(double) * D);
+    double* kk = (double*)malloc(sizeof(double) * (size_t)(nk * dh + 1));
+    double* vv = (double*)malloc(sizeof(double) * (size_t)(nk * dh + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        const int64_t p = pos0 + i;
+        load_row(x + (int64_t)i * D, D, xin);
+        or_rmsnorm(xin, attn_norm, D, s->rms_eps, xh);
+        or_gemv_blockq(wk->q, wk->scales, wk->rows, wk->k, wk->block, xh, kk);
+        or_gemv_blockq(wv->q, wv->scales, wv->rows, wv->k, wv->block, xh, vv);
+        for (int32_t j = 0; j < nk; ++j) {
+            or_rope(kk + (int64_t)j * dh, dh, p, s->rope_theta);
+            uint16_t* kd = kcache + ((int64_t)(kvh0 + j) * cap + p) * dh;
+            uint16_t* vd = vcache + ((int64_t)(kvh0 + j) * cap + p) * dh;
+            for (int32_t c = 0; c < dh; ++c) {
+                kd[c] = or_f64_to_f16(kk[(int64_t)j * dh + c]);
+                vd[c] = or_f64_to_f16(vv[(int64_t)j * dh + c]);
+            }
+        }
+    }
+    free(xin);
+    free(xh);
+    free(kk);
+    free(vv);
+    return OR_OK;
+}
+
+int32_t or_attn_partial_q(const or_shapes* s, const uint16_t* attn_norm, const or_qmat* wq, const or_qmat* wo,
+                          int32_t h0, int32_t h1, const uint16_t* x, int32_t rows, const int64_t* pos,
+                          const uint16_t* kcache, const uint16_t* vcache, int64_t cap, int64_t window,
+                          double* partial) {
+    if (!shapes_ok(s) || !attn_norm || h0 < 0 || h1 < h0 || h1 > s->n_heads || rows < 0) return OR_ERR_ARG;
+    const int32_t D = s->d_model, dh = s->d_head, nh = h1 - h0;
+    const int32_t group = s->n_heads / s->n_kv_heads;
+    if (nh > 0 && (!qmat_ok(wq, (int64_t)nh * dh, D) || !qmat_ok(wo, D, (int64_t)nh * dh))) return OR_ERR_ARG;
+    for (int32_t i = 0; i < rows; ++i)
+        if (pos[i] < 0 || pos[i] >= cap) return OR_ERR_ARG;
+    double* xin = (double*)malloc(sizeof(double) * D);
+    double* xh = (double*)malloc(sizeof(double) * D);
+    double* q = (double*)malloc(sizeof(double) * (size_t)(nh * dh + 1));
+    double* o = (double*)malloc(sizeof(double) * (size_t)(nh * dh + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        double* out = partial + (int64_t)i * D;
+        if (nh == 0) {
+            for (int32_t d = 0; d < D; ++d) out[d] = 0.0;
+            continue;
+        }
+        load_row(x + (int64_t)i * D, D, xin);
+        or_rmsnorm(xin, attn_norm, D, s->rms_eps, xh);
+        or_gemv_blockq(wq->q, wq->scales, wq->rows, wq->k, wq->block, xh, q);
+        for (int32_t h = 0; h < nh; ++h) or_rope(q + (int64_t)h * dh, dh, pos[i], s->rope_theta);
+        const int64_t first = window > 0 && pos[i] + 1 > window ? pos[i] + 1 - window : 0;
+#pragma omp parallel for schedule(static)
+        for (int32_t h = 0; h < nh; ++h) {
+            const int32_t j = (h0 + h) / group;
+            or_attend(q + (int64_t)h * dh, kcache + ((int64_t)j * cap + first) * dh,
+                      vcache + ((int64_t)j * cap + first) * dh, pos[i] + 1 - first, dh, NULL, o + (int64_t)h * dh);
+        }
+        or_gemv_blockq(wo->q, wo->scales, wo->rows, wo->k, wo->block, o, out);
+    }
+    free(xin);
+    free(xh);
+    free(q);
+    free(o);
+    return OR_OK;
+}
+
+int32_t or_ffn_partial_q(const or_shapes* s, const uint16_t* ffn_norm, const or_qmat* wg, const or_qmat* wu,
+                         const or_qmat* wd, int32_t nc, const uint16_t* h, int32_t rows, double* partial) {
+    if (!shapes_ok(s) || !ffn_norm || nc < 0 || rows < 0) return OR_ERR_ARG;
+    const int32_t D = s->d_model;
+    if (nc > 0 && (!qmat_ok(wg, nc, D) || !qmat_ok(wu, nc, D) || !qmat_ok(wd, D, nc))) return OR_ERR_ARG;
+    double* hin = (double*)malloc(sizeof(double) * D);
+    double* hh = (double*)malloc(sizeof(double) * D);
+    double* g = (double*)malloc(sizeof(double) * (size_t)(nc + 1));
+    double* u = (double*)malloc(sizeof(double) * (size_t)(nc + 1));
+    for (int32_t i = 0; i < rows; ++i) {
+        double* out = partial + (int64_t)i * D;
+        if (nc == 0) {
+            for (int32_t d = 0; d < D; ++d) out[d] = 0.0;
+            continue;
+        }
+        load_row(h + (int64_t)i * D, D, hin);
+        or_rmsnorm(hin, ffn_norm, D, s->rms_eps, hh);
+        or_gemv_blockq(wg->q, wg->scales, wg->rows, wg->k, wg->block, hh, g);
+        or_gemv_blockq(wu->q, wu->scales, wu->rows, wu->k, wu->block, hh, u);
+        for (int32_t j = 0; j < nc; ++j) g[j] = or_silu(g[j]) * u[j];
+        or_gemv_blockq(wd->q, wd->scales, wd->rows, wd->k, wd->block, g, out);
+    }
+    free(hin);
+    free(hh);
+    free(g);
+    free(u);
+    return OR_OK;
+}
+
 /* ---------------------------------------------------------------- quantized partials ------ */
 /* Communication scaling (Voltron Section 4.3.2): activations sent between devices are lowered to
  * INT8 or INT4.  Under tensor parallelism those are the shard partials sent to the main device.

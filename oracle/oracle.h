@@ -112,6 +112,33 @@ int32_t or_quantize_rows(const uint16_t* w, int64_t rows, int64_t k, int32_t bit
 void or_gemv_blockq(const int8_t* q, const uint16_t* scales, int64_t rows, int64_t k, int32_t block,
                     const double* x, double* y);
 
+/* A block-quantized weight matrix [rows][k] (codes q, one int8 per weight, and binary16 scales
+ * [rows][ceil(k / block)], as or_quantize_rows writes them); its dequantized weight is q * d. */
+typedef struct {
+    const int8_t* q;
+    const uint16_t* scales;
+    int64_t rows, k;
+    int32_t block;
+} or_qmat;
+
+/* The attention and FFN blocks of a shard whose projections are block-quantized (mixed-precision
+ * shards, Section 3.2.2 / 4.2.2): the same steps as or_kv_append, or_attn_partial_window and
+ * or_ffn_partial, every projection by the dequantized matrix.
+ *   or_kv_append_q:    wk, wv: rows of KV heads [kvh0, kvh1) of Wk / Wv, [nk*dh][D].
+ *   or_attn_partial_q: wq: rows of query heads [h0, h1) of Wq, [nh*dh][D]; wo: columns
+ *                      [h0*dh, h1*dh) of Wo, [D][nh*dh]; window as or_attn_partial_window.
+ *   or_ffn_partial_q:  wg, wu: rows [c0, c1) of W_gate / W_up, [nc][D]; wd: columns [c0, c1) of
+ *                      W_down, [D][nc]. */
+int32_t or_kv_append_q(const or_shapes* s, const uint16_t* attn_norm, const or_qmat* wk, const or_qmat* wv,
+                       int32_t kvh0, int32_t kvh1, const uint16_t* x, int32_t rows, int64_t pos0, uint16_t* kcache,
+                       uint16_t* vcache, int64_t cap);
+int32_t or_attn_partial_q(const or_shapes* s, const uint16_t* attn_norm, const or_qmat* wq, const or_qmat* wo,
+                          int32_t h0, int32_t h1, const uint16_t* x, int32_t rows, const int64_t* pos,
+                          const uint16_t* kcache, const uint16_t* vcache, int64_t cap, int64_t window,
+                          double* partial);
+int32_t or_ffn_partial_q(const or_shapes* s, const uint16_t* ffn_norm, const or_qmat* wg, const or_qmat* wu,
+                         const or_qmat* wd, int32_t nc, const uint16_t* h, int32_t rows, double* partial);
+
 /* Quantized shard partials (Section 4.3.2, communication scaling; reading in oracle.c):
  * codes q [n] and binary16 scales [ceil(n / block)] of a binary32 vector, and the combine of
  * n quantized partials with a binary16 residual (NULL: zero) into binary16 out [count]. */

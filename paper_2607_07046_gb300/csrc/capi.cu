@@ -1117,12 +1117,14 @@ extern "C" vt_status vt_kv_advance(vt_kv* kv, int32_t layer, int32_t n, vt_strea
     const int L = kv->p->m->s.n_layers;
     if (layer < -1 || layer >= L) return fail(VT_ERR_INVALID_ARG, "layer %d out of range", layer);
     const int first = layer < 0 ? 0 : layer, count = layer < 0 ? L : 1;
-    for (int l = first; l < first + count; ++l)
-        if ((int64_t)kv->h_len[l] + n > kv->cap || (int64_t)kv->h_len[l] + n < 0)
-            return fail(VT_ERR_KV_CAPACITY, "advancing layer %d from %d by %d leaves [0, %d]", l,
-                        kv->h_len[l], n, kv->cap);
-    VT_CUDA(launch_kv_advance(kv->len, first, count, n, (cudaStream_t)stream));
-    if (!capturing((cudaStream_t)stream))
+    const bool cap_mode = capturing((cudaStream_t)stream);
+    if (!cap_mode)  // while capturing, the device clamps and flags instead (the mirror is stale)
+        for (int l = first; l < first + count; ++l)
+            if ((int64_t)kv->h_len[l] + n > kv->cap || (int64_t)kv->h_len[l] + n < 0)
+                return fail(VT_ERR_KV_CAPACITY, "advancing layer %d from %d by %d leaves [0, %d]", l,
+                            kv->h_len[l], n, kv->cap);
+    VT_CUDA(launch_kv_advance(kv->len, first, count, n, kv->cap, kv->status, (cudaStream_t)stream));
+    if (!cap_mode)
         for (int l = first; l < first + count; ++l) kv->h_len[l] += n;
     return ok();
 }
@@ -1625,7 +1627,7 @@ extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, c
         VT_CUDA(launch_combine(c, st));
         cur = dst;
     }
-    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, 1, st));
+    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, 1, kv->cap, kv->status, st));
     if (!capturing(st))
         for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += 1;
     return ok();
@@ -1669,7 +1671,7 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
             cur = dst;
         }
     }
-    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, n, st));
+    VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, n, kv->cap, kv->status, st));
     if (!capturing(st))
         for (int l = 0; l < s.n_layers; ++l) kv->h_len[l] += n;
     return ok();

@@ -908,14 +908,22 @@ cudaError_t launch_fill_zero_f32(float* p, int64_t n, cudaStream_t st) {
     return launch_k(k_fill_zero_f32, dim3((unsigned)blocks), dim3(256), 0, st, p, n);
 }
 
-__global__ void k_kv_advance(int32_t* len, int first, int count, int delta) {
+// len[l] += delta for the layers [first, first + count); a result outside [0, cap] is clamped
+// into it and flagged VT_DEV_KV_OVERFLOW (the host checks this before launch, except while a
+// stream is being captured, when its length mirror does not follow the device).
+__global__ void k_kv_advance(int32_t* len, int first, int count, int delta, int cap, uint32_t* status) {
     pdl_wait();
     pdl_launch_dependents();
-    for (int i = threadIdx.x; i < count; i += blockDim.x) len[first + i] += delta;
+    for (int i = threadIdx.x; i < count; i += blockDim.x) {
+        const int64_t v = (int64_t)len[first + i] + delta;
+        if (v < 0 || v > cap) set_status(status, VT_DEV_KV_OVERFLOW);
+        len[first + i] = (int32_t)(v < 0 ? 0 : (v > cap ? cap : v));
+    }
 }
 
-cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, cudaStream_t st) {
-    return launch_k(k_kv_advance, dim3(1), dim3(128), 0, st, len, first, count, delta);
+cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, int cap, uint32_t* status,
+                              cudaStream_t st) {
+    return launch_k(k_kv_advance, dim3(1), dim3(128), 0, st, len, first, count, delta, cap, status);
 }
 
 __global__ void k_rope_table(float2* tab, int max_seq, int half, int dh, double theta) {

@@ -122,7 +122,8 @@ cudaError_t launch_ffn_decode(const FfnDecodeArgs& a, int grid, cudaStream_t st)
 cudaError_t launch_transpose_f16(const __half* src, int64_t src_ld, int rows, int cols, __half* dst,
                                  int64_t dst_ld, cudaStream_t st);
 cudaError_t launch_fill_zero_f32(float* p, int64_t n, cudaStream_t st);
-cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, cudaStream_t st);
+cudaError_t launch_kv_advance(int32_t* len, int first, int count, int delta, int cap, uint32_t* status,
+                              cudaStream_t st);
 cudaError_t launch_rope_table(float2* tab, int max_seq, int dh, double theta, cudaStream_t st);
 cudaError_t launch_embed(const __half* table, const int32_t* ids, int n, int d, int vocab,
                          __half* out, uint32_t* status, cudaStream_t st);

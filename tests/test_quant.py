@@ -13,6 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
+import synthetic
 
 
 def f16(a):
@@ -164,3 +165,95 @@ def test_quantized_combine_equals_numpy_and_stays_within_the_bound():
     z = oracle.quantize_vec(np.zeros(D, np.float32), 8)
     one = oracle.quantize_vec(parts[0], 8)
     assert np.array_equal(oracle.combine_q([z, one], None), oracle.combine_q([one], None))
+
+
+# ------------------------------------------------------------------ quantized shards (oracle)
+
+def _exact_layer(wl, bits, seed=7):
+    """Weights that are exactly q * d in binary16: codes drawn in [-qmax, qmax], one power-of-two
+    scale per block of 32 along each matrix's input axis.  Returns the binary16 weights and, per
+    matrix, its full (codes, scales)."""
+    rng = np.random.default_rng(seed)
+    qmax = 127 if bits == 8 else 7
+    shapes = {"wq": (wl.n_heads * wl.d_head, wl.d_model), "wk": (wl.n_kv_heads * wl.d_head, wl.d_model),
+              "wv": (wl.n_kv_heads * wl.d_head, wl.d_model), "wo": (wl.d_model, wl.n_heads * wl.d_head),
+              "w_gate": (wl.d_ffn, wl.d_model), "w_up": (wl.d_ffn, wl.d_model), "w_down": (wl.d_model, wl.d_ffn)}
+    w, qd = {}, {}
+    for name, (r, k) in shapes.items():
+        q = rng.integers(-qmax, qmax + 1, size=(r, k)).astype(np.int8)
+        e = rng.integers(6, 10, size=(r, (k + 31) // 32))
+        d = np.ldexp(1.0, -e).astype(np.float16)
+        deq = q.astype(np.float64) * np.repeat(d.astype(np.float64), 32, axis=1)[:, :k]
+        w[name] = deq.astype(np.float16)
+        assert np.array_equal(w[name].astype(np.float64), deq)  # exact in binary16
+        qd[name] = (q, d)
+    w["attn_norm"] = synthetic.normal_f16((wl.d_model,), 5, 1.0, 0.02)
+    w["ffn_norm"] = synthetic.normal_f16((wl.d_model,), 6, 1.0, 0.02)
+    return w, qd
+
+
+def _slice_q(qd, name, rows=None, cols=None):
+    q, d = qd[name]
+    if rows is not None:
+        return (q[rows[0]:rows[1]], d[rows[0]:rows[1]], 32)
+    return (np.ascontiguousarray(q[:, cols[0]:cols[1]]), np.ascontiguousarray(d[:, cols[0] // 32:(cols[1] + 31) // 32]), 32)
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_quantized_shard_functions_equal_the_binary16_ones_on_exact_weights(bits):
+    """When every weight is exactly its dequantized value, the quantized-shard attention, K/V append
+    and FFN functions must give bit for bit what the binary16 functions give (same sums in the same
+    order): this ties the quantized path to the pinned binary16 layer."""
+    wl = synthetic.small("qexact", n_layers=1, d_model=128, n_heads=4, n_kv_heads=2, d_head=32, d_ffn=96,
+                         head_ranges=((0, 2), (2, 4)), ffn_ranges=((0, 64), (64, 96)))
+    w, qd = _exact_layer(wl, bits)
+    dh, cap, L = wl.d_head, 16, 5
+    x = wl.hidden(3, stream=1)
+    for (h0, h1), (c0, c1) in zip(wl.head_ranges, wl.ffn_ranges):
+        k0, k1 = oracle.kv_heads_of(wl, (h0, h1))
+        qw = {"wq": _slice_q(qd, "wq", rows=(h0 * dh, h1 * dh)), "wk": _slice_q(qd, "wk", rows=(k0 * dh, k1 * dh)),
+              "wv": _slice_q(qd, "wv", rows=(k0 * dh, k1 * dh)), "wo": _slice_q(qd, "wo", cols=(h0 * dh, h1 * dh)),
+              "w_gate": _slice_q(qd, "w_gate", rows=(c0, c1)), "w_up": _slice_q(qd, "w_up", rows=(c0, c1)),
+              "w_down": _slice_q(qd, "w_down", cols=(c0, c1))}
+        kc1, vc1 = wl.kv_fill(0, L, cap)
+        kc2, vc2 = kc1.copy(), vc1.copy()
+        oracle.kv_append(wl, w, (k0, k1), x, L, kc1, vc1)
+        oracle.kv_append_q(wl, w, (k0, k1), x, L, kc2, vc2, qw)
+        assert np.array_equal(kc1, kc2) and np.array_equal(vc1, vc2)
+        pos = np.arange(L, L + 3)
+        for window in (0, 2):
+            a = oracle.attn_partial(wl, w, (h0, h1), x, pos, kc1, vc1, window)
+            b = oracle.attn_partial_q(wl, w, (h0, h1), x, pos, kc1, vc1, qw, window)
+            assert np.array_equal(a, b)
+        a = oracle.ffn_partial(wl, w, (c0, c1), x)
+        b = oracle.ffn_partial_q(wl, w, (c0, c1), x, qw)
+        assert np.array_equal(a, b)
+
+
+def test_mixed_layer_with_all_binary16_shards_is_the_binary16_layer():
+    wl = synthetic.small("qmix16", n_layers=1)
+    w = wl.layer_weights(0)
+    x = wl.hidden(2, stream=3)
+    kc1, vc1 = oracle.new_cache(wl, 16)
+    kc2, vc2 = oracle.new_cache(wl, 16)
+    ref = oracle.tp_layer(wl, w, x, 0, kc1, vc1)
+    got = oracle.tp_layer_mixed(wl, w, x, 0, kc2, vc2, [16, 16], [16, 16])
+    assert np.array_equal(ref[1], got[1]) and np.array_equal(kc1, kc2)
+
+
+@pytest.mark.parametrize("bits,bound", [(8, 2e-2), (4, 3e-1)])
+def test_mixed_layer_error_is_that_of_the_weight_rounding(bits, bound):
+    """Quantizing real binary16 weights moves the layer's partials by the quantization error only:
+    the relative difference stays within a loose bound set by d / 2 per weight (INT8: ~1/254 of
+    a block's largest weight; INT4: ~1/14), and shrinks from INT4 to INT8."""
+    wl = synthetic.small("qmixerr", n_layers=1, d_model=128, n_heads=4, n_kv_heads=2, d_head=32, d_ffn=96,
+                         head_ranges=((0, 2), (2, 4)), ffn_ranges=((0, 64), (64, 96)))
+    w = wl.layer_weights(0)
+    x = wl.hidden(2, stream=4)
+    kc1, vc1 = oracle.new_cache(wl, 16)
+    kc2, vc2 = oracle.new_cache(wl, 16)
+    _, _, ap, fp = oracle.tp_layer(wl, w, x, 0, kc1, vc1)
+    _, _, aq, fq = oracle.tp_layer_mixed(wl, w, x, 0, kc2, vc2, [bits, bits], [bits, bits])
+    for a, b in list(zip(ap, aq)) + list(zip(fp, fq)):
+        rel = np.linalg.norm(a - b) / np.linalg.norm(a)
+        assert 0 < rel < bound
