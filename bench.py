@@ -135,6 +135,29 @@ def decode_bytes_per_token(wl, kv_mean):
     return L * (w + kv)
 
 
+def quant_bytes_per_token(wl, bits, kv_mean):
+    """Algorithmic HBM bytes of one decode token with every shard block-quantized at `bits`: the
+    codes (one byte per weight at 8 bits, half a byte at 4; rows padded to whole blocks of 32) and
+    one fp16 scale per block of every projection, the RMSNorm gains, the cache at the mean length."""
+    D, H, Hk, dh, F, L = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, wl.n_layers
+    cb = 1.0 if bits == 8 else 0.5
+
+    def mat(rows, k):
+        nb = (k + 31) // 32
+        return rows * (nb * 32 * cb + nb * 2)
+
+    w = 0.0
+    for (h0, h1), (c0, c1) in zip(wl.head_ranges, wl.ffn_ranges):
+        hq, c = h1 - h0, c1 - c0
+        hk = hq * Hk // H
+        if hq:
+            w += mat((hq + 2 * hk) * dh, D) + mat(D, hq * dh) + 2 * D
+        if c:
+            w += mat(2 * c, D) + mat(D, c) + 2 * D
+    kv = 2 * 2 * Hk * dh * (kv_mean + 1)
+    return int(L * (w + kv))
+
+
 def kernels_per_token(wl):
     """Kernels of one vt_decode_token: per layer, 3 per non-empty ATTN shard (QKV GEMV,
     attention, O GEMV), 1 per non-empty FFN shard (fused FFN), 2 combines; 1 KV advance."""
@@ -497,7 +520,7 @@ def run_decode(args, rank, world):
     return line, clk.summary()
 
 
-def run_decode_workload(cid, steps, warmup):
+def run_decode_workload(cid, steps, warmup, bits=16):
     """Decode tok/s of one more workload (the 13B uneven 3-way and the 8B GQA 4-way shapes), timed
     like the headline one: vt_decode_token replayed as a CUDA graph over the workload's KV schedule
     (kv_len -> kv_len + decode_steps - 1, then rewound), inputs resident on the device."""
@@ -511,8 +534,10 @@ def run_decode_workload(cid, steps, warmup):
     cap = wl.kv_len + sched + 8
     stream = torch.cuda.Stream()
     t_setup = time.perf_counter()
+    prec = None if bits == 16 else (lambda l, d, b: bits)
     with torch.cuda.stream(stream):
-        st = Stack(shapes_for(vt, wl, cap), wl.layer_weights, wl.head_ranges, wl.ffn_ranges, cap, stream=stream)
+        st = Stack(shapes_for(vt, wl, cap), wl.layer_weights, wl.head_ranges, wl.ffn_ranges, cap, stream=stream,
+                   precision=prec)
     try:
         g = wl.n_heads // wl.n_kv_heads
         for l in range(wl.n_layers):
@@ -536,10 +561,11 @@ def run_decode_workload(cid, steps, warmup):
         st.close()
     hbm, _, _, peak_kind = measured_peaks()
     kv_mean = wl.kv_len + (min(steps, sched) - 1) / 2.0
-    step_bytes = decode_bytes_per_token(wl, kv_mean)
+    step_bytes = decode_bytes_per_token(wl, kv_mean) if bits == 16 else quant_bytes_per_token(wl, bits, kv_mean)
     achieved = step_bytes / (ms * 1e-3) / 1e9
     return {
-        "workload": wl.name,
+        "workload": wl.name if bits == 16 else f"{wl.name}, every shard block-quantized to {bits} bits "
+                                                f"(blocks of 32, fp16 scales)",
         "shape": f"{wl.n_layers} layers, D {wl.d_model}, {wl.n_heads} query / {wl.n_kv_heads} KV heads x "
                  f"{wl.d_head}, FFN {wl.d_ffn}; heads {[h1 - h0 for h0, h1 in wl.head_ranges]}, "
                  f"FFN columns {[c1 - c0 for c0, c1 in wl.ffn_ranges]}; KV {wl.kv_len} -> {wl.kv_len + sched - 1}",
@@ -620,6 +646,7 @@ def main():
     line["clocks"] = clocks
     if world == 1 and args.other_steps > 0 and not args.layers:
         line["other_workloads"] = [run_decode_workload(cid, args.other_steps, 8) for cid in (3, 5)]
+        line["quantized_shards"] = [run_decode_workload(2, args.other_steps, 8, bits) for bits in (8, 4)]
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_decode(synthetic.WORKLOADS[2])
         if "prefill" in line:

@@ -296,6 +296,34 @@ VT_API vt_status vt_shard_weights_read(const vt_partition* part, vt_shard shard,
 VT_API vt_status vt_shard_weight_layout(const vt_partition* part, vt_shard shard, int32_t which,
                                  int64_t* rows, int64_t* row_stride);
 
+/* vt_partition_set_precision (Section 3.2.2, precision heterogeneity: a device holds its shard at
+ * its own precision; Section 4.2.2 allocates the precision per layer; Section 5.1 names k-quant
+ * formats without defining them): stores shard `shard` at `bits` = 8 or 4 (block-quantized) or
+ * 16 (fp16, sliced again from the model).  Format (the library's reading of k-quant): every weight
+ * row is cut into blocks of 32 weights along its input axis; a block keeps the fp16 scale
+ * d = fp16(amax / qmax) (qmax 127 or 7) and each weight the code round-half-even(w / d) clamped to
+ * [-qmax, qmax], both divisions in fp32 (the codes of vt_quantize_rows, bit for bit).  Quantized
+ * tensors: ATTN: the QKV rows (rows along D) and the O columns (rows of Wo_s [D][h_s dh] along the
+ * shard's columns); FFN: the gate/up rows (along D) and the down projection as Wd[:, c0:c1]
+ * ([D][c] rows along the shard's columns).  Codes are stored packed (one byte per 8-bit code, two
+ * 4-bit codes per byte) with the fp16 scales, replacing the shard's fp16 weights (its bytes halve
+ * or quarter, plus one scale per 32 weights).  Decode (vt_decode_step, vt_decode_step_static,
+ * vt_decode_token_sharded) runs quantized shards with a dequantizing kernel; vt_decode_token then
+ * runs the per-shard kernels (vt_decode_token_fused_available says why); prefill needs fp16
+ * shards (VT_ERR_STATE).  Precisions are fixed while a KV cache of the partition exists
+ * (VT_ERR_STATE): set them before vt_kv_create.  An empty shard stores nothing and stays fp16.
+ * Synchronizes `stream`.  Errors: VT_ERR_INVALID_ARG (bad shard or bits), VT_ERR_ALLOC, VT_ERR_CUDA.
+ * vt_shard_precision returns a shard's bits (16, 8 or 4; 0 for a bad shard). */
+VT_API vt_status vt_partition_set_precision(vt_partition* part, vt_shard shard, int32_t bits, vt_stream stream);
+VT_API int32_t vt_shard_precision(const vt_partition* part, vt_shard shard);
+/* Test hook (library plumbing): the codes and scales of a block-quantized shard tensor, synchronous.
+ * which: 1 = QKV rows [(h_s + 2 hk_s) dh][D] (rows in the order of vt_shard_weight_layout), 2 = O
+ * [D][h_s dh], 4 = gate/up rows [2 c][D] (interleaved), 5 = down [D][c] (columns c0 .. c1 - 1 of
+ * Wd, not transposed).  codes: host int8 [rows][k]; scales: host fp16 [rows][ceil(k / 32)].
+ * VT_ERR_STATE when the tensor is not quantized. */
+VT_API vt_status vt_shard_qweights_read(const vt_partition* part, vt_shard shard, int32_t which, int8_t* codes,
+                                        void* scales);
+
 /* ---------------------------------------------------------------- KV cache ---------------------
  * vt_kv_create (Section 2.1, "LLM Inference": the KV cache that prefill fills and every decode
  * step appends to; split by KV head among the devices as tensor parallelism splits the heads,

@@ -117,6 +117,8 @@ cudaError_t init_library() {
         g_init_err = init_prefill_kernels();
         if (g_init_err != cudaSuccess) return;
         g_init_err = init_token_kernels();
+        if (g_init_err != cudaSuccess) return;
+        g_init_err = init_quant_kernels();
     });
     return g_init_err;
 }
@@ -147,22 +149,27 @@ struct vt_model {
 struct AttnShard {
     void* base = nullptr;
     __half* norm = nullptr;
-    __half* wqkv = nullptr;  // [(hq + 2 hk) dh][D]
-    __half* wo = nullptr;    // [D][hq dh]
+    __half* wqkv = nullptr;  // [(hq + 2 hk) dh][D] (fp16 shards)
+    __half* wo = nullptr;    // [D][hq dh]          (fp16 shards)
     int h0 = 0, h1 = 0, kv0 = 0, kv1 = 0;
+    int bits = 16;           // 16: fp16 weights; 8 / 4: block-quantized (qkv, o)
+    QMatDev qkv, o;          // quantized shards: QKV rows [(hq + 2 hk) dh][D] in the same row order, O [D][hq dh]
 };
 
 struct FfnShard {
     void* base = nullptr;
     __half* norm = nullptr;
-    __half* wgu = nullptr;  // [2c][D], gate/up rows interleaved
-    __half* wdt = nullptr;  // [c][D], row j = column c0 + j of Wd
+    __half* wgu = nullptr;  // [2c][D], gate/up rows interleaved (fp16 shards)
+    __half* wdt = nullptr;  // [c][D], row j = column c0 + j of Wd (fp16 shards)
     int c0 = 0, c1 = 0;
+    int bits = 16;          // 16: fp16 weights; 8 / 4: block-quantized (gu, down)
+    QMatDev gu, down;       // quantized shards: gate/up rows [2c][D] interleaved, down columns [D][c]
 };
 
 struct DecodeScratch {  // per device of the partition
     float* q = nullptr;     // [hq][dh] rotated queries of the token
     float* attn = nullptr;  // [hq][dh] attention output (input of the O projection)
+    float* u = nullptr;     // [c] SwiGLU activations (quantized FFN shards)
     int ffn_grid = 0;       // CTAs of the fused FFN kernel
 };
 
@@ -177,6 +184,7 @@ struct vt_partition {
     std::vector<DecodeScratch> dec;
     std::vector<void*> owned;  // every allocation besides the shard bases
     bool counted = false;      // counted in the model's n_partitions
+    mutable int n_kv = 0;      // live KV caches of the partition (precisions are fixed while any exists)
     uint32_t* status = nullptr;
     // whole-stack buffers
     float* dpart = nullptr;     // [n_dev][D] decode partials (kept zero between blocks)
@@ -191,7 +199,8 @@ struct vt_partition {
     int max_hq = 0, max_ld = 0;
     size_t q_slot = 0, u_slot = 0;
     // persistent decode-token kernel: shapes and scratch (the KV object adds its tables)
-    bool tok_ok = false;
+    bool tok_planned = false;  // the kernel has a plan (and scratch) for the partition's shapes
+    bool tok_ok = false;       // ... and every shard is fp16 (quantized shards run per-shard kernels)
     std::string tok_why;
     TokPlan tok_plan;
     TokArgs tok_base{};
@@ -485,27 +494,7 @@ extern "C" vt_status vt_quantize_rows(const void* w, int64_t rows, int64_t k, in
     if (!w || !q || !scales) return fail(VT_ERR_INVALID_ARG, "w, q and scales must not be NULL");
     if (rows < 0 || k < 0 || block < 1 || (bits != 8 && bits != 4))
         return fail(VT_ERR_INVALID_ARG, "rows %lld, k %lld, block %d, bits %d", (long long)rows, (long long)k, block, bits);
-    const __half* src = static_cast<const __half*>(w);
-    __half* sc = static_cast<__half*>(scales);
-    const int qmax = bits == 8 ? 127 : 7;
-    const int64_t nb = (k + block - 1) / block;
-    for (int64_t r = 0; r < rows; ++r)
-        for (int64_t b = 0; b < nb; ++b) {
-            const int64_t e0 = b * block, e1 = std::min(k, e0 + block);
-            float amax = 0.0f;
-            for (int64_t e = e0; e < e1; ++e) amax = std::max(amax, std::fabs(__half2float(src[r * k + e])));
-            const __half d16 = __float2half_rn(amax / (float)qmax);
-            const float d = __half2float(d16);
-            sc[r * nb + b] = d16;
-            for (int64_t e = e0; e < e1; ++e) {
-                int c = 0;
-                if (d != 0.0f) {
-                    const float x = std::nearbyint(__half2float(src[r * k + e]) / d);  // ties to even
-                    c = x > (float)qmax ? qmax : (x < (float)-qmax ? -qmax : (int)x);
-                }
-                q[r * k + e] = (int8_t)c;
-            }
-        }
+    quantize_rows_host(static_cast<const __half*>(w), rows, k, bits, block, q, static_cast<__half*>(scales));
     return ok();
 }
 
@@ -748,6 +737,88 @@ vt_status owned_alloc(vt_partition* p, size_t bytes, void** out) {
 
 }  // namespace
 
+// Bytes of the row-pointer table the gather kernel reads while a shard is sliced.
+static size_t gather_table_bytes(const vt_shapes& s) {
+    const size_t rows = std::max((size_t)(s.n_heads + 2 * s.n_kv_heads) * s.d_head, (size_t)2 * s.d_ffn);
+    return rows * sizeof(void*);
+}
+
+// The fp16 ATTN shard (l, d) sliced from the model's canonical weights into its own allocation:
+// gain, QKV rows (query heads, then K heads, then V heads; each head's rows in RoPE-pair order),
+// O columns.  rows_dev: a device table of gather_table_bytes (reused; the stream is synchronized).
+static vt_status slice_attn_fp16(vt_partition* p, int l, int d, const __half** rows_dev, cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const LayerPtrs& L = p->m->layer[l];
+    const int D = s.d_model, dh = s.d_head, H = s.n_heads;
+    AttnShard& as = p->attn[(size_t)l * p->n_dev + d];
+    const int hq = as.h1 - as.h0, hk = as.kv1 - as.kv0;
+    const int qkv_rows = (hq + 2 * hk) * dh;
+    if (hq == 0) return VT_OK;
+    const size_t bytes = align256((size_t)D * 2) + align256((size_t)qkv_rows * D * 2) + align256((size_t)D * hq * dh * 2);
+    as.base = p->m->alloc.get(bytes);
+    if (!as.base) return fail(VT_ERR_ALLOC, "shard allocation failed");
+    Bump b{static_cast<uint8_t*>(as.base)};
+    as.norm = b.take<__half>(D);
+    as.wqkv = b.take<__half>((size_t)qkv_rows * D);
+    as.wo = b.take<__half>((size_t)D * hq * dh);
+    as.bits = 16;
+    VT_CUDA(cudaMemcpyAsync(as.norm, L.attn_norm, (size_t)D * 2, cudaMemcpyDeviceToDevice, st));
+    std::vector<const __half*> rows_host;
+    for (int blk = 0; blk < hq + 2 * hk; ++blk) {
+        const __half* src;
+        int head;
+        if (blk < hq) {
+            src = L.wq;
+            head = as.h0 + blk;
+        } else if (blk < hq + hk) {
+            src = L.wk;
+            head = as.kv0 + blk - hq;
+        } else {
+            src = L.wv;
+            head = as.kv0 + blk - hq - hk;
+        }
+        for (int i = 0; i < dh / 2; ++i) {
+            rows_host.push_back(src + ((size_t)head * dh + i) * D);
+            rows_host.push_back(src + ((size_t)head * dh + i + dh / 2) * D);
+        }
+    }
+    VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*), cudaMemcpyHostToDevice, st));
+    VT_CUDA(launch_gather_rows(rows_dev, as.wqkv, (int)rows_host.size(), D, D, st));
+    VT_CUDA(cudaStreamSynchronize(st));  // rows_host / rows_dev are reused
+    VT_CUDA(cudaMemcpy2DAsync(as.wo, (size_t)hq * dh * 2, L.wo + (size_t)as.h0 * dh, (size_t)H * dh * 2,
+                              (size_t)hq * dh * 2, D, cudaMemcpyDeviceToDevice, st));
+    return VT_OK;
+}
+
+// The fp16 FFN shard (l, d): gain, gate/up rows interleaved, the transposed down columns.
+static vt_status slice_ffn_fp16(vt_partition* p, int l, int d, const __half** rows_dev, cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const LayerPtrs& L = p->m->layer[l];
+    const int D = s.d_model, F = s.d_ffn;
+    FfnShard& fs = p->ffn[(size_t)l * p->n_dev + d];
+    const int c = fs.c1 - fs.c0;
+    if (c == 0) return VT_OK;
+    const size_t bytes = align256((size_t)D * 2) + align256((size_t)2 * c * D * 2) + align256((size_t)c * D * 2);
+    fs.base = p->m->alloc.get(bytes);
+    if (!fs.base) return fail(VT_ERR_ALLOC, "shard allocation failed");
+    Bump b{static_cast<uint8_t*>(fs.base)};
+    fs.norm = b.take<__half>(D);
+    fs.wgu = b.take<__half>((size_t)2 * c * D);
+    fs.wdt = b.take<__half>((size_t)c * D);
+    fs.bits = 16;
+    VT_CUDA(cudaMemcpyAsync(fs.norm, L.ffn_norm, (size_t)D * 2, cudaMemcpyDeviceToDevice, st));
+    std::vector<const __half*> rows_host;
+    for (int j = 0; j < c; ++j) {
+        rows_host.push_back(L.w_gate + (size_t)(fs.c0 + j) * D);
+        rows_host.push_back(L.w_up + (size_t)(fs.c0 + j) * D);
+    }
+    VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*), cudaMemcpyHostToDevice, st));
+    VT_CUDA(launch_gather_rows(rows_dev, fs.wgu, (int)rows_host.size(), D, D, st));
+    VT_CUDA(cudaStreamSynchronize(st));
+    VT_CUDA(launch_transpose_f16(L.w_down + fs.c0, F, D, c, fs.wdt, D, st));
+    return VT_OK;
+}
+
 extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range* heads,
                                          const vt_range* cols, vt_stream stream,
                                          vt_partition** out) {
@@ -779,93 +850,23 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     };
 
     // host staging of row-pointer tables for the gather kernel (per layer)
-    std::vector<const __half*> rows_host;
-    const __half** rows_dev = nullptr;
-    size_t rows_cap = (size_t)(H + 2 * s.n_kv_heads) * dh;
-    if ((size_t)2 * F > rows_cap) rows_cap = (size_t)2 * F;
-    rows_dev = static_cast<const __half**>(A.get(rows_cap * sizeof(void*)));
+    const __half** rows_dev = static_cast<const __half**>(A.get(gather_table_bytes(s)));
     if (!rows_dev) return bail(fail(VT_ERR_ALLOC, "allocating the gather table failed"));
-
     vt_status r = VT_OK;
-    for (int l = 0; l < s.n_layers && r == VT_OK; ++l) {
-        const LayerPtrs& L = m->layer[l];
-        for (int d = 0; d < n; ++d) {
-            // ---------------------------------------------------------- ATTN shard
+    for (int l = 0; l < s.n_layers && r == VT_OK; ++l)
+        for (int d = 0; d < n && r == VT_OK; ++d) {
             AttnShard& as = p->attn[(size_t)l * n + d];
             as.h0 = heads[d].begin;
             as.h1 = heads[d].end;
             as.kv0 = as.h0 / g;
             as.kv1 = as.h1 / g;
-            const int hq = as.h1 - as.h0, hk = as.kv1 - as.kv0;
-            const int qkv_rows = (hq + 2 * hk) * dh;
-            if (hq > 0) {
-                const size_t bytes = align256((size_t)D * 2) + align256((size_t)qkv_rows * D * 2) +
-                                     align256((size_t)D * hq * dh * 2);
-                as.base = A.get(bytes);
-                if (!as.base) return bail(fail(VT_ERR_ALLOC, "shard allocation failed"));
-                Bump b{static_cast<uint8_t*>(as.base)};
-                as.norm = b.take<__half>(D);
-                as.wqkv = b.take<__half>((size_t)qkv_rows * D);
-                as.wo = b.take<__half>((size_t)D * hq * dh);
-                VT_CUDA(cudaMemcpyAsync(as.norm, L.attn_norm, (size_t)D * 2,
-                                        cudaMemcpyDeviceToDevice, st));
-                rows_host.clear();
-                for (int blk = 0; blk < hq + 2 * hk; ++blk) {
-                    const __half* src;
-                    int head;
-                    if (blk < hq) {
-                        src = L.wq;
-                        head = as.h0 + blk;
-                    } else if (blk < hq + hk) {
-                        src = L.wk;
-                        head = as.kv0 + blk - hq;
-                    } else {
-                        src = L.wv;
-                        head = as.kv0 + blk - hq - hk;
-                    }
-                    for (int i = 0; i < dh / 2; ++i) {
-                        rows_host.push_back(src + ((size_t)head * dh + i) * D);
-                        rows_host.push_back(src + ((size_t)head * dh + i + dh / 2) * D);
-                    }
-                }
-                VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*),
-                                        cudaMemcpyHostToDevice, st));
-                VT_CUDA(launch_gather_rows(rows_dev, as.wqkv, (int)rows_host.size(), D, D, st));
-                VT_CUDA(cudaStreamSynchronize(st));  // rows_host / rows_dev are reused
-                VT_CUDA(cudaMemcpy2DAsync(as.wo, (size_t)hq * dh * 2, L.wo + (size_t)as.h0 * dh,
-                                          (size_t)H * dh * 2, (size_t)hq * dh * 2, D,
-                                          cudaMemcpyDeviceToDevice, st));
-            }
-            // ---------------------------------------------------------- FFN shard
             FfnShard& fs = p->ffn[(size_t)l * n + d];
             fs.c0 = cols[d].begin;
             fs.c1 = cols[d].end;
-            const int c = fs.c1 - fs.c0;
-            if (c > 0) {
-                const size_t bytes = align256((size_t)D * 2) + align256((size_t)2 * c * D * 2) +
-                                     align256((size_t)c * D * 2);
-                fs.base = A.get(bytes);
-                if (!fs.base) return bail(fail(VT_ERR_ALLOC, "shard allocation failed"));
-                Bump b{static_cast<uint8_t*>(fs.base)};
-                fs.norm = b.take<__half>(D);
-                fs.wgu = b.take<__half>((size_t)2 * c * D);
-                fs.wdt = b.take<__half>((size_t)c * D);
-                VT_CUDA(cudaMemcpyAsync(fs.norm, L.ffn_norm, (size_t)D * 2,
-                                        cudaMemcpyDeviceToDevice, st));
-                rows_host.clear();
-                for (int j = 0; j < c; ++j) {
-                    rows_host.push_back(L.w_gate + (size_t)(fs.c0 + j) * D);
-                    rows_host.push_back(L.w_up + (size_t)(fs.c0 + j) * D);
-                }
-                VT_CUDA(cudaMemcpyAsync(rows_dev, rows_host.data(), rows_host.size() * sizeof(void*),
-                                        cudaMemcpyHostToDevice, st));
-                VT_CUDA(launch_gather_rows(rows_dev, fs.wgu, (int)rows_host.size(), D, D, st));
-                VT_CUDA(cudaStreamSynchronize(st));
-                VT_CUDA(launch_transpose_f16(L.w_down + fs.c0, F, D, c, fs.wdt, D, st));
-            }
+            if ((r = slice_attn_fp16(p, l, d, rows_dev, st)) == VT_OK) r = slice_ffn_fp16(p, l, d, rows_dev, st);
         }
-    }
     A.put(rows_dev);
+    if (r != VT_OK) return bail(r);
 
     // ------------------------------------------------------------------ decode scratch
     p->dec.resize(n);
@@ -873,12 +874,13 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         const int hq = heads[d].end - heads[d].begin, hk = hq / g, c = cols[d].end - cols[d].begin;
         DecodeScratch& ds = p->dec[d];
         ds.ffn_grid = ffn_grid(c);
-        const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2;
+        const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2 + align256((size_t)std::max(c, 1) * 4);
         void* q;
         if ((r = owned_alloc(p, bytes, &q)) != VT_OK) return bail(r);
         Bump b{static_cast<uint8_t*>(q)};
         ds.q = b.take<float>((size_t)std::max(hq, 1) * dh);
         ds.attn = b.take<float>((size_t)std::max(hq, 1) * dh);
+        ds.u = b.take<float>((size_t)std::max(c, 1));
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
         p->max_hq = std::max(p->max_hq, hq);
         p->max_ld = std::max(p->max_ld, round_up8(c + cols[d].begin % 8));
@@ -926,7 +928,7 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
             t.kv0[d] = heads[d].begin / g;
             t.cols[d] = cols[d].end - cols[d].begin;
         }
-        p->tok_ok = token_plan(t, p->max_hq, &p->tok_plan, &p->tok_why);
+        p->tok_ok = p->tok_planned = token_plan(t, p->max_hq, &p->tok_plan, &p->tok_why);
         if (p->tok_ok) {
             const size_t bytes = 2 * align256((size_t)H * dh * 4) + 2 * align256((size_t)n * D * 4) +
                                  align256(token_state_floats(p->tok_plan.grid, g, dh) * 4) +
@@ -972,6 +974,8 @@ extern "C" vt_status vt_shard_weight_layout(const vt_partition* p, vt_shard sh, 
     const AttnShard& a = p->a(sh.layer, sh.device);
     const FfnShard& f = p->f(sh.layer, sh.device);
     const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, c = f.c1 - f.c0;
+    if (((which == 1 || which == 2) && a.bits != 16) || ((which == 4 || which == 5) && f.bits != 16))
+        return fail(VT_ERR_STATE, "tensor %d of the shard is block-quantized: read it with vt_shard_qweights_read", which);
     switch (which) {
         case 0: *rows = hq > 0; *stride = s.d_model; break;
         case 1: *rows = (int64_t)(hq + 2 * hk) * s.d_head; *stride = s.d_model; break;
@@ -1010,11 +1014,172 @@ extern "C" vt_status vt_shard_weights_read(const vt_partition* p, vt_shard sh, i
     return ok();
 }
 
+// ------------------------------------------------------------------ shard precision
+
+// Quantized matrix storage for `rows` x `k` at `bits` carved from a Bump.
+static QMatDev take_qmat(Bump& b, int rows, int k, int bits) {
+    QMatDev m;
+    m.rows = rows;
+    m.k = k;
+    m.nb = (k + kQBlock - 1) / kQBlock;
+    m.bits = bits;
+    m.row_bytes = (int64_t)m.nb * (bits == 8 ? 32 : 16);
+    m.codes = b.take<uint8_t>(qmat_code_bytes(rows, k, bits));
+    m.scales = b.take<__half>((size_t)rows * m.nb);
+    return m;
+}
+
+static size_t qmat_bytes(int rows, int k, int bits) {
+    return align256(qmat_code_bytes(rows, k, bits)) + align256(qmat_scale_bytes(rows, k));
+}
+
+static void update_token_kernel(vt_partition* p) {
+    bool quantized = false;
+    for (const AttnShard& a : p->attn) quantized |= a.bits != 16;
+    for (const FfnShard& f : p->ffn) quantized |= f.bits != 16;
+    p->tok_ok = p->tok_planned && !quantized;
+    if (p->tok_planned && quantized) p->tok_why = "a shard is block-quantized: the token runs on the per-shard kernels";
+}
+
+extern "C" vt_status vt_partition_set_precision(vt_partition* p, vt_shard sh, int32_t bits, vt_stream stream) {
+    VT_TRY(check_shard(p, sh));
+    if (bits != 16 && bits != 8 && bits != 4) return fail(VT_ERR_INVALID_ARG, "bits %d must be 16, 8 or 4", bits);
+    if (p->n_kv > 0) return fail(VT_ERR_STATE, "shard precisions are fixed while a KV cache of the partition exists");
+    cudaStream_t st = (cudaStream_t)stream;
+    const vt_shapes& s = p->m->s;
+    const int D = s.d_model, dh = s.d_head, l = sh.layer, d = sh.device;
+    Allocator& A = p->m->alloc;
+    const __half** rows_dev = nullptr;
+    auto table = [&]() -> const __half** {
+        if (!rows_dev) rows_dev = static_cast<const __half**>(A.get(gather_table_bytes(s)));
+        return rows_dev;
+    };
+    vt_status r = VT_OK;
+    if (sh.block == VT_BLOCK_ATTN) {
+        AttnShard& a = p->attn[(size_t)l * p->n_dev + d];
+        const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, K = hq * dh, rows = (hq + 2 * hk) * dh;
+        if (hq == 0 || bits == a.bits) {
+            // an empty shard stores nothing and stays fp16
+        } else {
+            if (a.bits != 16) {  // back to the fp16 slices first
+                VT_CUDA(cudaStreamSynchronize(st));
+                A.put(a.base);
+                a.base = nullptr;
+                if (!table()) return fail(VT_ERR_ALLOC, "allocating the gather table failed");
+                r = slice_attn_fp16(p, l, d, rows_dev, st);
+            }
+            if (r == VT_OK && bits != 16) {
+                void* nb = A.get(align256((size_t)D * 2) + qmat_bytes(rows, D, bits) + qmat_bytes(D, K, bits));
+                if (!nb) {
+                    r = fail(VT_ERR_ALLOC, "allocating the quantized shard failed");
+                } else {
+                    Bump b{static_cast<uint8_t*>(nb)};
+                    __half* norm = b.take<__half>(D);
+                    const QMatDev qkv = take_qmat(b, rows, D, bits), o = take_qmat(b, D, K, bits);
+                    cudaError_t e = cudaMemcpyAsync(norm, a.norm, (size_t)D * 2, cudaMemcpyDeviceToDevice, st);
+                    if (e == cudaSuccess) e = launch_quantize_rows(a.wqkv, D, qkv, st);
+                    if (e == cudaSuccess) e = launch_quantize_rows(a.wo, K, o, st);
+                    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+                    if (e != cudaSuccess) {
+                        A.put(nb);
+                        r = fail(VT_ERR_CUDA, "quantizing the shard failed: %s", cudaGetErrorString(e));
+                    } else {
+                        A.put(a.base);
+                        a.base = nb;
+                        a.norm = norm;
+                        a.wqkv = a.wo = nullptr;
+                        a.qkv = qkv;
+                        a.o = o;
+                        a.bits = bits;
+                    }
+                }
+            }
+        }
+    } else {
+        FfnShard& f = p->ffn[(size_t)l * p->n_dev + d];
+        const int c = f.c1 - f.c0;
+        if (c == 0 || bits == f.bits) {
+            // an empty shard stores nothing and stays fp16
+        } else {
+            if (f.bits != 16) {
+                VT_CUDA(cudaStreamSynchronize(st));
+                A.put(f.base);
+                f.base = nullptr;
+                if (!table()) return fail(VT_ERR_ALLOC, "allocating the gather table failed");
+                r = slice_ffn_fp16(p, l, d, rows_dev, st);
+            }
+            if (r == VT_OK && bits != 16) {
+                void* nb = A.get(align256((size_t)D * 2) + qmat_bytes(2 * c, D, bits) + qmat_bytes(D, c, bits));
+                if (!nb) {
+                    r = fail(VT_ERR_ALLOC, "allocating the quantized shard failed");
+                } else {
+                    Bump b{static_cast<uint8_t*>(nb)};
+                    __half* norm = b.take<__half>(D);
+                    const QMatDev gu = take_qmat(b, 2 * c, D, bits), dn = take_qmat(b, D, c, bits);
+                    cudaError_t e = cudaMemcpyAsync(norm, f.norm, (size_t)D * 2, cudaMemcpyDeviceToDevice, st);
+                    if (e == cudaSuccess) e = launch_quantize_rows(f.wgu, D, gu, st);
+                    // the down projection is quantized along the shard's columns: rows of Wd[:, c0:c1]
+                    if (e == cudaSuccess) e = launch_quantize_rows(p->m->layer[l].w_down + f.c0, s.d_ffn, dn, st);
+                    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+                    if (e != cudaSuccess) {
+                        A.put(nb);
+                        r = fail(VT_ERR_CUDA, "quantizing the shard failed: %s", cudaGetErrorString(e));
+                    } else {
+                        A.put(f.base);
+                        f.base = nb;
+                        f.norm = norm;
+                        f.wgu = f.wdt = nullptr;
+                        f.gu = gu;
+                        f.down = dn;
+                        f.bits = bits;
+                    }
+                }
+            }
+        }
+    }
+    if (rows_dev) A.put(rows_dev);
+    update_token_kernel(p);
+    if (r != VT_OK) return r;
+    return ok();
+}
+
+extern "C" int32_t vt_shard_precision(const vt_partition* p, vt_shard sh) {
+    if (check_shard(p, sh) != VT_OK) return 0;
+    return sh.block == VT_BLOCK_ATTN ? p->a(sh.layer, sh.device).bits : p->f(sh.layer, sh.device).bits;
+}
+
+extern "C" vt_status vt_shard_qweights_read(const vt_partition* p, vt_shard sh, int32_t which, int8_t* codes,
+                                            void* scales) {
+    VT_TRY(check_shard(p, sh));
+    const bool attn = which == 1 || which == 2, ffn = which == 4 || which == 5;
+    if (!attn && !ffn) return fail(VT_ERR_INVALID_ARG, "tensor %d has no quantized form", which);
+    if ((attn && sh.block != VT_BLOCK_ATTN) || (ffn && sh.block != VT_BLOCK_FFN))
+        return fail(VT_ERR_INVALID_ARG, "tensor %d does not belong to block %d", which, sh.block);
+    const QMatDev* m = nullptr;
+    if (attn) {
+        const AttnShard& a = p->a(sh.layer, sh.device);
+        if (a.bits == 16 || a.h1 == a.h0) return fail(VT_ERR_STATE, "the shard is not block-quantized");
+        m = which == 1 ? &a.qkv : &a.o;
+    } else {
+        const FfnShard& f = p->f(sh.layer, sh.device);
+        if (f.bits == 16 || f.c1 == f.c0) return fail(VT_ERR_STATE, "the shard is not block-quantized");
+        m = which == 4 ? &f.gu : &f.down;
+    }
+    if (!codes || !scales) return fail(VT_ERR_INVALID_ARG, "codes and scales must not be NULL");
+    std::vector<uint8_t> raw(qmat_code_bytes(m->rows, m->k, m->bits));
+    VT_CUDA(cudaDeviceSynchronize());
+    VT_CUDA(cudaMemcpy(raw.data(), m->codes, raw.size(), cudaMemcpyDeviceToHost));
+    VT_CUDA(cudaMemcpy(scales, m->scales, qmat_scale_bytes(m->rows, m->k), cudaMemcpyDeviceToHost));
+    unpack_qcodes(raw.data(), m->rows, m->k, m->bits, codes);
+    return ok();
+}
+
 // ================================================================== KV cache
 
 extern "C" void vt_kv_destroy(vt_kv* kv) {
     if (!kv) return;
     cudaDeviceSynchronize();
+    --kv->p->n_kv;
     Allocator* A = kv->alloc();
     for (void* b : kv->buf) A->put(b);
     A->put(kv->len);
@@ -1032,6 +1197,7 @@ extern "C" vt_status vt_kv_create(const vt_partition* p, int32_t cap, vt_stream 
     vt_kv* kv = new vt_kv();
     kv->p = p;
     kv->cap = cap;
+    ++p->n_kv;
     kv->buf.assign((size_t)s.n_layers * p->n_dev, nullptr);
     Allocator* A = kv->alloc();
     for (int l = 0; l < s.n_layers; ++l)
@@ -1195,6 +1361,80 @@ extern "C" vt_status vt_kv_write_raw(vt_kv* kv, int32_t l, int32_t d, int32_t n_
 
 // ================================================================== shard compute
 
+// QKV projection of ATTN shard (l, d) with RoPE and the K/V append at the layer's length: the
+// fp16 GEMV or, for a block-quantized shard, the dequantizing one.  q: [hq][dh] rotated queries.
+// indep: the caller guarantees that `x` was written at least two kernel launches before (the
+// fp16 GEMV may then read it before griddepcontrol.wait).
+static cudaError_t attn_qkv(const vt_partition* p, int l, int d, const __half* x, vt_kv* kv, float* q,
+                            cudaStream_t st, int indep) {
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(l, d);
+    const int hq = a.h1 - a.h0, hk = a.kv1 - a.kv0, dh = s.d_head, D = s.d_model;
+    if (a.bits != 16) {
+        QGemvArgs g{};
+        g.w = a.qkv;
+        g.x = x;
+        g.gain = a.norm;
+        g.eps = s.rms_eps;
+        g.out = q;
+        g.kcache = kv->k(l, d);
+        g.vcache = kv->v(l, d);
+        g.cap = kv->cap;
+        g.len = kv->len + l;
+        g.rope = p->m->rope;
+        g.dh = dh;
+        g.hq = hq;
+        g.hk = hk;
+        g.status = kv->status;
+        return launch_gemv_q(kEpiQkvRope, g, st);
+    }
+    GemvArgs g{};
+    g.w = a.wqkv;
+    g.row_stride = D;
+    g.rows = (hq + 2 * hk) * dh;
+    g.k = D;
+    g.x = x;
+    g.gain = a.norm;
+    g.eps = s.rms_eps;
+    g.out = q;
+    g.kcache = kv->k(l, d);
+    g.vcache = kv->v(l, d);
+    g.cap = kv->cap;
+    g.len = kv->len + l;
+    g.rope = p->m->rope;
+    g.dh = dh;
+    g.hq = hq;
+    g.hk = hk;
+    g.status = kv->status;
+    g.indep = indep;
+    return launch_gemv(kEpiQkvRope, g, st);
+}
+
+// O projection of ATTN shard (l, d): out [D] = Wo_s . attn (fp32), fp16 or block-quantized.
+static cudaError_t attn_o(const vt_partition* p, int l, int d, const float* attn, float* out, uint32_t* status,
+                          cudaStream_t st) {
+    const vt_shapes& s = p->m->s;
+    const AttnShard& a = p->a(l, d);
+    const int hq = a.h1 - a.h0, dh = s.d_head, D = s.d_model;
+    if (a.bits != 16) {
+        QGemvArgs o{};
+        o.w = a.o;
+        o.vin = attn;
+        o.out = out;
+        o.status = status;
+        return launch_gemv_q(kEpiPlain, o, st);
+    }
+    GemvArgs o{};
+    o.w = a.wo;
+    o.row_stride = (int64_t)hq * dh;
+    o.rows = D;
+    o.k = hq * dh;
+    o.vin = attn;
+    o.out = out;
+    o.status = status;
+    return launch_gemv(kEpiPlain, o, st);
+}
+
 // indep: the caller guarantees that `x` was written at least two kernel launches before this
 // shard's first kernel, so that kernel may read it before griddepcontrol.wait (see k_gemv).
 static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* x, vt_kv* kv,
@@ -1207,26 +1447,7 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
         VT_CUDA(launch_fill_zero_f32(out, D, st));
         return VT_OK;
     }
-    GemvArgs g{};
-    g.w = a.wqkv;
-    g.row_stride = D;
-    g.rows = (hq + 2 * hk) * dh;
-    g.k = D;
-    g.x = x;
-    g.gain = a.norm;
-    g.eps = s.rms_eps;
-    g.out = ds.q;
-    g.kcache = kv->k(l, d);
-    g.vcache = kv->v(l, d);
-    g.cap = kv->cap;
-    g.len = kv->len + l;
-    g.rope = p->m->rope;
-    g.dh = dh;
-    g.hq = hq;
-    g.hk = hk;
-    g.status = kv->status;
-    g.indep = indep;
-    VT_CUDA(launch_gemv(kEpiQkvRope, g, st));
+    VT_CUDA(attn_qkv(p, l, d, x, kv, ds.q, st, indep));
 
     AttnDecodeArgs t{};
     t.q = ds.q;
@@ -1243,16 +1464,7 @@ static vt_status decode_attn(const vt_partition* p, int l, int d, const __half* 
     t.out = ds.attn;
     t.status = kv->status;
     VT_CUDA(launch_attn_decode(t, st));
-
-    GemvArgs o{};
-    o.w = a.wo;
-    o.row_stride = (int64_t)hq * dh;
-    o.rows = D;
-    o.k = hq * dh;
-    o.vin = ds.attn;
-    o.out = out;
-    o.status = kv->status;
-    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    VT_CUDA(attn_o(p, l, d, ds.attn, out, kv->status, st));
     return VT_OK;
 }
 
@@ -1264,6 +1476,25 @@ static vt_status decode_ffn(const vt_partition* p, int l, int d, const __half* x
     const FfnShard& f = p->f(l, d);
     const DecodeScratch& ds = p->dec[d];
     const int c = f.c1 - f.c0, D = s.d_model;
+    if (f.bits != 16 && c > 0) {
+        // block-quantized shard: gate/up rows with the SwiGLU epilogue, then the down columns (the
+        // partial is written, not added)
+        QGemvArgs g{};
+        g.w = f.gu;
+        g.x = x;
+        g.gain = f.norm;
+        g.eps = s.rms_eps;
+        g.out = ds.u;
+        g.status = p->status;
+        VT_CUDA(launch_gemv_q(kEpiSwiglu, g, st));
+        QGemvArgs o{};
+        o.w = f.down;
+        o.vin = ds.u;
+        o.out = out;
+        o.status = p->status;
+        VT_CUDA(launch_gemv_q(kEpiPlain, o, st));
+        return VT_OK;
+    }
     if (zero_first) VT_CUDA(launch_fill_zero_f32(out, D, st));
     if (c == 0) return VT_OK;
     FfnDecodeArgs g{};
@@ -1333,25 +1564,7 @@ extern "C" vt_status vt_decode_step_static(const vt_partition* p, vt_shard sh, c
     float* q = reinterpret_cast<float*>(b + lay.q);
     float* attn = reinterpret_cast<float*>(b + lay.attn);
 
-    GemvArgs g{};
-    g.w = a.wqkv;
-    g.row_stride = D;
-    g.rows = (hq + 2 * hk) * dh;
-    g.k = D;
-    g.x = static_cast<const __half*>(x);
-    g.gain = a.norm;
-    g.eps = s.rms_eps;
-    g.out = q;
-    g.kcache = kv->k(l, d);
-    g.vcache = kv->v(l, d);
-    g.cap = kv->cap;
-    g.len = kv->len + l;
-    g.rope = p->m->rope;
-    g.dh = dh;
-    g.hq = hq;
-    g.hk = hk;
-    g.status = kv->status;
-    VT_CUDA(launch_gemv(kEpiQkvRope, g, st));
+    VT_CUDA(attn_qkv(p, l, d, static_cast<const __half*>(x), kv, q, st, 0));
 
     StaticAttnArgs t{};
     t.q = q;
@@ -1370,15 +1583,7 @@ extern "C" vt_status vt_decode_step_static(const vt_partition* p, vt_shard sh, c
     t.out = attn;
     VT_CUDA(launch_attn_decode_static(t, st));
 
-    GemvArgs o{};
-    o.w = a.wo;
-    o.row_stride = (int64_t)hq * dh;
-    o.rows = D;
-    o.k = hq * dh;
-    o.vin = attn;
-    o.out = out;
-    o.status = kv->status;
-    VT_CUDA(launch_gemv(kEpiPlain, o, st));
+    VT_CUDA(attn_o(p, l, d, attn, out, kv->status, st));
     return ok();
 }
 
@@ -1461,6 +1666,9 @@ static void ffn_args(const vt_partition* p, vt_shard sh, const __half* x, int n,
 static vt_status prefill_shard(const vt_partition* p, vt_shard sh, const __half* x, int n, vt_kv* kv,
                                float* out, int row_offset, cudaStream_t st, bool xhat_ready = false) {
     const vt_shapes& s = p->m->s;
+    if ((sh.block == VT_BLOCK_ATTN ? p->a(sh.layer, sh.device).bits : p->f(sh.layer, sh.device).bits) != 16)
+        return fail(VT_ERR_STATE, "prefill runs on fp16 shards; shard (layer %d, device %d, block %d) is block-quantized",
+                    sh.layer, sh.device, sh.block);
     const int D = s.d_model;
     std::string err;
     if (sh.block == VT_BLOCK_ATTN) {
@@ -1644,6 +1852,10 @@ extern "C" vt_status vt_prefill_tokens(const vt_partition* p, vt_kv* kv, const v
         if ((int64_t)kv->h_len[l] + n > kv->cap)
             return fail(VT_ERR_KV_CAPACITY, "layer %d holds %d of %d positions; %d more do not fit", l,
                         kv->h_len[l], kv->cap, n);
+    for (const AttnShard& a : p->attn)
+        if (a.bits != 16 && a.h1 > a.h0) return fail(VT_ERR_STATE, "prefill runs on fp16 shards; an ATTN shard is block-quantized");
+    for (const FfnShard& f : p->ffn)
+        if (f.bits != 16 && f.c1 > f.c0) return fail(VT_ERR_STATE, "prefill runs on fp16 shards; an FFN shard is block-quantized");
     cudaStream_t st = (cudaStream_t)stream;
     const int D = s.d_model, nd = p->n_dev;
     for (int r0 = 0; r0 < n; r0 += kPrefillChunk) {

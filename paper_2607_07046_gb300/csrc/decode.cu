@@ -67,14 +67,6 @@ static cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 
 static __host__ __device__ __forceinline__ int round_up8(int k) { return (k + 7) & ~7; }
 
-__device__ __forceinline__ uint4 ldg_stream(const void* p) {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
-
 // Chunks per lane for a row of `k` columns: the choice with the best use of the 8 warps' lanes.
 int gemv_cpl(int k) {
     const int nch = round_up8(k) / 8;

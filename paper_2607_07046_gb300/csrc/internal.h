@@ -133,6 +133,7 @@ cudaError_t launch_gather_rows(const __half* const* src_rows, __half* dst, int n
 // One-time per-process setup of kernel attributes (dynamic shared-memory limits).
 cudaError_t init_decode_kernels();
 cudaError_t init_prefill_kernels();
+cudaError_t init_quant_kernels();
 
 // ------------------------------------------------------------------ prefill path (prefill.cu)
 struct PrefillAttnArgs {
@@ -192,6 +193,53 @@ cudaError_t launch_combine_norm(const CombineArgs& a, int rows, int d, const __h
                                 int split, cudaStream_t st);
 cudaError_t launch_rmsnorm_rows(const __half* x, const __half* gain, float eps, int rows, int d, __half* y,
                                 int split, cudaStream_t st);
+
+// ------------------------------------------------------------------ block-quantized shard weights (quant.cu)
+// A matrix [rows][k] stored as codes of 8 or 4 bits with one fp16 scale per block of kQBlock
+// weights along k (the dequantized weight is q * d).  Device layout (written by k_quantize_rows):
+//   codes: row r at codes + r * row_bytes, row_bytes = nb * 32 (8-bit) or nb * 16 (4-bit),
+//          nb = ceil(k / 32); biased codes u = q + 128 (8-bit, one byte each) or u = q + 8 (4-bit:
+//          each 32-bit word holds 8 codes, byte i = code i in its low nibble and code i + 4 in its
+//          high nibble); positions k .. nb * 32 - 1 hold the code of 0;
+//   scales: [rows][nb] fp16.
+constexpr int kQBlock = 32;
+
+struct QMatDev {
+    uint8_t* codes = nullptr;
+    __half* scales = nullptr;
+    int rows = 0, k = 0, nb = 0, bits = 16;
+    int64_t row_bytes = 0;
+};
+// Quantizes device fp16 rows (row r at w + r * ld, m.k values) into m's codes and scales, in the
+// layout above, with the decisions of vt_quantize_rows (bit-identical codes and scales).
+cudaError_t launch_quantize_rows(const __half* w, int64_t ld, const QMatDev& m, cudaStream_t st);
+
+// Host side: bytes of the codes and of the scales of a [rows][k] matrix at `bits`.
+size_t qmat_code_bytes(int64_t rows, int64_t k, int bits);
+size_t qmat_scale_bytes(int64_t rows, int64_t k);
+// The inverse of the packing for the codes: canonical int8 codes [rows][k].
+void unpack_qcodes(const uint8_t* codes, int64_t rows, int64_t k, int bits, int8_t* q);
+// Host quantizer shared with vt_quantize_rows: codes q [rows][k] (int8) and fp16 scales [rows][nb].
+void quantize_rows_host(const __half* w, int64_t rows, int64_t k, int bits, int block, int8_t* q, __half* scales);
+
+struct QGemvArgs {
+    QMatDev w;
+    // input: RMSNorm(x) * gain (x fp16 [k]) when x is set, else the fp32 vector vin [k]
+    const __half* x;
+    const __half* gain;
+    float eps;
+    const float* vin;
+    // epilogues as GemvArgs: plain out[rows]; SwiGLU out[rows / 2]; QKV: q to out, K / V appended
+    float* out;
+    __half* kcache;
+    __half* vcache;
+    int cap;
+    const int32_t* len;
+    const float2* rope;
+    int dh, hq, hk;
+    uint32_t* status;
+};
+cudaError_t launch_gemv_q(int epi, const QGemvArgs& a, cudaStream_t st);
 
 // ------------------------------------------------------------------ static-scratch decode attention
 // (static_scratch.cu) split-K decode attention whose scratch is one file-scope __device__ array.

@@ -14,8 +14,11 @@ class Stack:
 
     def __init__(self, shapes: vt.vt_shapes, layer_fn: Callable[[int], Dict[str, np.ndarray]],
                  head_ranges: Sequence[Tuple[int, int]], ffn_ranges: Sequence[Tuple[int, int]],
-                 capacity: int, embed: Optional[np.ndarray] = None, stream=None, windows=None):
-        """windows: None, one sliding attention window for every layer, or one per layer (0: none)."""
+                 capacity: int, embed: Optional[np.ndarray] = None, stream=None, windows=None,
+                 precision=None):
+        """windows: None, one sliding attention window for every layer, or one per layer (0: none).
+        precision: None, or a function (layer, device, block) -> bits (16, 8 or 4) applied to every
+        shard before the KV cache is created."""
         self.shapes = shapes
         self.model = self.part = self.kv = 0
         self.model = vt.vt_model_create(shapes, None, None, stream)
@@ -28,6 +31,13 @@ class Stack:
             for l, w in enumerate(ws):
                 vt.vt_model_set_window(self.model, l, w)
         self.part = vt.vt_partition_create(self.model, head_ranges, ffn_ranges, stream)
+        if precision is not None:
+            for l in range(shapes.n_layers):
+                for d in range(len(head_ranges)):
+                    for blk in (vt.VT_BLOCK_ATTN, vt.VT_BLOCK_FFN):
+                        bits = precision(l, d, blk)
+                        if bits != 16:
+                            vt.vt_partition_set_precision(self.part, (l, d, blk), bits, stream)
         self.kv = vt.vt_kv_create(self.part, capacity, stream) if capacity > 0 else 0
         self.head_ranges = list(head_ranges)
         self.ffn_ranges = list(ffn_ranges)

@@ -139,6 +139,9 @@ def lib() -> ctypes.CDLL:
             "vt_decode_token_sharded": (S, [_P, _P, _P, _P, _P]),
             "vt_decode_token_fused_available": (_I32, [_P, ctypes.POINTER(ctypes.c_char_p)]),
             "vt_prefill_tokens": (S, [_P, _P, _P, _I32, _P, _P]),
+            "vt_partition_set_precision": (S, [_P, vt_shard, _I32, _P]),
+            "vt_shard_precision": (_I32, [_P, vt_shard]),
+            "vt_shard_qweights_read": (S, [_P, vt_shard, _I32, _P, _P]),
             "vt_token_partials_read": (S, [_P, _I32, _P]),
         }
         for name, (res, args) in sig.items():
@@ -391,6 +394,23 @@ def vt_shard_weights_read(part: int, shard: Tuple[int, int, int], which: int) ->
                                        ctypes.byref(size)))
     assert size.value == out.nbytes
     return out
+
+
+def vt_partition_set_precision(part: int, shard: Tuple[int, int, int], bits: int, stream=None) -> None:
+    """Store one shard at 16 (fp16), 8 or 4 bits (block-quantized, blocks of 32, fp16 scales)."""
+    _check(lib().vt_partition_set_precision(part, vt_shard(*shard), int(bits), _stream(stream)))
+
+
+def vt_shard_precision(part: int, shard: Tuple[int, int, int]) -> int:
+    return int(lib().vt_shard_precision(part, vt_shard(*shard)))
+
+
+def vt_shard_qweights_read(part: int, shard: Tuple[int, int, int], which: int, rows: int, k: int):
+    """Codes int8 [rows, k] and fp16 scales [rows, ceil(k / 32)] of a quantized shard tensor."""
+    q = np.empty((rows, k), np.int8)
+    sc = np.empty((rows, (k + 31) // 32), np.float16)
+    _check(lib().vt_shard_qweights_read(part, vt_shard(*shard), int(which), q.ctypes.data, sc.ctypes.data))
+    return q, sc
 
 
 # ------------------------------------------------------------------ KV cache
