@@ -271,6 +271,23 @@ VT_API vt_status vt_embed(const vt_model* model, const int32_t* ids, int32_t n, 
 VT_API vt_status vt_partition_create(vt_model* model, int32_t n_devices, const vt_range* head_ranges,
                               const vt_range* ffn_col_ranges, vt_stream stream,
                               vt_partition** out);
+/* vt_partition_create_layers (Section 4.2.1: the plan is made layer by layer, ATTN and FFN as
+ * separate layers, each run by one device (MP) or split among devices (TP); Section 4.3.1: shards
+ * are pruned, the same number from every layer, to fit a shrinking memory budget): a partition
+ * with its own ranges per layer.  heads, cols: [n_layers][n_devices] ranges (layer-major); each
+ * layer follows vt_partition's rules (a block on one device with empty ranges elsewhere is MP).
+ * flags VT_PARTITION_PRUNE: a layer's ranges may leave heads / columns uncovered; those are pruned
+ * (their terms are omitted from the layer, as a dropped shard's would be) and an empty range may
+ * sit anywhere.  Each (layer, block, device) shard gets its own allocation, as in vt_partition.
+ * The fused decode kernel takes one partition for every layer: vt_decode_token runs a per-layer or
+ * pruned partition on the per-shard kernels.  vt_partition_validate_layers checks the same rules
+ * on the host.  Errors: as vt_partition_create; VT_ERR_INVALID_ARG for unknown flags. */
+#define VT_PARTITION_PRUNE 1u
+VT_API vt_status vt_partition_create_layers(vt_model* model, int32_t n_devices, const vt_range* head_ranges,
+                                            const vt_range* ffn_col_ranges, uint32_t flags, vt_stream stream,
+                                            vt_partition** out);
+VT_API vt_status vt_partition_validate_layers(const vt_shapes* shapes, int32_t n_devices, const vt_range* head_ranges,
+                                              const vt_range* ffn_col_ranges, uint32_t flags);
 /* Library plumbing: the partition's device count; its device status word (VT_DEV_* bits of
  * kernels that have no KV cache; synchronizes the device; clear != 0 resets it and re-arms the
  * fused decode kernel's grid barrier); destruction (the model must still exist). */
@@ -418,6 +435,31 @@ VT_API vt_status vt_prefill(const vt_partition* part, vt_shard shard, const void
  *   1 <= n <= VT_MAX_DEVICES. */
 VT_API vt_status vt_combine(const float* const* partials, int32_t n, int32_t rows, int32_t d,
                      const void* residual, void* out, vt_stream stream);
+
+/* ---------------------------------------------------------------- communication scaling -------
+ * Section 4.3.2: the activations sent between devices are lowered to INT8 or INT4 when the link
+ * is too slow; under tensor parallelism those are the shard partials on their way to the main
+ * device.  Format (the library's reading): blocks of 32 values, fp16 scale d = fp16(amax / qmax)
+ * (qmax 127 or 7) and codes round-half-even(x / d) clamped to [-qmax, qmax], decisions in fp32;
+ * codes stored as one int8 per value (8 bits) or two per byte (4 bits: value 2i in the low nibble,
+ * 2i + 1 in the high nibble, each stored as q + 8).
+ * vt_partial_code_bytes: bytes of the codes of `count` values (0 for bad arguments).
+ * vt_quantize_partial: device fp32 partial [count] -> device codes and fp16 scales
+ *   [ceil(count / 32)] (the partial is not modified).
+ * vt_combine_q: out[e] = fp16(residual[e] + sum_{s=0}^{n-1} q_s[e] d_s[e / 32]) summed in fp32 in
+ *   shard order; codes / scales: host arrays of n device pointers; residual nullable; out may
+ *   alias residual.
+ * vt_partition_set_comm_bits: device `device` (or every device when -1) sends its partials at
+ *   `bits` (16: fp32, the default; 8; 4) in the whole-token path: each such partial is quantized
+ *   as its shard finishes and the combine adds the dequantized values.  vt_decode_token then runs
+ *   the per-shard kernels.  May change between tokens.
+ * Errors: VT_ERR_INVALID_ARG for NULL pointers, bad counts, devices or bits. */
+VT_API size_t vt_partial_code_bytes(int64_t count, int32_t bits);
+VT_API vt_status vt_quantize_partial(const float* partial, int64_t count, int32_t bits, void* codes, void* scales,
+                                     vt_stream stream);
+VT_API vt_status vt_combine_q(const void* const* codes, const void* const* scales, int32_t n, int64_t count,
+                              int32_t bits, const void* residual, void* out, vt_stream stream);
+VT_API vt_status vt_partition_set_comm_bits(vt_partition* part, int32_t device, int32_t bits);
 
 /* ---------------------------------------------------------------- whole stack ------------------
  * vt_decode_token: one decode token through every layer (Voltron Section 2.1, decode phase; the

@@ -185,6 +185,9 @@ struct vt_partition {
     std::vector<void*> owned;  // every allocation besides the shard bases
     bool counted = false;      // counted in the model's n_partitions
     mutable int n_kv = 0;      // live KV caches of the partition (precisions are fixed while any exists)
+    std::vector<int> comm_bits;   // per device: precision of its partials on the way to the combine (16: fp32)
+    uint8_t* pcodes = nullptr;    // [n_dev][D] quantized partials of the whole-token path
+    __half* pscales = nullptr;    // [n_dev][ceil(D / 32)]
     uint32_t* status = nullptr;
     // whole-stack buffers
     float* dpart = nullptr;     // [n_dev][D] decode partials (kept zero between blocks)
@@ -255,25 +258,27 @@ extern "C" vt_status vt_shapes_validate(const vt_shapes* s) {
     return ok();
 }
 
-static vt_status check_ranges(const vt_range* r, int n, int total, int align, const char* what) {
+// allow_gaps: heads / columns left uncovered are pruned (Section 4.3.1, shard-wise pruning).
+static vt_status check_ranges(const vt_range* r, int n, int total, int align, const char* what, bool allow_gaps = false) {
     int expect = 0;
     for (int d = 0; d < n; ++d) {
         if (r[d].begin < 0 || r[d].end > total || r[d].begin > r[d].end)
             return fail(VT_ERR_PARTITION_RANGE, "%s range %d [%d, %d) is not inside [0, %d)", what, d,
                         r[d].begin, r[d].end, total);
+        if (allow_gaps && r[d].begin == r[d].end) continue;  // a pruned device: its position does not matter
         if (r[d].begin < expect)
             return fail(VT_ERR_PARTITION_OVERLAP, "%s range %d starts at %d, before %d", what, d,
                         r[d].begin, expect);
-        if (r[d].begin > expect)
+        if (r[d].begin > expect && !allow_gaps)
             return fail(VT_ERR_PARTITION_GAP, "%s range %d starts at %d, leaving [%d, %d) unassigned",
                         what, d, r[d].begin, expect, r[d].begin);
         if (align > 1 && (r[d].begin % align != 0 || r[d].end % align != 0))
             return fail(VT_ERR_PARTITION_GQA,
                         "%s range %d [%d, %d) does not align to KV groups of %d heads", what, d,
                         r[d].begin, r[d].end, align);
-        expect = r[d].end;
+        if (r[d].end > r[d].begin || !allow_gaps) expect = r[d].end;  // a pruned layout may place empty ranges anywhere
     }
-    if (expect != total)
+    if (expect != total && !allow_gaps)
         return fail(VT_ERR_PARTITION_GAP, "%s ranges cover [0, %d) of [0, %d)", what, expect, total);
     return VT_OK;
 }
@@ -286,6 +291,24 @@ extern "C" vt_status vt_partition_validate(const vt_shapes* s, int32_t n, const 
     if (!heads || !cols) return fail(VT_ERR_INVALID_ARG, "range arrays must not be NULL");
     VT_TRY(check_ranges(heads, n, s->n_heads, s->n_heads / s->n_kv_heads, "head"));
     VT_TRY(check_ranges(cols, n, s->d_ffn, 1, "ffn column"));
+    return ok();
+}
+
+extern "C" vt_status vt_partition_validate_layers(const vt_shapes* s, int32_t n, const vt_range* heads,
+                                                  const vt_range* cols, uint32_t flags) {
+    VT_TRY(vt_shapes_validate(s));
+    if (n < 1 || n > VT_MAX_DEVICES)
+        return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
+    if (!heads || !cols) return fail(VT_ERR_INVALID_ARG, "range arrays must not be NULL");
+    if (flags & ~VT_PARTITION_PRUNE) return fail(VT_ERR_INVALID_ARG, "unknown partition flags 0x%x", flags);
+    const bool gaps = (flags & VT_PARTITION_PRUNE) != 0;
+    for (int l = 0; l < s->n_layers; ++l) {
+        char what[64];
+        snprintf(what, sizeof what, "layer %d head", l);
+        VT_TRY(check_ranges(heads + (size_t)l * n, n, s->n_heads, s->n_heads / s->n_kv_heads, what, gaps));
+        snprintf(what, sizeof what, "layer %d ffn column", l);
+        VT_TRY(check_ranges(cols + (size_t)l * n, n, s->d_ffn, 1, what, gaps));
+    }
     return ok();
 }
 
@@ -819,12 +842,12 @@ static vt_status slice_ffn_fp16(vt_partition* p, int l, int d, const __half** ro
     return VT_OK;
 }
 
-extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range* heads,
-                                         const vt_range* cols, vt_stream stream,
-                                         vt_partition** out) {
+// heads / cols: [n_layers][n] ranges (per-layer partition table).
+static vt_status partition_create(vt_model* m, int32_t n, const vt_range* heads, const vt_range* cols, uint32_t flags,
+                                  vt_stream stream, vt_partition** out) {
     if (!out || !m) return fail(VT_ERR_INVALID_ARG, "NULL argument");
     *out = nullptr;
-    VT_TRY(vt_partition_validate(&m->s, n, heads, cols));
+    VT_TRY(vt_partition_validate_layers(&m->s, n, heads, cols, flags));
     for (int l = 0; l < m->s.n_layers; ++l)
         if (!m->loaded[l]) return fail(VT_ERR_STATE, "layer %d weights were never loaded", l);
     cudaStream_t st = (cudaStream_t)stream;
@@ -836,8 +859,8 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     p->n_dev = n;
     p->counted = true;
     ++m->n_partitions;
-    p->heads.assign(heads, heads + n);
-    p->cols.assign(cols, cols + n);
+    p->heads.assign(heads, heads + (size_t)m->s.n_layers * n);
+    p->cols.assign(cols, cols + (size_t)m->s.n_layers * n);
     p->attn.resize((size_t)s.n_layers * n);
     p->ffn.resize((size_t)s.n_layers * n);
     Allocator& A = m->alloc;
@@ -856,13 +879,13 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     for (int l = 0; l < s.n_layers && r == VT_OK; ++l)
         for (int d = 0; d < n && r == VT_OK; ++d) {
             AttnShard& as = p->attn[(size_t)l * n + d];
-            as.h0 = heads[d].begin;
-            as.h1 = heads[d].end;
+            as.h0 = heads[(size_t)l * n + d].begin;
+            as.h1 = heads[(size_t)l * n + d].end;
             as.kv0 = as.h0 / g;
             as.kv1 = as.h1 / g;
             FfnShard& fs = p->ffn[(size_t)l * n + d];
-            fs.c0 = cols[d].begin;
-            fs.c1 = cols[d].end;
+            fs.c0 = cols[(size_t)l * n + d].begin;
+            fs.c1 = cols[(size_t)l * n + d].end;
             if ((r = slice_attn_fp16(p, l, d, rows_dev, st)) == VT_OK) r = slice_ffn_fp16(p, l, d, rows_dev, st);
         }
     A.put(rows_dev);
@@ -871,7 +894,14 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     // ------------------------------------------------------------------ decode scratch
     p->dec.resize(n);
     for (int d = 0; d < n; ++d) {
-        const int hq = heads[d].end - heads[d].begin, hk = hq / g, c = cols[d].end - cols[d].begin;
+        // sized for this device's largest shard over the layers
+        int hq = 0, c = 0;
+        for (int l = 0; l < s.n_layers; ++l) {
+            hq = std::max(hq, p->a(l, d).h1 - p->a(l, d).h0);
+            c = std::max(c, p->f(l, d).c1 - p->f(l, d).c0);
+            p->max_ld = std::max(p->max_ld, round_up8(p->f(l, d).c1 - p->f(l, d).c0 + p->f(l, d).c0 % 8));
+        }
+        const int hk = hq / g;
         DecodeScratch& ds = p->dec[d];
         ds.ffn_grid = ffn_grid(c);
         const size_t bytes = align256((size_t)std::max(hq, 1) * dh * 4) * 2 + align256((size_t)std::max(c, 1) * 4);
@@ -883,7 +913,6 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         ds.u = b.take<float>((size_t)std::max(c, 1));
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
         p->max_hq = std::max(p->max_hq, hq);
-        p->max_ld = std::max(p->max_ld, round_up8(c + cols[d].begin % 8));
         (void)hk;
     }
     // ------------------------------------------------------------------ stack + prefill scratch
@@ -908,6 +937,16 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
         p->p_u = b.take<__half>((size_t)n * p->u_slot);
         VT_CUDA(cudaMemsetAsync(q, 0, bytes, st));
     }
+    // ------------------------------------------------------------------ quantized partials (communication scaling)
+    {
+        p->comm_bits.assign(n, 16);
+        const size_t nbq = (size_t)(D + kQBlock - 1) / kQBlock;
+        void* q;
+        if ((r = owned_alloc(p, align256((size_t)n * D) + align256((size_t)n * nbq * 2), &q)) != VT_OK) return bail(r);
+        Bump b{static_cast<uint8_t*>(q)};
+        p->pcodes = b.take<uint8_t>((size_t)n * D);
+        p->pscales = b.take<__half>((size_t)n * nbq);
+    }
     // ------------------------------------------------------------------ decode-token kernel
     {
         TokArgs& t = p->tok_base;
@@ -928,7 +967,19 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
             t.kv0[d] = heads[d].begin / g;
             t.cols[d] = cols[d].end - cols[d].begin;
         }
-        p->tok_ok = p->tok_planned = token_plan(t, p->max_hq, &p->tok_plan, &p->tok_why);
+        // the fused kernel takes one partition for every layer, covering every head and column
+        bool uniform = (flags & VT_PARTITION_PRUNE) == 0;
+        for (int l = 1; l < s.n_layers && uniform; ++l)
+            for (int d = 0; d < n; ++d)
+                uniform &= heads[(size_t)l * n + d].begin == heads[d].begin && heads[(size_t)l * n + d].end == heads[d].end &&
+                           cols[(size_t)l * n + d].begin == cols[d].begin && cols[(size_t)l * n + d].end == cols[d].end;
+        if (uniform) {
+            p->tok_ok = p->tok_planned = token_plan(t, p->max_hq, &p->tok_plan, &p->tok_why);
+        } else {
+            p->tok_ok = p->tok_planned = false;
+            p->tok_why = (flags & VT_PARTITION_PRUNE) ? "a pruned partition runs on the per-shard kernels"
+                                                      : "a per-layer partition runs on the per-shard kernels";
+        }
         if (p->tok_ok) {
             const size_t bytes = 2 * align256((size_t)H * dh * 4) + 2 * align256((size_t)n * D * 4) +
                                  align256(token_state_floats(p->tok_plan.grid, g, dh) * 4) +
@@ -948,6 +999,25 @@ extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range*
     VT_CUDA(cudaStreamSynchronize(st));
     *out = p;
     return ok();
+}
+
+extern "C" vt_status vt_partition_create(vt_model* m, int32_t n, const vt_range* heads, const vt_range* cols,
+                                         vt_stream stream, vt_partition** out) {
+    if (!out || !m) return fail(VT_ERR_INVALID_ARG, "NULL argument");
+    *out = nullptr;
+    VT_TRY(vt_partition_validate(&m->s, n, heads, cols));
+    std::vector<vt_range> hl((size_t)m->s.n_layers * n), cl((size_t)m->s.n_layers * n);
+    for (int l = 0; l < m->s.n_layers; ++l)
+        for (int d = 0; d < n; ++d) {
+            hl[(size_t)l * n + d] = heads[d];
+            cl[(size_t)l * n + d] = cols[d];
+        }
+    return partition_create(m, n, hl.data(), cl.data(), 0, stream, out);
+}
+
+extern "C" vt_status vt_partition_create_layers(vt_model* m, int32_t n, const vt_range* heads, const vt_range* cols,
+                                                uint32_t flags, vt_stream stream, vt_partition** out) {
+    return partition_create(m, n, heads, cols, flags, stream, out);
 }
 
 extern "C" int32_t vt_partition_devices(const vt_partition* p) { return p ? p->n_dev : 0; }
@@ -1034,11 +1104,13 @@ static size_t qmat_bytes(int rows, int k, int bits) {
 }
 
 static void update_token_kernel(vt_partition* p) {
-    bool quantized = false;
+    bool quantized = false, comm = false;
     for (const AttnShard& a : p->attn) quantized |= a.bits != 16;
     for (const FfnShard& f : p->ffn) quantized |= f.bits != 16;
-    p->tok_ok = p->tok_planned && !quantized;
+    for (int b : p->comm_bits) comm |= b != 16;
+    p->tok_ok = p->tok_planned && !quantized && !comm;
     if (p->tok_planned && quantized) p->tok_why = "a shard is block-quantized: the token runs on the per-shard kernels";
+    else if (p->tok_planned && comm) p->tok_why = "partials are quantized for transmission: the token runs on the per-shard kernels";
 }
 
 extern "C" vt_status vt_partition_set_precision(vt_partition* p, vt_shard sh, int32_t bits, vt_stream stream) {
@@ -1794,6 +1866,79 @@ extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const voi
     return ok();
 }
 
+// The combine of one block of the whole-token path: the plain fp32 combine, or, when some
+// device's partials travel quantized (communication scaling), each such partial quantized as it
+// leaves its shard and the combine of the dequantized values (both clear the fp32 partials).
+static vt_status combine_block(const vt_partition* p, int l, vt_block block, const CombineArgs& c, cudaStream_t st) {
+    bool any = false;
+    for (int b : p->comm_bits) any |= b != 16;
+    if (!any) {
+        VT_CUDA(launch_combine(c, st));
+        return VT_OK;
+    }
+    const int D = p->m->s.d_model, nbq = (D + kQBlock - 1) / kQBlock;
+    CombineQArgs q{};
+    q.n = p->n_dev;
+    q.clear = 1;
+    q.count = D;
+    q.residual = c.residual;
+    q.out = c.out;
+    for (int d = 0; d < p->n_dev; ++d) {
+        const bool empty = block == VT_BLOCK_ATTN ? p->a(l, d).h1 == p->a(l, d).h0 : p->f(l, d).c1 == p->f(l, d).c0;
+        q.bits[d] = empty ? 16 : p->comm_bits[d];
+        q.fparts[d] = c.parts[d];
+        q.codes[d] = p->pcodes + (size_t)d * D;
+        q.scales[d] = p->pscales + (size_t)d * nbq;
+        if (q.bits[d] != 16)
+            VT_CUDA(launch_quantize_vec(c.parts[d], D, q.bits[d], p->pcodes + (size_t)d * D, p->pscales + (size_t)d * nbq, 1, st));
+    }
+    VT_CUDA(launch_combine_q(q, st));
+    return VT_OK;
+}
+
+extern "C" vt_status vt_partition_set_comm_bits(vt_partition* p, int32_t device, int32_t bits) {
+    if (!p) return fail(VT_ERR_INVALID_ARG, "partition is NULL");
+    if (device < -1 || device >= p->n_dev) return fail(VT_ERR_INVALID_ARG, "device %d out of range", device);
+    if (bits != 16 && bits != 8 && bits != 4) return fail(VT_ERR_INVALID_ARG, "bits %d must be 16, 8 or 4", bits);
+    for (int d = 0; d < p->n_dev; ++d)
+        if (device < 0 || d == device) p->comm_bits[d] = bits;
+    update_token_kernel(p);
+    return ok();
+}
+
+extern "C" size_t vt_partial_code_bytes(int64_t count, int32_t bits) {
+    if (count < 0 || (bits != 8 && bits != 4)) return 0;
+    return bits == 8 ? (size_t)count : (size_t)((count + 1) / 2);
+}
+
+extern "C" vt_status vt_quantize_partial(const float* partial, int64_t count, int32_t bits, void* codes, void* scales,
+                                         vt_stream stream) {
+    if (count < 0 || (bits != 8 && bits != 4)) return fail(VT_ERR_INVALID_ARG, "count %lld, bits %d", (long long)count, bits);
+    if (count > 0 && (!partial || !codes || !scales)) return fail(VT_ERR_INVALID_ARG, "NULL pointer");
+    VT_CUDA(launch_quantize_vec(const_cast<float*>(partial), count, bits, static_cast<uint8_t*>(codes),
+                                static_cast<__half*>(scales), 0, (cudaStream_t)stream));
+    return ok();
+}
+
+extern "C" vt_status vt_combine_q(const void* const* codes, const void* const* scales, int32_t n, int64_t count,
+                                  int32_t bits, const void* residual, void* out, vt_stream stream) {
+    if (!codes || !scales || !out || n < 1 || n > VT_MAX_DEVICES || count < 0 || (bits != 8 && bits != 4))
+        return fail(VT_ERR_INVALID_ARG, "bad vt_combine_q arguments");
+    CombineQArgs q{};
+    q.n = n;
+    q.count = count;
+    q.residual = static_cast<const __half*>(residual);
+    q.out = static_cast<__half*>(out);
+    for (int s = 0; s < n; ++s) {
+        if (!codes[s] || !scales[s]) return fail(VT_ERR_INVALID_ARG, "codes or scales of partial %d are NULL", s);
+        q.bits[s] = bits;
+        q.codes[s] = static_cast<const uint8_t*>(codes[s]);
+        q.scales[s] = static_cast<const __half*>(scales[s]);
+    }
+    VT_CUDA(launch_combine_q(q, (cudaStream_t)stream));
+    return ok();
+}
+
 extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
                                              vt_stream stream) {
     VT_TRY(check_token_args(p, kv, x_in, x_out));
@@ -1821,7 +1966,7 @@ extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, c
         }
         c.residual = cur;
         c.out = p->hbuf;
-        VT_CUDA(launch_combine(c, st));
+        VT_TRY(combine_block(p, l, VT_BLOCK_ATTN, c, st));
         launched = false;
         for (int d = 0; d < n; ++d) {
             const FfnShard& fs = p->f(l, d);
@@ -1832,7 +1977,7 @@ extern "C" vt_status vt_decode_token_sharded(const vt_partition* p, vt_kv* kv, c
         __half* dst = (l == s.n_layers - 1) ? static_cast<__half*>(x_out) : p->xbuf;
         c.residual = p->hbuf;
         c.out = dst;
-        VT_CUDA(launch_combine(c, st));
+        VT_TRY(combine_block(p, l, VT_BLOCK_FFN, c, st));
         cur = dst;
     }
     VT_CUDA(launch_kv_advance(kv->len, 0, s.n_layers, 1, kv->cap, kv->status, st));

@@ -241,6 +241,23 @@ struct QGemvArgs {
 };
 cudaError_t launch_gemv_q(int epi, const QGemvArgs& a, cudaStream_t st);
 
+// Quantized shard partials (communication scaling): x [n] fp32 -> codes (int8 per value at 8
+// bits, two 4-bit values per byte) + fp16 scales [ceil(n / 32)]; clear != 0 zeroes x after reading.
+cudaError_t launch_quantize_vec(float* x, int64_t n, int bits, uint8_t* codes, __half* scales, int clear,
+                                cudaStream_t st);
+struct CombineQArgs {
+    int bits[VT_MAX_DEVICES];            // per shard: 16 (fp32 partial) or 8 / 4 (codes + scales)
+    float* fparts[VT_MAX_DEVICES];       // bits 16
+    const uint8_t* codes[VT_MAX_DEVICES];
+    const __half* scales[VT_MAX_DEVICES];
+    int n;
+    int clear;                           // zero the fp32 partials after reading them
+    int64_t count;
+    const __half* residual;              // nullable
+    __half* out;
+};
+cudaError_t launch_combine_q(const CombineQArgs& a, cudaStream_t st);
+
 // ------------------------------------------------------------------ static-scratch decode attention
 // (static_scratch.cu) split-K decode attention whose scratch is one file-scope __device__ array.
 constexpr size_t kStaticScratchBytes = (size_t)1 << 20;  // 1 MiB

@@ -356,6 +356,121 @@ cudaError_t launch_gemv_q(int epi, const QGemvArgs& a, cudaStream_t st) {
     }
 }
 
+// ================================================================== quantized shard partials
+//
+// Communication scaling (Voltron Section 4.3.2): the activations sent between devices are lowered
+// to 8 or 4 bits.  Under tensor parallelism those are the fp32 shard partials sent to the main
+// device.  Format: blocks of 32 values, fp16 scale d = fp16(amax / qmax) and codes
+// round-half-even(x / d) clamped to [-qmax, qmax], fp32 decisions (the oracle's vector format);
+// stored as one int8 per value (8 bits) or two per byte (4 bits: value 2 i in the low nibble and
+// 2 i + 1 in the high nibble, each as q + 8).
+
+// One thread per block of 32 values.  clear: zero the partial after reading it (the partials of the
+// whole-token path are accumulated into zeroed buffers).
+template <int BITS>
+__global__ void k_quantize_vec(float* __restrict__ x, int64_t n, uint8_t* __restrict__ codes, __half* __restrict__ scales,
+                               int clear) {
+    constexpr int QMAX = BITS == 8 ? 127 : 7;
+    pdl_wait();
+    const int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, nb = (n + kQBlock - 1) / kQBlock;
+    if (b < nb) {
+        const int64_t e0 = b * kQBlock;
+        const int m = (int)(n - e0 < (int64_t)kQBlock ? n - e0 : (int64_t)kQBlock);
+        float v[kQBlock];
+        float amax = 0.f;
+#pragma unroll
+        for (int e = 0; e < kQBlock; ++e) {
+            v[e] = e < m ? x[e0 + e] : 0.f;
+            amax = fmaxf(amax, fabsf(v[e]));
+        }
+        const __half d16 = __float2half_rn(amax / (float)QMAX);
+        const float d = __half2float(d16);
+        scales[b] = d16;
+        int q[kQBlock];
+#pragma unroll
+        for (int e = 0; e < kQBlock; ++e) {
+            int c = 0;
+            if (d != 0.f) {
+                const float r = rintf(v[e] / d);
+                c = r > (float)QMAX ? QMAX : (r < (float)-QMAX ? -QMAX : (int)r);
+            }
+            q[e] = c;
+        }
+        if constexpr (BITS == 8) {
+            for (int e = 0; e < m; ++e) codes[e0 + e] = (uint8_t)(int8_t)q[e];
+        } else {
+            for (int e = 0; e < m; e += 2) {
+                const uint32_t lo = (uint32_t)(q[e] + 8), hi = e + 1 < m ? (uint32_t)(q[e + 1] + 8) : 8u;
+                codes[(e0 + e) >> 1] = (uint8_t)(lo | (hi << 4));
+            }
+        }
+        if (clear)
+            for (int e = 0; e < m; ++e) x[e0 + e] = 0.f;
+    }
+    pdl_launch_dependents();
+}
+
+cudaError_t launch_quantize_vec(float* x, int64_t n, int bits, uint8_t* codes, __half* scales, int clear,
+                                cudaStream_t st) {
+    const int64_t nb = (n + kQBlock - 1) / kQBlock;
+    if (nb <= 0) return cudaSuccess;
+    const unsigned grid = (unsigned)((nb + 127) / 128);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(128);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = g_use_pdl ? 1 : 0;
+    if (bits == 8) return cudaLaunchKernelEx(&cfg, k_quantize_vec<8>, x, n, codes, scales, clear);
+    if (bits == 4) return cudaLaunchKernelEx(&cfg, k_quantize_vec<4>, x, n, codes, scales, clear);
+    return cudaErrorInvalidValue;
+}
+
+// out[e] = fp16(residual[e] + sum_s p_s[e]) with shards in order, fp32: p_s is the fp32 partial
+// (bits 16; zeroed after reading when clear is set) or the dequantized code q_s[e] d_s[e / 32].
+__global__ void k_combine_q(const __grid_constant__ CombineQArgs a) {
+    pdl_wait();
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < a.count; e += (int64_t)gridDim.x * blockDim.x) {
+        float acc = a.residual ? __half2float(a.residual[e]) : 0.f;
+        for (int s = 0; s < a.n; ++s) {
+            const int bits = a.bits[s];
+            if (bits == 16) {
+                acc += __ldcg(a.fparts[s] + e);
+                if (a.clear) a.fparts[s][e] = 0.f;
+                continue;
+            }
+            int q;
+            if (bits == 8) {
+                q = (int)(int8_t)a.codes[s][e];
+            } else {
+                const uint8_t byte = a.codes[s][e >> 1];
+                q = (int)((e & 1) ? (byte >> 4) : (byte & 15)) - 8;
+            }
+            acc = fmaf((float)q, __half2float(a.scales[s][e / kQBlock]), acc);
+        }
+        a.out[e] = __float2half_rn(acc);
+    }
+    pdl_launch_dependents();
+}
+
+cudaError_t launch_combine_q(const CombineQArgs& a, cudaStream_t st) {
+    if (a.count <= 0) return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((a.count + 255) / 256, (int64_t)(g_num_sms > 0 ? g_num_sms : 148) * 8);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = g_use_pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k_combine_q, a);
+}
+
 cudaError_t init_quant_kernels() {
     const int lim = 200 * 1024;
     cudaError_t e;

@@ -15,10 +15,12 @@ class Stack:
     def __init__(self, shapes: vt.vt_shapes, layer_fn: Callable[[int], Dict[str, np.ndarray]],
                  head_ranges: Sequence[Tuple[int, int]], ffn_ranges: Sequence[Tuple[int, int]],
                  capacity: int, embed: Optional[np.ndarray] = None, stream=None, windows=None,
-                 precision=None):
+                 precision=None, layer_ranges=None):
         """windows: None, one sliding attention window for every layer, or one per layer (0: none).
         precision: None, or a function (layer, device, block) -> bits (16, 8 or 4) applied to every
-        shard before the KV cache is created."""
+        shard before the KV cache is created.  layer_ranges: None, or (head ranges per layer, FFN
+        ranges per layer, flags) for vt_partition_create_layers (head_ranges / ffn_ranges then only
+        give the device count)."""
         self.shapes = shapes
         self.model = self.part = self.kv = 0
         self.model = vt.vt_model_create(shapes, None, None, stream)
@@ -30,7 +32,11 @@ class Stack:
             ws = [windows] * shapes.n_layers if isinstance(windows, int) else list(windows)
             for l, w in enumerate(ws):
                 vt.vt_model_set_window(self.model, l, w)
-        self.part = vt.vt_partition_create(self.model, head_ranges, ffn_ranges, stream)
+        if layer_ranges is not None:  # per-layer table (head ranges per layer, FFN ranges per layer, flags)
+            lh, lc, flags = layer_ranges
+            self.part = vt.vt_partition_create_layers(self.model, lh, lc, flags, stream)
+        else:
+            self.part = vt.vt_partition_create(self.model, head_ranges, ffn_ranges, stream)
         if precision is not None:
             for l in range(shapes.n_layers):
                 for d in range(len(head_ranges)):

@@ -34,6 +34,7 @@ VT_DEV_WAIT_TIMEOUT = 2
 VT_DEV_BAD_TOKEN = 4
 VT_BLOCK_ATTN = 0
 VT_BLOCK_FFN = 1
+VT_PARTITION_PRUNE = 1
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -116,6 +117,10 @@ def lib() -> ctypes.CDLL:
             "vt_partition_create": (S, [_P, _I32, ctypes.POINTER(vt_range), ctypes.POINTER(vt_range),
                                         _P, ctypes.POINTER(_P)]),
             "vt_partition_devices": (_I32, [_P]),
+            "vt_partition_create_layers": (S, [_P, _I32, ctypes.POINTER(vt_range), ctypes.POINTER(vt_range),
+                                               ctypes.c_uint32, _P, ctypes.POINTER(_P)]),
+            "vt_partition_validate_layers": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(vt_range),
+                                                 ctypes.POINTER(vt_range), ctypes.c_uint32]),
             "vt_partition_status": (S, [_P, ctypes.POINTER(ctypes.c_uint32), _I32]),
             "vt_partition_destroy": (None, [_P]),
             "vt_shard_weights_read": (S, [_P, vt_shard, _I32, _P, ctypes.c_size_t,
@@ -142,6 +147,10 @@ def lib() -> ctypes.CDLL:
             "vt_partition_set_precision": (S, [_P, vt_shard, _I32, _P]),
             "vt_shard_precision": (_I32, [_P, vt_shard]),
             "vt_shard_qweights_read": (S, [_P, vt_shard, _I32, _P, _P]),
+            "vt_partial_code_bytes": (ctypes.c_size_t, [ctypes.c_int64, _I32]),
+            "vt_quantize_partial": (S, [_P, ctypes.c_int64, _I32, _P, _P, _P]),
+            "vt_combine_q": (S, [ctypes.POINTER(_P), ctypes.POINTER(_P), _I32, ctypes.c_int64, _I32, _P, _P, _P]),
+            "vt_partition_set_comm_bits": (S, [_P, _I32, _I32]),
             "vt_token_partials_read": (S, [_P, _I32, _P]),
         }
         for name, (res, args) in sig.items():
@@ -364,6 +373,30 @@ def vt_partition_create(model: int, head_ranges, ffn_col_ranges, stream=None) ->
     return out.value
 
 
+def _layer_ranges(per_layer):
+    n = len(per_layer[0])
+    if any(len(r) != n for r in per_layer):
+        raise ValueError("every layer needs one range per device")
+    return _ranges([r for layer in per_layer for r in layer]), n
+
+
+def vt_partition_create_layers(model: int, head_ranges, ffn_col_ranges, flags: int = 0, stream=None) -> int:
+    """head_ranges, ffn_col_ranges: one list of per-device ranges per layer."""
+    h, n = _layer_ranges(head_ranges)
+    c, n2 = _layer_ranges(ffn_col_ranges)
+    if n != n2:
+        raise ValueError("one head range and one FFN range per device")
+    out = _P()
+    _check(lib().vt_partition_create_layers(model, n, h, c, int(flags), _stream(stream), ctypes.byref(out)))
+    return out.value
+
+
+def vt_partition_validate_layers(shapes: vt_shapes, head_ranges, ffn_col_ranges, flags: int = 0) -> int:
+    h, n = _layer_ranges(head_ranges)
+    c, _ = _layer_ranges(ffn_col_ranges)
+    return int(lib().vt_partition_validate_layers(ctypes.byref(shapes), n, h, c, int(flags)))
+
+
 def vt_partition_devices(part: int) -> int:
     return int(lib().vt_partition_devices(part))
 
@@ -411,6 +444,31 @@ def vt_shard_qweights_read(part: int, shard: Tuple[int, int, int], which: int, r
     sc = np.empty((rows, (k + 31) // 32), np.float16)
     _check(lib().vt_shard_qweights_read(part, vt_shard(*shard), int(which), q.ctypes.data, sc.ctypes.data))
     return q, sc
+
+
+def vt_partial_code_bytes(count: int, bits: int) -> int:
+    return int(lib().vt_partial_code_bytes(int(count), int(bits)))
+
+
+def vt_quantize_partial(partial, bits: int, codes, scales, stream=None) -> None:
+    """Device fp32 partial -> device codes (uint8 tensor of vt_partial_code_bytes) and fp16 scales."""
+    import torch
+    _check(lib().vt_quantize_partial(_ptr(partial, torch.float32), partial.numel(), int(bits), _ptr(codes, torch.uint8),
+                                     _ptr(scales, torch.float16), _stream(stream)))
+
+
+def vt_combine_q(codes: Sequence, scales: Sequence, bits: int, residual, out, stream=None) -> None:
+    import torch
+    n = len(codes)
+    ca = (_P * n)(*[_ptr(c, torch.uint8) for c in codes])
+    sa = (_P * n)(*[_ptr(s_, torch.float16) for s_ in scales])
+    _check(lib().vt_combine_q(ca, sa, n, out.numel(), int(bits),
+                              _ptr(residual, torch.float16) if residual is not None else None,
+                              _ptr(out, torch.float16), _stream(stream)))
+
+
+def vt_partition_set_comm_bits(part: int, device: int, bits: int) -> None:
+    _check(lib().vt_partition_set_comm_bits(part, int(device), int(bits)))
 
 
 # ------------------------------------------------------------------ KV cache

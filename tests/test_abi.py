@@ -98,3 +98,22 @@ def test_workload_partitions_are_valid(vtlib):
                               wl.d_ffn, wl.vocab, wl.max_seq, wl.rms_eps, wl.rope_theta)
         assert vtlib.vt_shapes_validate(s) == 0, (wl.name, vtlib.vt_last_error())
         assert vtlib.vt_partition_validate(s, wl.head_ranges, wl.ffn_ranges) == 0, wl.name
+
+
+def test_partition_table_rules(vtlib):
+    """Per-layer partition tables (host-only validation): gaps need VT_PARTITION_PRUNE, KV-group
+    alignment and ordering still hold, unknown flags are refused."""
+    from tests.test_gpu_layers import PER_LAYER, PRUNED, WL
+    vt = vtlib
+    wl = WL
+    s = vt.make_shapes(wl.n_layers, wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, wl.vocab,
+                       wl.max_seq, wl.rms_eps, wl.rope_theta)
+    heads, cols = PRUNED
+    assert vt.vt_partition_validate_layers(s, heads, cols, 0) == vt.VT_ERR_PARTITION_GAP
+    assert vt.vt_partition_validate_layers(s, heads, cols, vt.VT_PARTITION_PRUNE) == vt.VT_OK
+    assert vt.vt_partition_validate_layers(s, *PER_LAYER, 0) == vt.VT_OK
+    bad = [[(0, 3), (3, 6), (6, 8)]] + PER_LAYER[0][1:]  # a head range off the KV groups of 2
+    assert vt.vt_partition_validate_layers(s, bad, PER_LAYER[1], 0) == vt.VT_ERR_PARTITION_GQA
+    over = [[(0, 4), (2, 6), (6, 8)]] + PER_LAYER[0][1:]
+    assert vt.vt_partition_validate_layers(s, over, PER_LAYER[1], vt.VT_PARTITION_PRUNE) == vt.VT_ERR_PARTITION_OVERLAP
+    assert vt.vt_partition_validate_layers(s, *PER_LAYER, 2) == vt.VT_ERR_INVALID_ARG
