@@ -20,6 +20,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <cstdlib>
 #include <string>
 
 #include "device.cuh"
@@ -549,6 +550,293 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
     }
 }
 
+// ================================================================== persistent tensor-core GEMM
+//
+// The grouped projections of a block (every shard's GEMM of one kind) as one persistent launch:
+// one CTA per SM walks output tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of the group in
+// an order where the 128-row tile is the fastest index, so the tiles that share a weight tile run
+// at the same time and the weights leave DRAM once.  Tiles are 128 x BN with BN chosen per launch
+// (256, 192, 160 or 128: the width that wastes least of the last round of tiles).
+//   warp 0   TMA producer: A (128 x 64) and B (BN x 64) boxes into a ring of stages (as many as
+//            fit in shared memory), one k-tile per stage, continuing across tiles;
+//   warp 1   tensor memory (512 columns: two accumulators of up to 256) and the MMA thread: the
+//            tile's k-tiles into accumulator (tile index & 1), then a commit that releases it to
+//            the epilogue;
+//   warps 2-5 epilogue: each warp reads its 32 accumulator lanes (rows) in chunks of 32 columns
+//            and writes the tile's outputs from registers; after the last chunk it hands the
+//            accumulator back, so the epilogue of one tile overlaps the MMAs of the next.
+// Every wait is bounded; on a timeout the CTA sets VT_DEV_WAIT_TIMEOUT and an abort flag, every
+// role stops at its next wait, copies and MMAs in flight are waited for (bounded), and tensor
+// memory is freed.
+
+constexpr int kPStages = 8;     // most ring stages
+constexpr int kPTmemCols = 512;  // two accumulators
+constexpr size_t kPGemmSmem = 227 * 1024;
+
+struct PGemmGroup {
+    int n_groups, tiles_m, bn, total_tiles, stages;
+    int tile_end[kGemmGroups];  // cumulative tiles (tiles_m x column tiles of each group)
+    CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
+    GemmArgs a[kGemmGroups];
+};
+
+__device__ __forceinline__ void ptile(const PGemmGroup& G, int t, int& g, int& m0, int& n0) {
+    g = 0;
+    while (g + 1 < G.n_groups && t >= G.tile_end[g]) ++g;
+    const int u = t - (g > 0 ? G.tile_end[g - 1] : 0);
+    m0 = (u % G.tiles_m) * kBM;
+    n0 = (u / G.tiles_m) * G.bn;
+}
+
+// Epilogue of 32 consecutive columns [col0, col0 + 32) of row `row` (col0 a multiple of 32).
+template <int EPI>
+__device__ __forceinline__ void pepi_chunk(const GemmArgs& a, int row, int col0, const uint32_t (&r)[32], int pos) {
+    if constexpr (EPI == kGemmF32) {
+        float* dst = a.c + (size_t)row * a.ldc + col0;
+        if (col0 + 32 <= a.n) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                reinterpret_cast<float4*>(dst)[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                                                __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (col0 + j < a.n) dst[j] = __uint_as_float(r[j]);
+        }
+    } else if constexpr (EPI == kGemmQkv) {
+        // 16 RoPE pairs (columns 2p, 2p + 1 = dims i0 + p and i0 + p + dh / 2 of one head block)
+        if (col0 >= a.n) return;
+        const int dh = a.dh, half = dh / 2;
+        const int b = col0 / dh, i0 = (col0 % dh) / 2;
+        float lo[16], hi[16];
+        if (b < a.hq + a.hk) {
+            const float2* cs = a.rope + (size_t)pos * half + i0;
+#pragma unroll
+            for (int p = 0; p < 16; ++p) {
+                const float2 c = cs[p];
+                const float x0 = __uint_as_float(r[2 * p]), x1 = __uint_as_float(r[2 * p + 1]);
+                lo[p] = x0 * c.x - x1 * c.y;
+                hi[p] = x0 * c.y + x1 * c.x;
+            }
+        } else {
+#pragma unroll
+            for (int p = 0; p < 16; ++p) {
+                lo[p] = __uint_as_float(r[2 * p]);
+                hi[p] = __uint_as_float(r[2 * p + 1]);
+            }
+        }
+        __half* dst;
+        if (b < a.hq) dst = a.q + ((size_t)row * a.hq + b) * dh;
+        else if (b < a.hq + a.hk) dst = a.kcache + ((size_t)(b - a.hq) * a.cap + pos) * dh;
+        else dst = a.vcache + ((size_t)(b - a.hq - a.hk) * a.cap + pos) * dh;
+        uint32_t wl[8], wh[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const __half2 l2 = __floats2half2_rn(lo[2 * j], lo[2 * j + 1]), h2 = __floats2half2_rn(hi[2 * j], hi[2 * j + 1]);
+            wl[j] = *reinterpret_cast<const uint32_t*>(&l2);
+            wh[j] = *reinterpret_cast<const uint32_t*>(&h2);
+        }
+        uint4* dl = reinterpret_cast<uint4*>(dst + i0);
+        uint4* dhp = reinterpret_cast<uint4*>(dst + i0 + half);
+        dl[0] = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+        dl[1] = make_uint4(wl[4], wl[5], wl[6], wl[7]);
+        dhp[0] = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+        dhp[1] = make_uint4(wh[4], wh[5], wh[6], wh[7]);
+    } else {
+        // (gate, up) pairs of intermediate columns col0 / 2 + p
+        __half* dst = a.u + (size_t)row * a.ldu + a.ushift + col0 / 2;
+        if (col0 == 0)
+            for (int j = 0; j < a.ushift; ++j) dst[j - a.ushift] = __float2half_rn(0.f);
+#pragma unroll
+        for (int p = 0; p < 16; ++p)
+            if (col0 + 2 * p < a.n) dst[p] = __float2half_rn(silu(__uint_as_float(r[2 * p])) * __uint_as_float(r[2 * p + 1]));
+    }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constant__ PGemmGroup G) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const int S = G.stages, BN = G.bn;
+    const uint32_t b_bytes = (uint32_t)BN * kBK * 2, stage_bytes = (uint32_t)kABytes + b_bytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
+    uint64_t* empty = full + kPStages;
+    uint64_t* tfull = empty + kPStages;  // [2] accumulator b holds a finished tile
+    uint64_t* tempty = tfull + 2;        // [2] accumulator b was read by the epilogue
+    uint64_t* done = tempty + 2;         // every MMA issued by this CTA has completed
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+    __shared__ int s_err;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 1);
+            mbar_init(&tempty[b], 4);
+        }
+        mbar_init(done, 1);
+        s_err = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(tmem_slot, kPTmemCols);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = *tmem_slot;
+    uint32_t* status = G.a[0].status;
+    auto abort_cta = [&]() {
+        s_err = 1;
+        set_status(status, VT_DEV_WAIT_TIMEOUT);
+    };
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            pdl_wait();  // A was written by the preceding kernel
+            uint32_t k = 0;  // stages filled so far
+            for (int t = blockIdx.x; t < G.total_tiles && !*(volatile int*)&s_err; t += gridDim.x) {
+                int g, m0, n0;
+                ptile(G, t, g, m0, n0);
+                const GemmArgs& a = G.a[g];
+                for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
+                    const int s = (int)(k % (uint32_t)S);
+                    if (k >= (uint32_t)S && !mbar_wait(&empty[s], ((k / S) - 1) & 1)) {
+                        abort_cta();
+                        break;
+                    }
+                    if (*(volatile int*)&s_err) break;
+                    uint8_t* st = smem + (size_t)s * stage_bytes;
+                    mbar_arrive_expect_tx(&full[s], stage_bytes);
+                    tc::tma_load_2d(st, &G.ta[g], kt * kBK, m0, &full[s]);
+                    tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
+                }
+            }
+            // no copy may be in flight when the CTA ends
+            for (uint32_t i = k > (uint32_t)S ? k - S : 0; i < k; ++i)
+                if (!mbar_wait(&full[i % S], (i / S) & 1)) set_status(status, VT_DEV_WAIT_TIMEOUT);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            uint32_t k = 0;
+            int it = 0;
+            for (int t = blockIdx.x; t < G.total_tiles && !*(volatile int*)&s_err; t += gridDim.x, ++it) {
+                int g, m0, n0;
+                ptile(G, t, g, m0, n0);
+                const GemmArgs& a = G.a[g];
+                const int buf = it & 1;
+                if (it >= 2 && !mbar_wait(&tempty[buf], ((it >> 1) - 1) & 1)) {
+                    abort_cta();
+                    break;
+                }
+                tc::fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
+                const uint32_t idesc = tc::idesc_f16(kBM, BN);
+                bool ok = true;
+                for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
+                    const int s = (int)(k % (uint32_t)S);
+                    if (!mbar_wait(&full[s], (k / S) & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after();
+                    const uint32_t sa = smem_u32(smem + (size_t)s * stage_bytes), sb = sa + kABytes;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk)
+                        tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
+                                    (kt | kk) != 0);
+                    tc::mma_commit(&empty[s]);
+                }
+                if (!ok) {
+                    abort_cta();
+                    break;
+                }
+                tc::mma_commit(&tfull[buf]);
+            }
+            tc::mma_commit(done);
+            if (!mbar_wait(done, 0)) set_status(status, VT_DEV_WAIT_TIMEOUT);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 2-5)
+        const int sub = warp & 3;  // accumulator lanes [32 sub, 32 sub + 32)
+        int it = 0;
+        for (int t = blockIdx.x; t < G.total_tiles; t += gridDim.x, ++it) {
+            int g, m0, n0;
+            ptile(G, t, g, m0, n0);
+            const GemmArgs& a = G.a[g];
+            const int buf = it & 1;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(&tfull[buf], (it >> 1) & 1) && !*(volatile int*)&s_err;
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) {
+                if (lane == 0) abort_cta();
+                break;
+            }
+            tc::fence_after();
+            const int row = m0 + sub * 32 + lane;
+            int pos = 0;
+            bool row_ok = row < a.m;
+            if constexpr (EPI == kGemmQkv) {
+                pos = *a.len + a.row_offset + row;
+                if (row_ok && (pos < 0 || pos >= a.cap)) {
+                    set_status(a.status, VT_DEV_KV_OVERFLOW);
+                    row_ok = false;
+                }
+            }
+            const uint32_t base = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(buf * 256);
+            for (int c = 0; c < BN; c += 32) {
+                uint32_t r[32];
+                tc::tmem_ld32(base + (uint32_t)c, r);  // warp-collective: every lane takes part
+                tc::tmem_ld_wait();
+                if (row_ok && n0 + c < a.n) pepi_chunk<EPI>(a, row, n0 + c, r, pos);
+            }
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_dealloc(tmem, kPTmemCols);
+    }
+}
+
+// Tile width for a persistent launch: the one whose rounds of tiles (over `ctas` CTAs) take least,
+// a tile's time growing with its width plus a fixed share (its A box and epilogue).
+static int choose_bn(const int* n, int groups, int tiles_m, int ctas, int* total) {
+    static const int cand[] = {256, 192, 160, 128};
+    int best = 256, best_t = 0;
+    double best_cost = 1e30;
+    for (int bn : cand) {
+        int tiles = 0;
+        for (int g = 0; g < groups; ++g) tiles += tiles_m * ((n[g] + bn - 1) / bn);
+        const int rounds = (tiles + ctas - 1) / ctas;
+        const double cost = (double)rounds * (bn + 48);
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            best = bn;
+            best_t = tiles;
+        }
+    }
+    *total = best_t;
+    return best;
+}
+
+static size_t pgemm_stage_bytes(int bn) { return (size_t)kABytes + (size_t)bn * kBK * 2; }
+static int pgemm_stages(int bn) {
+    const size_t room = kPGemmSmem - 1024 - 256;
+    int s = (int)(room / pgemm_stage_bytes(bn));
+    return s > kPStages ? kPStages : s;
+}
+
 // ================================================================== causal attention
 
 struct PrefillAttnKArgs {
@@ -757,6 +1045,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
 // ================================================================== host side
 
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static bool g_gemm_persistent = true;  // VT_GEMM_PERSISTENT=0 keeps every GEMM on k_gemm
 constexpr int kMaxSplit = 4;
 static int g_split_clusters[kMaxSplit + 1];  // co-resident clusters of S GEMM CTAs (index S)
 
@@ -792,6 +1081,13 @@ cudaError_t init_prefill_kernels() {
             nc = 0;
         }
         g_split_clusters[sp] = nc;
+    }
+    for (auto f : {k_gemm_p<kGemmF32>, k_gemm_p<kGemmQkv>, k_gemm_p<kGemmSwiglu>})
+        if ((e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(kPGemmSmem - 1024))) != cudaSuccess)
+            return e;
+    {
+        const char* v = getenv("VT_GEMM_PERSISTENT");
+        g_gemm_persistent = !(v && v[0] == '0');
     }
     if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)prefill_attn_smem<128>())) != cudaSuccess)
@@ -862,13 +1158,72 @@ struct GemmSpec {
     int kb = 0;  // > 0: B has kb columns and A's k = 2 kb columns hold the hi and lo halves of the input
 };
 
-// Launches the GEMMs of `specs` (all with m rows) kGemmGroups at a time, one CTA (or split-K
-// cluster) per output tile of every GEMM: the shards of a block fill the GPU together instead of
-// a few tiles each.
+
+// The grouped GEMMs of `specs` (all with m rows) as one persistent launch.  B maps are encoded
+// with the chosen tile width as their box height.
+template <int EPI>
+static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaStream_t st, std::string* err) {
+    PGemmGroup G{};
+    G.n_groups = ng;
+    G.tiles_m = (m + kBM - 1) / kBM;
+    int ns[kGemmGroups];
+    for (int g = 0; g < ng; ++g) ns[g] = specs[g].n;
+    const int ctas_max = g_num_sms > 0 ? g_num_sms : 148;
+    int total = 0;
+    G.bn = choose_bn(ns, ng, G.tiles_m, ctas_max, &total);
+    G.total_tiles = total;
+    G.stages = pgemm_stages(G.bn);
+    int acc = 0;
+    for (int g = 0; g < ng; ++g) {
+        const GemmSpec& sp = specs[g];
+        if (sp.kb > 0 && (sp.kb % kBK != 0 || sp.k != 2 * sp.kb)) {
+            *err = "a split GEMM needs k = 2 kb with kb a multiple of 64";
+            return VT_ERR_INVALID_ARG;
+        }
+        if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) ||
+            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn, err))
+            return VT_ERR_INVALID_ARG;
+        GemmArgs& a = G.a[g];
+        a = sp.base;
+        a.m = m;
+        a.n = sp.n;
+        a.b = static_cast<const __half*>(sp.B);
+        a.ldb = sp.ldb;
+        a.k_tiles = (sp.k + kBK - 1) / kBK;
+        a.kb_wrap = sp.kb > 0 ? sp.kb / kBK : 0;
+        acc += G.tiles_m * ((sp.n + G.bn - 1) / G.bn);
+        G.tile_end[g] = acc;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)std::min(total, ctas_max));
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn) + 256;
+    cfg.stream = st;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_p<EPI>, G);
+    if (e != cudaSuccess) {
+        *err = std::string("persistent GEMM launch failed: ") + cudaGetErrorString(e);
+        return VT_ERR_CUDA;
+    }
+    return VT_OK;
+}
+
+// Launches the GEMMs of `specs` (all with m rows) kGemmGroups at a time.  A group with at least
+// as many 128 x 256 tiles as half the SMs runs as one persistent launch (k_gemm_p); a smaller one
+// (short prompts, a single shard) as one CTA, or split-K cluster, per output tile (k_gemm), so
+// that its few tiles still spread over the GPU.
 template <int EPI>
 static vt_status run_gemm_group(const GemmSpec* specs, int n_specs, int m, cudaStream_t st, std::string* err) {
     for (int g0 = 0; g0 < n_specs; g0 += kGemmGroups) {
         const int ng = std::min(kGemmGroups, n_specs - g0);
+        {
+            int tiles = 0;
+            for (int g = 0; g < ng; ++g) tiles += ((m + kBM - 1) / kBM) * ((specs[g0 + g].n + kBN - 1) / kBN);
+            if (g_gemm_persistent && 2 * tiles >= (g_num_sms > 0 ? g_num_sms : 148)) {
+                const vt_status r = run_gemm_persistent<EPI>(specs + g0, ng, m, st, err);
+                if (r != VT_OK) return r;
+                continue;
+            }
+        }
         GemmGroup G{};
         G.n_groups = ng;
         int tiles_n = 0, max_k_tiles = 1, min_k_tiles = 1 << 30;
