@@ -410,7 +410,9 @@ VT_API vt_status vt_decode_step(const vt_partition* part, vt_shard shard, const 
  *   VT_ERR_INVALID_ARG (it uses no scratch; call vt_decode_step).
  *   First call on a device: looks up the array's device address with cudaGetSymbolAddress, with
  *   that device current, and keeps it.  Any failure is VT_ERR_CUDA.  Make that first call before
- *   any stream capture on that device begins.
+ *   any stream capture on that device begins.  The kept address is the array's for the life of
+ *   the device's primary context: do not use the library across a cudaDeviceReset (the module
+ *   would load again and the array could move).
  *   Must start at zero: only the 64 per-KV-head arrival counters at the start of the array.  The
  *   module loader zeroes them, and every call leaves them at zero.
  *   Races: the array is shared by every call in the process on that device.  Two calls in flight

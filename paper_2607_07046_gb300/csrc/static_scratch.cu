@@ -103,13 +103,21 @@ __global__ void __launch_bounds__(kSplitWarps * 32) k_attn_decode_split(const __
             o[h][e] = 0.f;
         }
     }
+    // one vector load per lane for its EPL elements of a K row and of a V row (8 or 4 bytes)
+    auto load_row = [&](const __half* row, float (&dst)[EPL]) {
+        if constexpr (EPL == 4) {
+            const uint2 u = __ldcg(reinterpret_cast<const uint2*>(row + lane * 4));
+            const float2 f0 = h2_to_f2(u.x), f1 = h2_to_f2(u.y);
+            dst[0] = f0.x; dst[1] = f0.y; dst[2] = f1.x; dst[3] = f1.y;
+        } else {
+            const float2 f0 = h2_to_f2(__ldcg(reinterpret_cast<const unsigned int*>(row + lane * 2)));
+            dst[0] = f0.x; dst[1] = f0.y;
+        }
+    };
     for (int p = t0 + warp; p < t1; p += kSplitWarps) {
         float kv[EPL], vv[EPL];
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) {
-            kv[e] = __half2float(__ldcg(kbase + (int64_t)p * DH + lane * EPL + e));
-            vv[e] = __half2float(__ldcg(vbase + (int64_t)p * DH + lane * EPL + e));
-        }
+        load_row(kbase + (int64_t)p * DH, kv);
+        load_row(vbase + (int64_t)p * DH, vv);
 #pragma unroll
         for (int h = 0; h < G; ++h) {
             float sc = 0.f;

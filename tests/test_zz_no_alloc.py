@@ -44,11 +44,23 @@ def _fill(vt, st, wl, L):
     vt.vt_kv_set_length(st.kv, -1, L)
 
 
+def _gqa(name, n_heads, n_kv_heads):
+    return synthetic.small(name, n_layers=1, d_model=512, n_heads=n_heads, n_kv_heads=n_kv_heads, d_head=64,
+                           d_ffn=256, head_ranges=((0, n_heads // 2), (n_heads // 2, n_heads)),
+                           ffn_ranges=((0, 128), (128, 256)), kv_len=20, decode_steps=2, prompt_len=0, model_id=150)
+
+
 CASES = [
     # (workload, cached positions before the first token): 2-way MHA with dh 64 and a length that
-    # leaves ragged slices; one layer of the 8B GQA model (4 query heads per KV head, dh 128).
+    # leaves ragged slices; one layer of the 8B GQA model (4 query heads per KV head, dh 128);
+    # 8 and 2 query heads per KV head at lengths that leave most of the 16 slices empty (the
+    # merge then weighs empty slices by zero).
     ("tiny", lambda: synthetic.WORKLOADS[1], 100),
     ("8b-gqa", lambda: dataclasses.replace(synthetic.WORKLOADS[5], n_layers=1), 300),
+    ("gqa8-L0", lambda: _gqa("gqa8", 16, 2), 0),
+    ("gqa8-L1", lambda: _gqa("gqa8", 16, 2), 1),
+    ("gqa2-L15", lambda: _gqa("gqa2", 8, 4), 15),
+    ("gqa2-L17", lambda: _gqa("gqa2", 8, 4), 17),
 ]
 
 
