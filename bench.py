@@ -578,6 +578,79 @@ def run_decode_workload(cid, steps, warmup, bits=16):
     }
 
 
+# ------------------------------------------------------------------ shard latency sweep
+
+def run_sweep(args):
+    """Latency of one shard's decode step (vt_decode_step) against the shard's width (the 7B
+    layer split n ways, n = 1, 2, 4, 8) and, for ATTN shards, the KV length: the measurements
+    behind the planner's time model (a device's time for a shard = its bytes / a streaming rate).
+    Each timed step is cold: the L2 is flushed (a 256 MB write) before it, and steps walk a stack
+    of layers.  Fits time = t0 + bytes / rate over all points and feeds the fitted rate to
+    vt_plan_layers for a 4-device plan of the 7B stack over a slow and a fast link."""
+    import torch
+
+    from paper_2607_07046_gb300 import build as vt_build
+    from paper_2607_07046_gb300 import vt
+    from paper_2607_07046_gb300.stack import Stack
+
+    vt_build.build()
+    torch.cuda.set_device(0)
+    base = synthetic.WORKLOADS[2]
+    layers = 4
+    lengths = [128, 1024, 4096, 16384]
+    cap = max(lengths) + 8
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    D, dh, H, F = base.d_model, base.d_head, base.n_heads, base.d_ffn
+    points = []
+    for n in (1, 2, 4, 8):
+        import dataclasses
+        wl = dataclasses.replace(base, n_layers=layers, head_ranges=synthetic._even(H, n),
+                                 ffn_ranges=synthetic._even(F, n))
+        shapes = shapes_for(vt, wl, cap)
+        with Stack(shapes, wl.layer_weights, wl.head_ranges, wl.ffn_ranges, cap) as st:
+            x = torch.from_numpy(wl.hidden(1).reshape(-1)).cuda()
+            out = torch.empty(D, dtype=torch.float32, device="cuda")
+            hq, c = H // n, F // n
+            w_attn = 2 * ((hq + 2 * hq) * dh * D + D * hq * dh)
+            w_ffn = 2 * 3 * D * c
+
+            def timed(fn, reps=12):
+                ts = []
+                for i in range(reps):
+                    flush.zero_()
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                    fn(i % layers)
+                    e1.record()
+                    e1.synchronize()
+                    ts.append(e0.elapsed_time(e1) * 1e3)
+                return float(np.median(ts[2:]))
+
+            for L in lengths:
+                vt.vt_kv_set_length(st.kv, -1, L)
+                us = timed(lambda l: vt.vt_decode_step(st.part, (l, 0, vt.VT_BLOCK_ATTN), x, st.kv, out))
+                byt = w_attn + 2 * 2 * hq * dh * (L + 1)
+                points.append({"block": "attn", "shards": n, "heads": hq, "kv_len": L, "us": round(us, 2),
+                               "bytes": byt, "gbs": round(byt / us / 1e3, 1)})
+            us = timed(lambda l: vt.vt_decode_step(st.part, (l, 0, vt.VT_BLOCK_FFN), x, None, out))
+            points.append({"block": "ffn", "shards": n, "cols": c, "us": round(us, 2), "bytes": w_ffn,
+                           "gbs": round(w_ffn / us / 1e3, 1)})
+    # least-squares fit of time = t0 + bytes / rate
+    A = np.array([[1.0, p["bytes"]] for p in points])
+    y = np.array([p["us"] * 1e-6 for p in points])
+    (t0, inv_rate), *_ = np.linalg.lstsq(A, y, rcond=None)
+    rate = 1.0 / inv_rate
+    sh = shapes_for(vt, base, base.kv_len + 8)
+    plans = {}
+    for name, link in (("wifi_60MBps", 60e6), ("nvlink_900GBps", 900e9)):
+        pl, tot = vt.vt_plan_layers(sh, [rate] * 4, None, None, link, 2e-6, 1, base.kv_len)
+        plans[name] = {"tp_blocks": sum(1 for b in pl if b["tp"]), "mp_blocks": sum(1 for b in pl if not b["tp"]),
+                       "token_s": tot, "first_ffn": pl[1]["ranges"]}
+    return {"sweep": "shard decode-step latency, 7B layer split n ways, cold L2", "points": points,
+            "fit": {"t0_us": round(t0 * 1e6, 2), "rate_gbs": round(rate / 1e9, 1)},
+            "plans_with_fitted_rate": plans}
+
+
 # ------------------------------------------------------------------ reference arm (CPU oracle)
 
 def run_reference(args):
@@ -626,12 +699,17 @@ def main():
                     help="timed tokens of the per-shard entry point, for context (0: skip)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: only the first N layers of the stack")
+    ap.add_argument("--sweep", action="store_true",
+                    help="only the shard latency sweep (width x KV length) and the planner fed with its rate")
     ap.add_argument("--min-timed-s", type=float, default=0.3,
                     help="repeat the K-step timed region until it covers this many seconds in total")
     ap.add_argument("--other-steps", type=int, default=64,
                     help="timed tokens of the 13B and 8B decode workloads, 1 GPU only (0: skip)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.sweep:
+        print(json.dumps(run_sweep(args)), flush=True)
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
