@@ -728,29 +728,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         if (lane == 0) {
             pdl_wait();  // A was written by the preceding kernel
             uint32_t k = 0;  // stages filled so far
-            // The weights (B) are read once, so every B box comes from DRAM: its L2 prefetch runs
-            // kPrefetch k-tiles ahead of its load (into the next work unit near a unit's end), so
-            // that the loads that fill the ring find their data in L2.
-            constexpr int kPrefetch = 16;
-            auto prefetch_b = [&](int t, int kt) {
-                if (t >= G.total_units) return;
-                int g2, m2, n2;
-                ptile(G, t, rank, g2, m2, n2);
-                const GemmArgs& a2 = G.a[g2];
-                if (kt < a2.k_tiles) tc::tma_prefetch_2d(&G.tb[g2], bk_tile(a2, kt) * kBK, n2 + rank * bq);
-            };
-            {
-                int g, m0, n0;
-                ptile(G, cid, rank, g, m0, n0);
-                for (int kt = 0; kt < kPrefetch; ++kt) prefetch_b(cid, kt);
-            }
             for (int t = cid; t < G.total_units && !*(volatile int*)&s_err; t += nclus) {
                 int g, m0, n0;
                 ptile(G, t, rank, g, m0, n0);
                 const GemmArgs& a = G.a[g];
                 for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
-                    if (kt + kPrefetch < a.k_tiles) prefetch_b(t, kt + kPrefetch);
-                    else prefetch_b(t + nclus, kt + kPrefetch - a.k_tiles);
                     const int s = (int)(k % (uint32_t)S);
                     // the stage is free in every CTA of the cluster (this CTA writes into all of them)
                     if (k >= (uint32_t)S && !mbar_wait(&empty[s], ((k / S) - 1) & 1)) {
