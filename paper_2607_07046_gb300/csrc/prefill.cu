@@ -42,23 +42,6 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
-// The same box written to the same shared-memory offset in every CTA of the cluster in `mask`,
-// completing as transaction bytes on the mbarrier at `bar`'s offset in each of them.
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar,
-                                               uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(
-            smem_u32(dst)),
-        "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar)), "h"(mask)
-        : "memory");
-}
-
-// Pulls the box at (x, y) into L2 without writing shared memory.
-__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
-    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map), "r"(x), "r"(y)
-                 : "memory");
-}
-
 // 16-byte store into the shared memory of a CTA of the cluster (address from mapa).
 __device__ __forceinline__ void dsmem_st4(uint32_t addr, float a, float b, float c, float d) {
     asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
@@ -86,14 +69,6 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
-}
-// Arrives once on the mbarrier at `bar`'s offset in every CTA of the cluster in `mask` when every
-// MMA this thread issued so far has completed.
-__device__ __forceinline__ void mma_commit_mc(uint64_t* bar, uint16_t mask) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-                     smem_u32(bar)),
-                 "h"(mask)
-                 : "memory");
 }
 // Arrives once on `bar` when every MMA this thread issued so far has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -574,8 +549,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
 // The grouped projections of a block (every shard's GEMM of one kind) as one persistent launch:
 // one CTA per SM walks output tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of the group in
 // an order where the 128-row tile is the fastest index, so the tiles that share a weight tile run
-// at the same time and the weights leave DRAM once.  Tiles are 128 x BN with BN chosen per launch
-// (256, 192, 160 or 128: the width that wastes least of the last round of tiles).
+// at the same time and the weights leave DRAM once.  Tiles are 128 x 256.
 //   warp 0   TMA producer: A (128 x 64) and B (BN x 64) boxes into a ring of stages (as many as
 //            fit in shared memory), one k-tile per stage, continuing across tiles;
 //   warp 1   tensor memory (512 columns: two accumulators of up to 256) and the MMA thread: the
@@ -593,22 +567,19 @@ constexpr int kPTmemCols = 512;  // two accumulators
 constexpr size_t kPGemmSmem = 227 * 1024;
 
 struct PGemmGroup {
-    int n_groups, tiles_m, bn, total_units, stages;
-    int csize;                  // CTAs per cluster (1, 2, 4): the row tiles that share a weight tile
-    int tile_end[kGemmGroups];  // cumulative work units (tiles_m / csize x column tiles of each group)
+    int n_groups, tiles_m, bn, total_tiles, stages;
+    int tile_end[kGemmGroups];  // cumulative tiles (tiles_m x column tiles of each group)
     CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
     GemmArgs a[kGemmGroups];
 };
 
-// Work unit t: csize row tiles (rank r of the cluster takes row tile mg csize + r) of one column
-// tile of one group; the row-tile group is the fastest index.
-__device__ __forceinline__ void ptile(const PGemmGroup& G, int t, int rank, int& g, int& m0, int& n0) {
+// Tile t of the group: the row tile is the fastest index.
+__device__ __forceinline__ void ptile(const PGemmGroup& G, int t, int& g, int& m0, int& n0) {
     g = 0;
     while (g + 1 < G.n_groups && t >= G.tile_end[g]) ++g;
     const int u = t - (g > 0 ? G.tile_end[g - 1] : 0);
-    const int mgroups = G.tiles_m / G.csize;
-    m0 = ((u % mgroups) * G.csize + rank) * kBM;
-    n0 = (u / mgroups) * G.bn;
+    m0 = (u % G.tiles_m) * kBM;
+    n0 = (u / G.tiles_m) * G.bn;
 }
 
 // Epilogue of 32 consecutive columns [col0, col0 + 32) of row `row` (col0 a multiple of 32).
@@ -680,12 +651,10 @@ template <int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constant__ PGemmGroup G) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    const int S = G.stages, BN = G.bn, C = G.csize;
+    const int S = G.stages, BN = G.bn;
     const uint32_t b_bytes = (uint32_t)BN * kBK * 2, stage_bytes = (uint32_t)kABytes + b_bytes;
-    const int bq = BN / C;  // rows of each B tile this CTA loads (and multicasts to the cluster)
-    const uint16_t cmask = (uint16_t)((1u << C) - 1u);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
-    uint64_t* empty = full + kPStages;   // count C: every CTA of the cluster released the stage
+    uint64_t* empty = full + kPStages;
     uint64_t* tfull = empty + kPStages;  // [2] accumulator b holds a finished tile
     uint64_t* tempty = tfull + 2;        // [2] accumulator b was read by the epilogue
     uint64_t* done = tempty + 2;         // every MMA issued by this CTA has completed
@@ -693,12 +662,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
     __shared__ int s_err;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int rank = C > 1 ? (int)cluster_rank() : 0;
-    const int cid = (int)blockIdx.x / C, nclus = (int)gridDim.x / C;
+    const int cid = (int)blockIdx.x, nctas = (int)gridDim.x;
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], (uint32_t)C);
+            mbar_init(&empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull[b], 1);
@@ -714,7 +682,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
     }
     tc::fence_before();
     __syncthreads();
-    if (C > 1) cluster_sync();  // every CTA's barriers exist before any multicast reaches them
     tc::fence_after();
     const uint32_t tmem = *tmem_slot;
     uint32_t* status = G.a[0].status;
@@ -728,26 +695,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         if (lane == 0) {
             pdl_wait();  // A was written by the preceding kernel
             uint32_t k = 0;  // stages filled so far
-            for (int t = cid; t < G.total_units && !*(volatile int*)&s_err; t += nclus) {
+            for (int t = cid; t < G.total_tiles && !*(volatile int*)&s_err; t += nctas) {
                 int g, m0, n0;
-                ptile(G, t, rank, g, m0, n0);
+                ptile(G, t, g, m0, n0);
                 const GemmArgs& a = G.a[g];
                 for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
                     const int s = (int)(k % (uint32_t)S);
-                    // the stage is free in every CTA of the cluster (this CTA writes into all of them)
                     if (k >= (uint32_t)S && !mbar_wait(&empty[s], ((k / S) - 1) & 1)) {
                         abort_cta();
                         break;
                     }
                     if (*(volatile int*)&s_err) break;
                     uint8_t* st = smem + (size_t)s * stage_bytes;
-                    mbar_arrive_expect_tx(&full[s], stage_bytes);  // own A + the whole B tile from the cluster
+                    mbar_arrive_expect_tx(&full[s], stage_bytes);
                     tc::tma_load_2d(st, &G.ta[g], kt * kBK, m0, &full[s]);
-                    if (C > 1)
-                        tc::tma_load_2d_mc(st + kABytes + (size_t)rank * bq * kBK * 2, &G.tb[g], bk_tile(a, kt) * kBK,
-                                           n0 + rank * bq, &full[s], cmask);
-                    else
-                        tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
+                    tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
                 }
             }
             // no copy may be in flight when the CTA ends
@@ -759,9 +721,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         if (lane == 0) {
             uint32_t k = 0;
             int it = 0;
-            for (int t = cid; t < G.total_units && !*(volatile int*)&s_err; t += nclus, ++it) {
+            for (int t = cid; t < G.total_tiles && !*(volatile int*)&s_err; t += nctas, ++it) {
                 int g, m0, n0;
-                ptile(G, t, rank, g, m0, n0);
+                ptile(G, t, g, m0, n0);
                 const GemmArgs& a = G.a[g];
                 const int buf = it & 1;
                 if (it >= 2 && !mbar_wait(&tempty[buf], ((it >> 1) - 1) & 1)) {
@@ -784,8 +746,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                     for (int kk = 0; kk < kBK / 16; ++kk)
                         tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
                                     (kt | kk) != 0);
-                    if (C > 1) tc::mma_commit_mc(&empty[s], cmask);  // released in every CTA of the cluster
-                    else tc::mma_commit(&empty[s]);
+                    tc::mma_commit(&empty[s]);
                 }
                 if (!ok) {
                     abort_cta();
@@ -800,9 +761,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         // ------------------------------------------------------------ epilogue (warps 2-5)
         const int sub = warp & 3;  // accumulator lanes [32 sub, 32 sub + 32)
         int it = 0;
-        for (int t = cid; t < G.total_units; t += nclus, ++it) {
+        for (int t = cid; t < G.total_tiles; t += nctas, ++it) {
             int g, m0, n0;
-            ptile(G, t, rank, g, m0, n0);
+            ptile(G, t, g, m0, n0);
             const GemmArgs& a = G.a[g];
             const int buf = it & 1;
             int ok = 1;
@@ -837,35 +798,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
     }
     tc::fence_before();
     __syncthreads();
-    // no CTA leaves while a peer may still multicast into its stages or arrive on its barriers
-    if (C > 1) cluster_sync();
     if (warp == 1) {
         tc::fence_after();
         tc::tmem_dealloc(tmem, kPTmemCols);
     }
 }
 
-// Tile width for a persistent launch: the one whose rounds of work units (over `clusters`
-// clusters of csize CTAs) take least, a tile's time growing with its width plus a fixed share
-// (its A box and epilogue).
-static int choose_bn(const int* n, int groups, int mgroups, int clusters, int* total) {
-    static const int cand[] = {256, 192, 160, 128};
-    int best = 256, best_t = 0;
-    double best_cost = 1e30;
-    for (int bn : cand) {
-        int units = 0;
-        for (int g = 0; g < groups; ++g) units += mgroups * ((n[g] + bn - 1) / bn);
-        const int rounds = (units + clusters - 1) / clusters;
-        const double cost = (double)rounds * (bn + 48);
-        if (cost < best_cost - 1e-9) {
-            best_cost = cost;
-            best = bn;
-            best_t = units;
-        }
-    }
-    *total = best_t;
-    return best;
-}
+// Tile width of the persistent GEMM: 128 x 256.  Per k-tile the ring moves the A and B boxes
+// through shared memory at a rate that does not grow with a narrower B (measured: a stage costs
+// about 600-700 cycles of copy and issue whatever its width), so the widest tile does the most MMA
+// work per stage; measured against 128, 160 and 192 on the 7B prefill, it is the fastest.
+constexpr int kPBn = 256;
 
 static size_t pgemm_stage_bytes(int bn) { return (size_t)kABytes + (size_t)bn * kBK * 2; }
 static int pgemm_stages(int bn) {
@@ -1096,7 +1039,6 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
 
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static bool g_gemm_persistent = true;  // VT_GEMM_PERSISTENT=0 keeps every GEMM on k_gemm
-static int g_pgemm_clusters[5];        // co-resident clusters of 2 and 4 persistent-GEMM CTAs
 constexpr int kMaxSplit = 4;
 static int g_split_clusters[kMaxSplit + 1];  // co-resident clusters of S GEMM CTAs (index S)
 
@@ -1139,25 +1081,6 @@ cudaError_t init_prefill_kernels() {
     {
         const char* v = getenv("VT_GEMM_PERSISTENT");
         g_gemm_persistent = !(v && v[0] == '0');
-    }
-    for (int cs = 2; cs <= 4; cs += 2) {
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(cs * 64);
-        cfg.blockDim = dim3(kGemmThreads);
-        cfg.dynamicSmemBytes = kPGemmSmem - 1024;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = cs;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        int nc = 0;
-        if (cudaOccupancyMaxActiveClusters(&nc, k_gemm_p<kGemmF32>, &cfg) != cudaSuccess) {
-            cudaGetLastError();
-            nc = 0;
-        }
-        g_pgemm_clusters[cs] = nc;
     }
     if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)prefill_attn_smem<128>())) != cudaSuccess)
@@ -1229,22 +1152,16 @@ struct GemmSpec {
 };
 
 
-// The grouped GEMMs of `specs` (all with m rows) as one persistent launch.  B maps are encoded
-// with the chosen tile width as their box height.
+// The grouped GEMMs of `specs` (all with m rows) as one persistent launch: one CTA per SM, or
+// one per tile when there are fewer tiles.
 template <int EPI>
 static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaStream_t st, std::string* err) {
     PGemmGroup G{};
     G.n_groups = ng;
     G.tiles_m = (m + kBM - 1) / kBM;
-    // the row tiles that share a weight tile form a cluster and load each B tile once
-    G.csize = (G.tiles_m % 4 == 0 && g_pgemm_clusters[4] > 0) ? 4 : ((G.tiles_m % 2 == 0 && g_pgemm_clusters[2] > 0) ? 2 : 1);
-    const int clusters = G.csize == 1 ? (g_num_sms > 0 ? g_num_sms : 148) : g_pgemm_clusters[G.csize];
-    int ns[kGemmGroups];
-    for (int g = 0; g < ng; ++g) ns[g] = specs[g].n;
-    int total = 0;
-    G.bn = choose_bn(ns, ng, G.tiles_m / G.csize, clusters, &total);
-    G.total_units = total;
+    G.bn = kPBn;
     G.stages = pgemm_stages(G.bn);
+    const int ctas = g_num_sms > 0 ? g_num_sms : 148;
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
         const GemmSpec& sp = specs[g];
@@ -1253,7 +1170,7 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
             return VT_ERR_INVALID_ARG;
         }
         if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) ||
-            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn / G.csize, err))
+            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn, err))
             return VT_ERR_INVALID_ARG;
         GemmArgs& a = G.a[g];
         a = sp.base;
@@ -1263,21 +1180,15 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
         a.ldb = sp.ldb;
         a.k_tiles = (sp.k + kBK - 1) / kBK;
         a.kb_wrap = sp.kb > 0 ? sp.kb / kBK : 0;
-        acc += (G.tiles_m / G.csize) * ((sp.n + G.bn - 1) / G.bn);
+        acc += G.tiles_m * ((sp.n + G.bn - 1) / G.bn);
         G.tile_end[g] = acc;
     }
+    G.total_tiles = acc;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(G.csize * std::min(total, clusters)));
+    cfg.gridDim = dim3((unsigned)std::min(acc, ctas));
     cfg.blockDim = dim3(kGemmThreads);
     cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn) + 256;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)G.csize;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = G.csize > 1 ? 1 : 0;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_p<EPI>, G);
     if (e != cudaSuccess) {
         *err = std::string("persistent GEMM launch failed: ") + cudaGetErrorString(e);
