@@ -66,6 +66,26 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
     return false;
 }
 
+// Cluster forms: an arrival on the mbarrier at cluster address `bar` (this CTA's or a peer's),
+// releasing this thread's prior writes at cluster scope, and a bounded wait on this CTA's
+// barrier that acquires at cluster scope (for arrivals that come from a peer).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+        uint32_t ok;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        if (ok) return true;
+    }
+    return false;
+}
+
 // ------------------------------------------------------------------ bulk asynchronous copies
 // Global -> shared copy of `bytes` (multiple of 16, both addresses 16-byte aligned) completing
 // as transaction bytes on `bar` (the CTA's own shared memory, addressed in the cluster window).

@@ -42,6 +42,17 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+// The same load issued by either CTA of a pair that shares one MMA (cta_group::2): the box lands in
+// this CTA's shared memory and its bytes complete on the mbarrier at cluster address `bar`, which
+// may be in the peer CTA.
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
 // 16-byte store into the shared memory of a CTA of the cluster (address from mapa).
 __device__ __forceinline__ void dsmem_st4(uint32_t addr, float a, float b, float c, float d) {
     asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
@@ -58,6 +69,17 @@ __device__ __forceinline__ void tmem_relinquish() {
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
+// Pair forms (cta_group::2): one warp of each CTA of the pair takes part; both get the same address.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -70,6 +92,32 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// One MMA over a CTA pair (issued by the even CTA): A rows [0, M/2) from this CTA's shared memory
+// and [M/2, M) from the peer's, B rows [0, N/2) here and [N/2, N) in the peer, both at the same
+// offsets; each CTA's tensor memory receives its M/2 rows of D.
+__device__ __forceinline__ void mma_f16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrives once on the mbarrier at `bar`'s offset in both CTAs of the pair when every pair MMA
+// issued so far has completed.
+__device__ __forceinline__ void mma_commit_pair_both(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+}
+// Arrives once on this CTA's `bar` when every pair MMA issued so far has completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
 // Arrives once on `bar` when every MMA this thread issued so far has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
@@ -567,18 +615,18 @@ constexpr int kPTmemCols = 512;  // two accumulators
 constexpr size_t kPGemmSmem = 227 * 1024;
 
 struct PGemmGroup {
-    int n_groups, tiles_m, bn, total_tiles, stages;
+    int n_groups, tiles_m, tm, bn, total_tiles, stages;
     int tile_end[kGemmGroups];  // cumulative tiles (tiles_m x column tiles of each group)
     CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
     GemmArgs a[kGemmGroups];
 };
 
-// Tile t of the group: the row tile is the fastest index.
+// Tile t of the group: the row tile (tm rows: 128, or 256 for a CTA pair) is the fastest index.
 __device__ __forceinline__ void ptile(const PGemmGroup& G, int t, int& g, int& m0, int& n0) {
     g = 0;
     while (g + 1 < G.n_groups && t >= G.tile_end[g]) ++g;
     const int u = t - (g > 0 ? G.tile_end[g - 1] : 0);
-    m0 = (u % G.tiles_m) * kBM;
+    m0 = (u % G.tiles_m) * G.tm;
     n0 = (u / G.tiles_m) * G.bn;
 }
 
@@ -647,12 +695,12 @@ __device__ __forceinline__ void pepi_chunk(const GemmArgs& a, int row, int col0,
     }
 }
 
-template <int EPI>
+template <int EPI, int CG>
 __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constant__ PGemmGroup G) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    const int S = G.stages, BN = G.bn;
-    const uint32_t b_bytes = (uint32_t)BN * kBK * 2, stage_bytes = (uint32_t)kABytes + b_bytes;
+    const int S = G.stages, BN = G.bn, BNc = BN / CG;  // BNc: rows of each B tile this CTA holds
+    const uint32_t b_bytes = (uint32_t)BNc * kBK * 2, stage_bytes = (uint32_t)kABytes + b_bytes;
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
     uint64_t* empty = full + kPStages;
     uint64_t* tfull = empty + kPStages;  // [2] accumulator b holds a finished tile
@@ -662,7 +710,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
     __shared__ int s_err;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int cid = (int)blockIdx.x, nctas = (int)gridDim.x;
+    // CG = 2: the two CTAs of a cluster share each tile; rank 0 issues the MMAs.  Its `full`
+    // barriers count both CTAs' bytes and its `tempty` barriers both CTAs' epilogue warps; the
+    // commits that release a stage or a finished accumulator arrive in both CTAs.
+    const int rank = CG == 2 ? (int)cluster_rank() : 0;
+    const int cid = (int)blockIdx.x / CG, nctas = (int)gridDim.x / CG;
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
@@ -670,18 +722,24 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull[b], 1);
-            mbar_init(&tempty[b], 4);
+            mbar_init(&tempty[b], 4 * CG);
         }
         mbar_init(done, 1);
         s_err = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
-        tc::tmem_alloc(tmem_slot, kPTmemCols);
-        tc::tmem_relinquish();
+        if constexpr (CG == 2) {
+            tc::tmem_alloc_pair(tmem_slot, kPTmemCols);
+            tc::tmem_relinquish_pair();
+        } else {
+            tc::tmem_alloc(tmem_slot, kPTmemCols);
+            tc::tmem_relinquish();
+        }
     }
     tc::fence_before();
-    __syncthreads();
+    if constexpr (CG == 2) cluster_sync();  // the peer's barriers exist before any copy or commit reaches them
+    else __syncthreads();
     tc::fence_after();
     const uint32_t tmem = *tmem_slot;
     uint32_t* status = G.a[0].status;
@@ -689,6 +747,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
         s_err = 1;
         set_status(status, VT_DEV_WAIT_TIMEOUT);
     };
+    // cluster addresses of rank 0's barriers (this CTA's own when CG = 1)
+    const uint32_t full0 = CG == 2 ? dsmem_addr(full, 0) : smem_u32(full);
+    const uint32_t tempty0 = CG == 2 ? dsmem_addr(tempty, 0) : smem_u32(tempty);
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -707,18 +768,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                     }
                     if (*(volatile int*)&s_err) break;
                     uint8_t* st = smem + (size_t)s * stage_bytes;
-                    mbar_arrive_expect_tx(&full[s], stage_bytes);
-                    tc::tma_load_2d(st, &G.ta[g], kt * kBK, m0, &full[s]);
-                    tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
+                    if constexpr (CG == 2) {
+                        // rank 0 expects both CTAs' bytes; each CTA loads its own A rows and B half
+                        if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * stage_bytes);
+                        const uint32_t fb = full0 + (uint32_t)s * 8;
+                        tc::tma_load_2d_pair(st, &G.ta[g], kt * kBK, m0 + rank * kBM, fb);
+                        tc::tma_load_2d_pair(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0 + rank * BNc, fb);
+                    } else {
+                        mbar_arrive_expect_tx(&full[s], stage_bytes);
+                        tc::tma_load_2d(st, &G.ta[g], kt * kBK, m0, &full[s]);
+                        tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
+                    }
                 }
             }
-            // no copy may be in flight when the CTA ends
-            for (uint32_t i = k > (uint32_t)S ? k - S : 0; i < k; ++i)
-                if (!mbar_wait(&full[i % S], (i / S) & 1)) set_status(status, VT_DEV_WAIT_TIMEOUT);
+            // no copy may be in flight when the CTA ends (rank 0's barriers count both CTAs' copies;
+            // the final cluster barrier keeps the peer until then)
+            if (rank == 0)
+                for (uint32_t i = k > (uint32_t)S ? k - S : 0; i < k; ++i)
+                    if (!mbar_wait(&full[i % S], (i / S) & 1)) set_status(status, VT_DEV_WAIT_TIMEOUT);
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        // ------------------------------------------------------------ MMA issuer (rank 0)
+        if (lane == 0 && rank == 0) {
             uint32_t k = 0;
             int it = 0;
             for (int t = cid; t < G.total_tiles && !*(volatile int*)&s_err; t += nctas, ++it) {
@@ -726,13 +797,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                 ptile(G, t, g, m0, n0);
                 const GemmArgs& a = G.a[g];
                 const int buf = it & 1;
-                if (it >= 2 && !mbar_wait(&tempty[buf], ((it >> 1) - 1) & 1)) {
+                if (it >= 2 && !(CG == 2 ? mbar_wait_cluster(&tempty[buf], ((it >> 1) - 1) & 1)
+                                         : mbar_wait(&tempty[buf], ((it >> 1) - 1) & 1))) {
                     abort_cta();
                     break;
                 }
                 tc::fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
-                const uint32_t idesc = tc::idesc_f16(kBM, BN);
+                const uint32_t idesc = tc::idesc_f16(kBM * CG, BN);
                 bool ok = true;
                 for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
                     const int s = (int)(k % (uint32_t)S);
@@ -743,18 +815,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                     tc::fence_after();
                     const uint32_t sa = smem_u32(smem + (size_t)s * stage_bytes), sb = sa + kABytes;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk)
-                        tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
-                                    (kt | kk) != 0);
-                    tc::mma_commit(&empty[s]);
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        if constexpr (CG == 2)
+                            tc::mma_f16_pair(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
+                                             (kt | kk) != 0);
+                        else
+                            tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
+                                        (kt | kk) != 0);
+                    }
+                    if constexpr (CG == 2) tc::mma_commit_pair_both(&empty[s]);
+                    else tc::mma_commit(&empty[s]);
                 }
                 if (!ok) {
                     abort_cta();
                     break;
                 }
-                tc::mma_commit(&tfull[buf]);
+                if constexpr (CG == 2) tc::mma_commit_pair_both(&tfull[buf]);
+                else tc::mma_commit(&tfull[buf]);
             }
-            tc::mma_commit(done);
+            if constexpr (CG == 2) tc::mma_commit_pair(done);
+            else tc::mma_commit(done);
             if (!mbar_wait(done, 0)) set_status(status, VT_DEV_WAIT_TIMEOUT);
         }
     } else {
@@ -774,7 +854,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                 break;
             }
             tc::fence_after();
-            const int row = m0 + sub * 32 + lane;
+            const int row = m0 + rank * kBM + sub * 32 + lane;
             int pos = 0;
             bool row_ok = row < a.m;
             if constexpr (EPI == kGemmQkv) {
@@ -793,27 +873,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
             }
             tc::fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[buf]);
+            if (lane == 0) {
+                if constexpr (CG == 2) mbar_arrive_cluster(tempty0 + (uint32_t)buf * 8);
+                else mbar_arrive(&tempty[buf]);
+            }
         }
     }
     tc::fence_before();
-    __syncthreads();
+    // no CTA of a pair leaves while the other may still copy into its barriers or write its accumulators
+    if constexpr (CG == 2) cluster_sync();
+    else __syncthreads();
     if (warp == 1) {
         tc::fence_after();
-        tc::tmem_dealloc(tmem, kPTmemCols);
+        if constexpr (CG == 2) tc::tmem_dealloc_pair(tmem, kPTmemCols);
+        else tc::tmem_dealloc(tmem, kPTmemCols);
     }
 }
 
-// Tile width of the persistent GEMM: 128 x 256.  Per k-tile the ring moves the A and B boxes
-// through shared memory at a rate that does not grow with a narrower B (measured: a stage costs
-// about 600-700 cycles of copy and issue whatever its width), so the widest tile does the most MMA
-// work per stage; measured against 128, 160 and 192 on the 7B prefill, it is the fastest.
+// Tile width of the single-CTA persistent GEMM: 128 x 256.  Its ring moves 384 lines of 128 bytes
+// (A 128 + B 256) per k-tile through shared memory, which the copy engine delivers at about half a
+// line per cycle (measured: a stage of that size fills in 600-700 cycles), against 512 cycles of
+// MMA; narrower tiles do less MMA work per line, so the widest is the fastest (measured against
+// 128, 160 and 192 on the 7B prefill).
 constexpr int kPBn = 256;
 
-static size_t pgemm_stage_bytes(int bn) { return (size_t)kABytes + (size_t)bn * kBK * 2; }
-static int pgemm_stages(int bn) {
+// bn_cta: rows of the B tile one CTA holds (the tile width, or half of it for a CTA pair)
+static size_t pgemm_stage_bytes(int bn_cta) { return (size_t)kABytes + (size_t)bn_cta * kBK * 2; }
+static int pgemm_stages(int bn_cta) {
     const size_t room = kPGemmSmem - 1024 - 256;
-    int s = (int)(room / pgemm_stage_bytes(bn));
+    int s = (int)(room / pgemm_stage_bytes(bn_cta));
     return s > kPStages ? kPStages : s;
 }
 
@@ -1039,6 +1127,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
 
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static bool g_gemm_persistent = true;  // VT_GEMM_PERSISTENT=0 keeps every GEMM on k_gemm
+static int g_pgemm_pairs = 0;          // co-resident CTA pairs of the persistent GEMM (0: single CTAs)
 constexpr int kMaxSplit = 4;
 static int g_split_clusters[kMaxSplit + 1];  // co-resident clusters of S GEMM CTAs (index S)
 
@@ -1075,12 +1164,35 @@ cudaError_t init_prefill_kernels() {
         }
         g_split_clusters[sp] = nc;
     }
-    for (auto f : {k_gemm_p<kGemmF32>, k_gemm_p<kGemmQkv>, k_gemm_p<kGemmSwiglu>})
+    for (auto f : {k_gemm_p<kGemmF32, 1>, k_gemm_p<kGemmQkv, 1>, k_gemm_p<kGemmSwiglu, 1>, k_gemm_p<kGemmF32, 2>,
+                   k_gemm_p<kGemmQkv, 2>, k_gemm_p<kGemmSwiglu, 2>})
         if ((e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(kPGemmSmem - 1024))) != cudaSuccess)
             return e;
     {
         const char* v = getenv("VT_GEMM_PERSISTENT");
         g_gemm_persistent = !(v && v[0] == '0');
+        // VT_GEMM_PAIR=0 keeps the persistent GEMM on single CTAs
+        const char* pv = getenv("VT_GEMM_PAIR");
+        g_pgemm_pairs = 0;
+        if (!(pv && pv[0] == '0')) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(2 * 64);
+            cfg.blockDim = dim3(kGemmThreads);
+            cfg.dynamicSmemBytes = kPGemmSmem - 1024;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = 2;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            int nc = 0;
+            if (cudaOccupancyMaxActiveClusters(&nc, k_gemm_p<kGemmF32, 2>, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                nc = 0;
+            }
+            g_pgemm_pairs = nc;
+        }
     }
     if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)prefill_attn_smem<128>())) != cudaSuccess)
@@ -1152,16 +1264,37 @@ struct GemmSpec {
 };
 
 
-// The grouped GEMMs of `specs` (all with m rows) as one persistent launch: one CTA per SM, or
-// one per tile when there are fewer tiles.
-template <int EPI>
+// Width of a CTA-pair tile (256 rows): per k-tile each CTA moves 128 + w/2 lines of 128 bytes
+// through its ring (about half a line per cycle) while the pair's MMAs take 2w cycles, so a k-tile
+// costs max(2w, 256 + w) cycles; the width is the one whose rounds of tiles over the co-resident
+// pairs cost least (ties to the wider).
+static int choose_pair_bn(const GemmSpec* specs, int ng, int tiles_m, int pairs) {
+    int best = 256;
+    long best_cost = -1;
+    for (int w = 256; w >= 128; w -= 32) {
+        int tiles = 0;
+        for (int g = 0; g < ng; ++g) tiles += tiles_m * ((specs[g].n + w - 1) / w);
+        const long rounds = (tiles + pairs - 1) / pairs;
+        const long cost = rounds * (long)std::max(2 * w, 256 + w);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = w;
+        }
+    }
+    return best;
+}
+
+// The grouped GEMMs of `specs` (all with m rows) as one persistent launch: one CTA (CG = 1) or
+// one CTA pair (CG = 2, 256-row tiles) per SM or SM pair, or one per tile when there are fewer.
+template <int EPI, int CG>
 static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaStream_t st, std::string* err) {
     PGemmGroup G{};
     G.n_groups = ng;
-    G.tiles_m = (m + kBM - 1) / kBM;
-    G.bn = kPBn;
-    G.stages = pgemm_stages(G.bn);
-    const int ctas = g_num_sms > 0 ? g_num_sms : 148;
+    G.tm = kBM * CG;
+    G.tiles_m = (m + G.tm - 1) / G.tm;
+    const int slots = CG == 2 ? g_pgemm_pairs : (g_num_sms > 0 ? g_num_sms : 148);
+    G.bn = CG == 2 ? choose_pair_bn(specs, ng, G.tiles_m, slots) : kPBn;
+    G.stages = pgemm_stages(G.bn / CG);
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
         const GemmSpec& sp = specs[g];
@@ -1170,7 +1303,7 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
             return VT_ERR_INVALID_ARG;
         }
         if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) ||
-            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn, err))
+            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn / CG, err))
             return VT_ERR_INVALID_ARG;
         GemmArgs& a = G.a[g];
         a = sp.base;
@@ -1185,11 +1318,18 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
     }
     G.total_tiles = acc;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)std::min(acc, ctas));
+    cfg.gridDim = dim3((unsigned)(CG * std::min(acc, slots)));
     cfg.blockDim = dim3(kGemmThreads);
-    cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn) + 256;
+    cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn / CG) + 256;
     cfg.stream = st;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_p<EPI>, G);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CG;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = CG == 2 ? 1 : 0;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_p<EPI, CG>, G);
     if (e != cudaSuccess) {
         *err = std::string("persistent GEMM launch failed: ") + cudaGetErrorString(e);
         return VT_ERR_CUDA;
@@ -1209,7 +1349,8 @@ static vt_status run_gemm_group(const GemmSpec* specs, int n_specs, int m, cudaS
             int tiles = 0;
             for (int g = 0; g < ng; ++g) tiles += ((m + kBM - 1) / kBM) * ((specs[g0 + g].n + kBN - 1) / kBN);
             if (g_gemm_persistent && 2 * tiles >= (g_num_sms > 0 ? g_num_sms : 148)) {
-                const vt_status r = run_gemm_persistent<EPI>(specs + g0, ng, m, st, err);
+                const vt_status r = g_pgemm_pairs > 0 ? run_gemm_persistent<EPI, 2>(specs + g0, ng, m, st, err)
+                                                      : run_gemm_persistent<EPI, 1>(specs + g0, ng, m, st, err);
                 if (r != VT_OK) return r;
                 continue;
             }
