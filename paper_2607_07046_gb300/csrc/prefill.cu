@@ -42,6 +42,23 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+// 3-D tiled TMA load: box (0, y, z) of a map whose third dimension steps one 64-column k-tile, so
+// one box brings several consecutive k-tiles of the same rows (one swizzled tile after the other).
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int y, int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(
+            smem_u32(dst)),
+        "l"(map), "r"(0), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* map, int y, int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+        "%4}], [%5];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(0), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+
 // The same load issued by either CTA of a pair that shares one MMA (cta_group::2): the box lands in
 // this CTA's shared memory and its bytes complete on the mbarrier at cluster address `bar`, which
 // may be in the peer CTA.
@@ -594,18 +611,24 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
 
 // ================================================================== persistent tensor-core GEMM
 //
-// The grouped projections of a block (every shard's GEMM of one kind) as one persistent launch:
-// one CTA per SM walks output tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of the group in
-// an order where the 128-row tile is the fastest index, so the tiles that share a weight tile run
-// at the same time and the weights leave DRAM once.  Tiles are 128 x 256.
-//   warp 0   TMA producer: A (128 x 64) and B (BN x 64) boxes into a ring of stages (as many as
-//            fit in shared memory), one k-tile per stage, continuing across tiles;
-//   warp 1   tensor memory (512 columns: two accumulators of up to 256) and the MMA thread: the
-//            tile's k-tiles into accumulator (tile index & 1), then a commit that releases it to
-//            the epilogue;
+// The grouped projections of a block (every shard's GEMM of one kind) as one persistent launch.
+// Each worker walks output tiles t = w, w + workers, ... of the group in an order where the row
+// tile is the fastest index, so the tiles that share a weight tile run at the same time and the
+// weights leave DRAM once.  A worker is a pair of CTAs on two SMs (CG = 2: 256 x BN tiles, one
+// tcgen05.mma cta_group::2 over both CTAs' shared memory, each CTA holding 128 rows of A, half of
+// B and its 128 rows of the accumulator) or a single CTA (CG = 1: 128 x 256 tiles).
+//   warp 0   TMA producer: per stage, one box of A rows and one of B rows, each bringing two
+//            consecutive k-tiles (3-D tensor maps) or one, into a ring of stages as deep as shared
+//            memory allows, continuing across tiles.  The copy engine's cost is per box, so two
+//            k-tiles per box nearly halve it;
+//   warp 1   tensor memory (512 columns: two accumulators of up to 256) and, in the CTA of rank 0,
+//            the MMA thread: the tile's k-tiles into accumulator (tile index & 1), a commit per
+//            stage that frees it in both CTAs, and a commit that releases the accumulator to both
+//            CTAs' epilogues;
 //   warps 2-5 epilogue: each warp reads its 32 accumulator lanes (rows) in chunks of 32 columns
-//            and writes the tile's outputs from registers; after the last chunk it hands the
-//            accumulator back, so the epilogue of one tile overlaps the MMAs of the next.
+//            and writes the tile's outputs (fp32 partials through a shared-memory turn so each
+//            store writes whole rows); after the last chunk it hands the accumulator back, so the
+//            epilogue of one tile overlaps the MMAs of the next.
 // Every wait is bounded; on a timeout the CTA sets VT_DEV_WAIT_TIMEOUT and an abort flag, every
 // role stops at its next wait, copies and MMAs in flight are waited for (bounded), and tensor
 // memory is freed.
@@ -613,9 +636,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm(const __grid_constant_
 constexpr int kPStages = 8;     // most ring stages
 constexpr int kPTmemCols = 512;  // two accumulators
 constexpr size_t kPGemmSmem = 227 * 1024;
+constexpr size_t kPBarBytes = 256;                    // barriers and the tensor-memory slot
+constexpr size_t kPEpiBytes = 4 * 32 * 33 * 4;        // fp32 epilogue staging, one 32 x 33 block per warp
 
 struct PGemmGroup {
     int n_groups, tiles_m, tm, bn, total_tiles, stages;
+    int kts;  // k-tiles per stage: 2 (one 3-D box per operand brings two) or 1
     int tile_end[kGemmGroups];  // cumulative tiles (tiles_m x column tiles of each group)
     CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
     GemmArgs a[kGemmGroups];
@@ -689,10 +715,40 @@ __device__ __forceinline__ void pepi_chunk(const GemmArgs& a, int row, int col0,
         __half* dst = a.u + (size_t)row * a.ldu + a.ushift + col0 / 2;
         if (col0 == 0)
             for (int j = 0; j < a.ushift; ++j) dst[j - a.ushift] = __float2half_rn(0.f);
+        if (col0 + 32 <= a.n && ((uintptr_t)dst & 15) == 0) {
+            uint32_t w[8];
 #pragma unroll
-        for (int p = 0; p < 16; ++p)
-            if (col0 + 2 * p < a.n) dst[p] = __float2half_rn(silu(__uint_as_float(r[2 * p])) * __uint_as_float(r[2 * p + 1]));
+            for (int p = 0; p < 8; ++p) {
+                const __half2 h = __floats2half2_rn(silu(__uint_as_float(r[4 * p])) * __uint_as_float(r[4 * p + 1]),
+                                                    silu(__uint_as_float(r[4 * p + 2])) * __uint_as_float(r[4 * p + 3]));
+                w[p] = *reinterpret_cast<const uint32_t*>(&h);
+            }
+            reinterpret_cast<uint4*>(dst)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+            reinterpret_cast<uint4*>(dst)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        } else {
+#pragma unroll
+            for (int p = 0; p < 16; ++p)
+                if (col0 + 2 * p < a.n)
+                    dst[p] = __float2half_rn(silu(__uint_as_float(r[2 * p])) * __uint_as_float(r[2 * p + 1]));
+        }
     }
+}
+
+// fp32 epilogue of a warp's 32 rows [row0, row0 + 32) x 32 columns [col0, col0 + 32): lane l holds
+// row row0 + l.  The chunk is turned around in shared memory (`stg`, 32 x 33 floats, padded so
+// both the row-wise writes and the column-wise reads hit 32 distinct banks), then each store
+// instruction writes one row's 32 consecutive floats (one 128-byte line) instead of 32 scattered
+// 16-byte pieces.
+__device__ __forceinline__ void pepi_f32_rows(const GemmArgs& a, float* stg, int row0, int col0, const uint32_t (&r)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(r[j]);
+    __syncwarp();
+    const int col = col0 + lane;
+    const int rows = min(32, a.m - row0);
+    if (col < a.n)
+        for (int i = 0; i < rows; ++i) a.c[(size_t)(row0 + i) * a.ldc + col] = stg[i * 33 + lane];
+    __syncwarp();
 }
 
 template <int EPI, int CG>
@@ -700,13 +756,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int S = G.stages, BN = G.bn, BNc = BN / CG;  // BNc: rows of each B tile this CTA holds
-    const uint32_t b_bytes = (uint32_t)BNc * kBK * 2, stage_bytes = (uint32_t)kABytes + b_bytes;
+    const int T = G.kts;
+    // stage: T A tiles (128 x 64) then T B tiles (BNc x 64), each a 128-byte-swizzled K-major tile
+    const uint32_t a_bytes = (uint32_t)(T * kABytes), b_tile = (uint32_t)BNc * kBK * 2;
+    const uint32_t stage_bytes = a_bytes + (uint32_t)T * b_tile;
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
     uint64_t* empty = full + kPStages;
     uint64_t* tfull = empty + kPStages;  // [2] accumulator b holds a finished tile
     uint64_t* tempty = tfull + 2;        // [2] accumulator b was read by the epilogue
     uint64_t* done = tempty + 2;         // every MMA issued by this CTA has completed
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+    float* epi_stage = reinterpret_cast<float*>(smem + (size_t)S * stage_bytes + kPBarBytes);  // [4][32][33]
     __shared__ int s_err;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -760,7 +820,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                 int g, m0, n0;
                 ptile(G, t, g, m0, n0);
                 const GemmArgs& a = G.a[g];
-                for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
+                for (int kt = 0; kt < a.k_tiles; kt += T, ++k) {
                     const int s = (int)(k % (uint32_t)S);
                     if (k >= (uint32_t)S && !mbar_wait(&empty[s], ((k / S) - 1) & 1)) {
                         abort_cta();
@@ -768,16 +828,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                     }
                     if (*(volatile int*)&s_err) break;
                     uint8_t* st = smem + (size_t)s * stage_bytes;
+                    // a 3-D box past the last k-tile is filled with zeros and still counts its bytes
+                    const uint32_t fb = full0 + (uint32_t)s * 8;
+                    const int ya = m0 + rank * kBM, yb = n0 + rank * BNc, kb = bk_tile(a, kt);
                     if constexpr (CG == 2) {
                         // rank 0 expects both CTAs' bytes; each CTA loads its own A rows and B half
                         if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * stage_bytes);
-                        const uint32_t fb = full0 + (uint32_t)s * 8;
-                        tc::tma_load_2d_pair(st, &G.ta[g], kt * kBK, m0 + rank * kBM, fb);
-                        tc::tma_load_2d_pair(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0 + rank * BNc, fb);
+                        if (T == 2) {
+                            tc::tma_load_3d_pair(st, &G.ta[g], ya, kt, fb);
+                            tc::tma_load_3d_pair(st + a_bytes, &G.tb[g], yb, kb, fb);
+                        } else {
+                            tc::tma_load_2d_pair(st, &G.ta[g], kt * kBK, ya, fb);
+                            tc::tma_load_2d_pair(st + a_bytes, &G.tb[g], kb * kBK, yb, fb);
+                        }
                     } else {
                         mbar_arrive_expect_tx(&full[s], stage_bytes);
-                        tc::tma_load_2d(st, &G.ta[g], kt * kBK, m0, &full[s]);
-                        tc::tma_load_2d(st + kABytes, &G.tb[g], bk_tile(a, kt) * kBK, n0, &full[s]);
+                        if (T == 2) {
+                            tc::tma_load_3d(st, &G.ta[g], ya, kt, fb);
+                            tc::tma_load_3d(st + a_bytes, &G.tb[g], yb, kb, fb);
+                        } else {
+                            tc::tma_load_2d(st, &G.ta[g], kt * kBK, ya, &full[s]);
+                            tc::tma_load_2d(st + a_bytes, &G.tb[g], kb * kBK, yb, &full[s]);
+                        }
                     }
                 }
             }
@@ -806,22 +878,25 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
                 const uint32_t idesc = tc::idesc_f16(kBM * CG, BN);
                 bool ok = true;
-                for (int kt = 0; kt < a.k_tiles; ++kt, ++k) {
+                for (int kt = 0; kt < a.k_tiles; kt += T, ++k) {
                     const int s = (int)(k % (uint32_t)S);
                     if (!mbar_wait(&full[s], (k / S) & 1)) {
                         ok = false;
                         break;
                     }
                     tc::fence_after();
-                    const uint32_t sa = smem_u32(smem + (size_t)s * stage_bytes), sb = sa + kABytes;
+                    const uint32_t s0 = smem_u32(smem + (size_t)s * stage_bytes);
+                    for (int j = 0; j < T && kt + j < a.k_tiles; ++j) {
+                        const uint32_t sa = s0 + (uint32_t)j * kABytes, sb = s0 + a_bytes + (uint32_t)j * b_tile;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        if constexpr (CG == 2)
-                            tc::mma_f16_pair(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
-                                             (kt | kk) != 0);
-                        else
-                            tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
-                                        (kt | kk) != 0);
+                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                            if constexpr (CG == 2)
+                                tc::mma_f16_pair(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
+                                                 (kt + j | kk) != 0);
+                            else
+                                tc::mma_f16(d_tmem, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32), idesc,
+                                            (kt + j | kk) != 0);
+                        }
                     }
                     if constexpr (CG == 2) tc::mma_commit_pair_both(&empty[s]);
                     else tc::mma_commit(&empty[s]);
@@ -869,7 +944,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
                 uint32_t r[32];
                 tc::tmem_ld32(base + (uint32_t)c, r);  // warp-collective: every lane takes part
                 tc::tmem_ld_wait();
-                if (row_ok && n0 + c < a.n) pepi_chunk<EPI>(a, row, n0 + c, r, pos);
+                if constexpr (EPI == kGemmF32) {
+                    if (n0 + c < a.n) pepi_f32_rows(a, epi_stage + sub * (32 * 33), row - lane, n0 + c, r);
+                } else {
+                    if (row_ok && n0 + c < a.n) pepi_chunk<EPI>(a, row, n0 + c, r, pos);
+                }
             }
             tc::fence_before();
             __syncwarp();
@@ -897,11 +976,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1) k_gemm_p(const __grid_constan
 // 128, 160 and 192 on the 7B prefill).
 constexpr int kPBn = 256;
 
-// bn_cta: rows of the B tile one CTA holds (the tile width, or half of it for a CTA pair)
-static size_t pgemm_stage_bytes(int bn_cta) { return (size_t)kABytes + (size_t)bn_cta * kBK * 2; }
-static int pgemm_stages(int bn_cta) {
-    const size_t room = kPGemmSmem - 1024 - 256;
-    int s = (int)(room / pgemm_stage_bytes(bn_cta));
+// bn_cta: rows of the B tile one CTA holds (the tile width, or half of it for a CTA pair);
+// kts: k-tiles per stage
+static size_t pgemm_stage_bytes(int bn_cta, int kts) { return (size_t)kts * ((size_t)kABytes + (size_t)bn_cta * kBK * 2); }
+static int pgemm_stages(int bn_cta, int kts) {
+    // the launch may use kPGemmSmem - 1024 bytes, 1024 of them lost to aligning the ring
+    const size_t room = kPGemmSmem - 2048 - kPBarBytes - kPEpiBytes;
+    int s = (int)(room / pgemm_stage_bytes(bn_cta, kts));
     return s > kPStages ? kPStages : s;
 }
 
@@ -1228,6 +1309,33 @@ static bool make_map(CUtensorMap* map, const void* base, int64_t inner, int64_t 
     return true;
 }
 
+// The same operand as a 3-D map {64, rows, inner / 64} whose third dimension steps one k-tile
+// (128 bytes), read in boxes of 64 x box_rows x 2: two consecutive k-tiles per copy.  inner must
+// be a multiple of 64 (the box does not stop at the row's end).
+static bool make_map_k2(CUtensorMap* map, const void* base, int64_t inner, int64_t rows, int64_t ld, int box_rows,
+                        std::string* err) {
+    if (!g_encode) {
+        *err = "the tensor-map encoder is not available";
+        return false;
+    }
+    if (((uintptr_t)base & 15) != 0 || (ld * 2) % 16 != 0 || inner % kBK != 0) {
+        *err = "a GEMM operand is not 16-byte aligned or its K is not a multiple of 64";
+        return false;
+    }
+    const cuuint64_t dims[3] = {(cuuint64_t)kBK, (cuuint64_t)rows, (cuuint64_t)(inner / kBK)};
+    const cuuint64_t strides[2] = {(cuuint64_t)ld * 2, (cuuint64_t)kBK * 2};
+    const cuuint32_t box[3] = {(cuuint32_t)kBK, (cuuint32_t)box_rows, 2};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+                                estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled (3-D) failed (" + std::to_string((int)r) + ")";
+        return false;
+    }
+    return true;
+}
+
 // Split factor for `tiles` output tiles of `k_tiles` k-tiles, from a time model of one launch:
 // per wave, a fixed cost (first loads, epilogue) plus the k-tiles of one split; with S > 1, the
 // cluster reduction of the accumulators.  The constants are measured on GB300 (microseconds).
@@ -1264,18 +1372,19 @@ struct GemmSpec {
 };
 
 
-// Width of a CTA-pair tile (256 rows): per k-tile each CTA moves 128 + w/2 lines of 128 bytes
-// through its ring (about half a line per cycle) while the pair's MMAs take 2w cycles, so a k-tile
-// costs max(2w, 256 + w) cycles; the width is the one whose rounds of tiles over the co-resident
-// pairs cost least (ties to the wider).
-static int choose_pair_bn(const GemmSpec* specs, int ng, int tiles_m, int pairs) {
+// Width of a CTA-pair tile (256 rows).  The copy engine's cost is per box rather than per byte
+// (measured on GB300: a ring stage of one A box and one B box turns over in about 1000 cycles
+// whether the boxes carry one k-tile or two), so a k-tile costs about 500 cycles of copying with
+// two k-tiles per box, 900 with one, against 2w cycles of MMA; the width is the one whose rounds
+// of tiles over the co-resident pairs cost least (ties to the wider).
+static int choose_pair_bn(const GemmSpec* specs, int ng, int tiles_m, int pairs, int kts) {
     int best = 256;
     long best_cost = -1;
     for (int w = 256; w >= 128; w -= 32) {
         int tiles = 0;
         for (int g = 0; g < ng; ++g) tiles += tiles_m * ((specs[g].n + w - 1) / w);
         const long rounds = (tiles + pairs - 1) / pairs;
-        const long cost = rounds * (long)std::max(2 * w, 256 + w);
+        const long cost = rounds * (long)std::max(2 * w, kts == 2 ? 500 : 900);
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;
             best = w;
@@ -1293,8 +1402,13 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
     G.tm = kBM * CG;
     G.tiles_m = (m + G.tm - 1) / G.tm;
     const int slots = CG == 2 ? g_pgemm_pairs : (g_num_sms > 0 ? g_num_sms : 148);
-    G.bn = CG == 2 ? choose_pair_bn(specs, ng, G.tiles_m, slots) : kPBn;
-    G.stages = pgemm_stages(G.bn / CG);
+    // two k-tiles per box needs every K (and the wrap of a split GEMM) in whole pairs of k-tiles'
+    // worth of columns: a 3-D box past K would read the next row instead of zeros
+    G.kts = 2;
+    for (int g = 0; g < ng; ++g)
+        if (specs[g].k % kBK != 0 || (specs[g].kb > 0 && specs[g].kb % (2 * kBK) != 0)) G.kts = 1;
+    G.bn = CG == 2 ? choose_pair_bn(specs, ng, G.tiles_m, slots, G.kts) : kPBn;
+    G.stages = pgemm_stages(G.bn / CG, G.kts);
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
         const GemmSpec& sp = specs[g];
@@ -1302,9 +1416,12 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
             *err = "a split GEMM needs k = 2 kb with kb a multiple of 64";
             return VT_ERR_INVALID_ARG;
         }
-        if (!make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) ||
-            !make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn / CG, err))
-            return VT_ERR_INVALID_ARG;
+        const bool ok = G.kts == 2
+                            ? make_map_k2(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) &&
+                                  make_map_k2(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn / CG, err)
+                            : make_map(&G.ta[g], sp.A, sp.k, m, sp.lda, kBM, err) &&
+                                  make_map(&G.tb[g], sp.B, sp.kb > 0 ? sp.kb : sp.k, sp.n, sp.ldb, G.bn / CG, err);
+        if (!ok) return VT_ERR_INVALID_ARG;
         GemmArgs& a = G.a[g];
         a = sp.base;
         a.m = m;
@@ -1320,7 +1437,7 @@ static vt_status run_gemm_persistent(const GemmSpec* specs, int ng, int m, cudaS
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(CG * std::min(acc, slots)));
     cfg.blockDim = dim3(kGemmThreads);
-    cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn / CG) + 256;
+    cfg.dynamicSmemBytes = 1024 + (size_t)G.stages * pgemm_stage_bytes(G.bn / CG, G.kts) + kPBarBytes + kPEpiBytes;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
