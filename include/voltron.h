@@ -503,6 +503,15 @@ VT_API int32_t vt_decode_token_fused_available(const vt_partition* part, const c
  * Valid after a vt_decode_token that ran fused; VT_ERR_STATE when the partition has no fused
  * kernel. */
 VT_API vt_status vt_token_partials_read(const vt_partition* part, int32_t block, float* host_dst);
+/* Test hook (library plumbing) for the bounded waits of the fused decode-token kernel: in the
+ * next vt_decode_token launches, CTA `cta` (0 <= cta < grid; -1: none) does not publish its
+ * arrival at the launch's first grid barrier, and a grid-barrier wait gives up after
+ * `spin_polls` polls (0: the built-in limit, several seconds).  The other CTAs then give up
+ * waiting, the kernel returns with VT_DEV_WAIT_TIMEOUT in the KV status word and the token's
+ * output and appended K/V undefined (the lengths still advance by one).  vt_kv_status or
+ * vt_partition_status with clear = 1 removes both settings and re-arms the barrier.
+ * Synchronous.  VT_ERR_STATE when the partition has no fused kernel. */
+VT_API vt_status vt_token_test_barrier(vt_partition* part, int32_t cta, uint32_t spin_polls, vt_stream stream);
 /* vt_prefill_tokens (Section 2.1, prefill phase, through the tensor-parallel layers of Section
  * 3.2.1): n prompt rows through every layer (same order as vt_decode_token), then every layer's
  * KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same.  The shards of a

@@ -1846,6 +1846,19 @@ extern "C" vt_status vt_token_partials_read(const vt_partition* p, int32_t block
     return ok();
 }
 
+extern "C" vt_status vt_token_test_barrier(vt_partition* p, int32_t cta, uint32_t spin_polls, vt_stream stream) {
+    if (!p || cta < -1) return fail(VT_ERR_INVALID_ARG, "bad vt_token_test_barrier arguments");
+    if (!p->tok_ok) return fail(VT_ERR_STATE, "the partition has no fused decode-token kernel: %s", p->tok_why.c_str());
+    if (cta >= p->tok_plan.grid) return fail(VT_ERR_INVALID_ARG, "cta %d is outside the grid of %d", cta, p->tok_plan.grid);
+    // two consecutive words of the sync area: the skipping CTA + 1, then the poll limit
+    const uint32_t words[2] = {(uint32_t)(cta + 1), spin_polls};
+    static_assert(kTokSyncTestSpin == kTokSyncTestSkip + 1, "test words are adjacent");
+    VT_CUDA(cudaMemcpyAsync(p->tok_base.sync + kTokSyncTestSkip, words, sizeof(words), cudaMemcpyHostToDevice,
+                            (cudaStream_t)stream));
+    VT_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+    return ok();
+}
+
 extern "C" vt_status vt_decode_token(const vt_partition* p, vt_kv* kv, const void* x_in, void* x_out,
                                      vt_stream stream) {
     VT_TRY(check_token_args(p, kv, x_in, x_out));

@@ -309,6 +309,8 @@ constexpr int kTokMaxGrid = 1024;
 // words of TokArgs::sync (zero at creation; zeroed again by a status clear)
 constexpr int kTokSyncEpoch = 0;                            // barriers completed by earlier launches
 constexpr int kTokSyncAbort = 2;                            // nonzero: the token gave up on a wait
+constexpr int kTokSyncTestSkip = 4;  // test hook: c + 1 makes CTA c skip its arrival at the launch's first grid barrier
+constexpr int kTokSyncTestSpin = 5;  // test hook: nonzero replaces the polls after which a grid-barrier wait gives up
 constexpr int kTokSyncFlags = 64;                           // [grid] epoch of each CTA's last arrival
 constexpr int kTokSyncWords = kTokSyncFlags + kTokMaxGrid;
 

@@ -245,7 +245,11 @@ __device__ __forceinline__ void ring_release(Ring& r, int lane) {
 // the weight stream for its L2 round trip (one copy of the barrier instead of four measured 7%
 // of the token time).
 
-__device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epoch) {
+// spin: polls before the wait gives up; skip_epoch: the barrier (epoch) at which this CTA does
+// not publish its arrival (0: none) -- both from the test words of the sync area, which a status
+// clear zeroes, so outside a test every CTA arrives and waits up to kTokSpin polls.
+__device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live, uint32_t epoch, uint32_t spin,
+                                       uint32_t skip_epoch) {
     consumer_bar(1, kTokConsumers);
     const int lane = threadIdx.x & 31;
     if (threadIdx.x < 32) {
@@ -254,7 +258,7 @@ __device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live,
         if (ok) {
             // the CTA's writes precede this store through the CTA barrier above, and a release
             // store makes them visible to every thread that acquires the flag
-            if (lane == 0) st_release(flags + blockIdx.x, epoch);
+            if (lane == 0 && epoch != skip_epoch) st_release(flags + blockIdx.x, epoch);
             // each poll is one round of independent loads; the abort word is read only every 64
             // polls, so a poll costs one L2 round trip
             for (uint32_t i = 1;; ++i) {
@@ -265,7 +269,7 @@ __device__ __noinline__ bool grid_sync(const TokArgs& a, int* s_flag, bool live,
                     int stop = 0;
                     if (lane == 0) {
                         if (ld_volatile(a.sync + kTokSyncAbort)) stop = 1;
-                        else if (i > kTokSpin) {
+                        else if (i > spin) {
                             stop = 1;
                             abort_token(a);
                         }
@@ -748,7 +752,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
     uint64_t* full = reinterpret_cast<uint64_t*>(p);
     uint64_t* empty = full + S;
     __shared__ int s_flag;
-    __shared__ uint32_t s_epoch;
+    __shared__ uint32_t s_epoch, s_test_skip, s_test_spin;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int c = blockIdx.x, NC = gridDim.x;
@@ -759,6 +763,8 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
         }
         fence_mbar_init();
         s_epoch = a.sync[kTokSyncEpoch];
+        s_test_skip = a.sync[kTokSyncTestSkip];
+        s_test_spin = a.sync[kTokSyncTestSpin];
     }
     for (int l = tid; l < a.n_layers; l += blockDim.x) lens[l] = a.len[l];
     __syncthreads();
@@ -851,6 +857,8 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kTokConsumerRegs));
     bool live = ld_volatile(a.sync + kTokSyncAbort) == 0;
     uint32_t epoch = s_epoch;
+    const uint32_t spin = s_test_spin ? s_test_spin : kTokSpin;
+    const uint32_t skip_epoch = s_test_skip == (uint32_t)c + 1u ? s_epoch + 1u : 0u;
     const uint32_t ring_s = smem_u32(ring_base);
     uint32_t bh[STEPS][2], bl[STEPS][2];  // hi / lo fp16 B fragments of the normalised input
     uint32_t gf[STEPS][2];                // RMSNorm gains at the B positions, loaded before the barrier that precedes the norm
@@ -950,7 +958,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
             });
             if (!ok && c == 0 && tid == 0) set_status(a.status, VT_DEV_KV_OVERFLOW);
         }
-        live = grid_sync(a, &s_flag, live, ++epoch);
+        live = grid_sync(a, &s_flag, live, ++epoch, spin, skip_epoch);
 
         // ------------------------------------------------------------ attention slices
         if (c == 0 && live)  // nobody reads the previous layer's FFN partials any more
@@ -977,7 +985,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
             }
             mtab[idx] = base;
         }
-        live = grid_sync(a, &s_flag, live, ++epoch);
+        live = grid_sync(a, &s_flag, live, ++epoch, spin, skip_epoch);
 
         // ------------------------------------------------------------ O rows
         {
@@ -1044,7 +1052,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
             });
         }
         prefetch_bgain<STEPS>(a.layer[l].ffn_norm, mld, gd.L, gf);
-        live = grid_sync(a, &s_flag, live, ++epoch);
+        live = grid_sync(a, &s_flag, live, ++epoch, spin, skip_epoch);
 
         // ------------------------------------------------------------ FFN columns
         // h = x + sum of the ATTN partials (shards in order), rounded to fp16
@@ -1111,7 +1119,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
             }
         });
         if (l + 1 < a.n_layers) prefetch_bgain<STEPS>(a.layer[l + 1].attn_norm, mld, gd.L, gf);
-        live = grid_sync(a, &s_flag, live, ++epoch);
+        live = grid_sync(a, &s_flag, live, ++epoch, spin, skip_epoch);
     }
 
     // ---------------------------------------------------------------- output and KV lengths

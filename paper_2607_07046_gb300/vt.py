@@ -38,6 +38,7 @@ VT_PARTITION_PRUNE = 1
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
+_U32 = ctypes.c_uint32
 
 
 class VtError(RuntimeError):
@@ -152,6 +153,7 @@ def lib() -> ctypes.CDLL:
             "vt_combine_q": (S, [ctypes.POINTER(_P), ctypes.POINTER(_P), _I32, ctypes.c_int64, _I32, _P, _P, _P]),
             "vt_partition_set_comm_bits": (S, [_P, _I32, _I32]),
             "vt_token_partials_read": (S, [_P, _I32, _P]),
+            "vt_token_test_barrier": (S, [_P, _I32, _U32, _P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -582,6 +584,12 @@ def vt_token_partials_read(part: int, block: int, n_devices: int, d_model: int) 
     out = np.empty((n_devices, d_model), np.float32)
     _check(lib().vt_token_partials_read(part, int(block), out.ctypes.data))
     return out
+
+
+def vt_token_test_barrier(part: int, cta: int, spin_polls: int, stream=None) -> None:
+    """Test hook: CTA `cta` of the next fused tokens skips its first grid-barrier arrival and
+    grid-barrier waits give up after `spin_polls` polls, until a status clear."""
+    _check(lib().vt_token_test_barrier(part, int(cta), int(spin_polls), _stream(stream)))
 
 
 def vt_prefill_tokens(part: int, kv: int, x_in, n: int, x_out, stream=None) -> None:

@@ -243,3 +243,60 @@ def test_capture_leaves_the_host_length_mirror(vtlib):
         assert vt.vt_kv_length(st.kv, 0) == L0 + 1
         assert vt.vt_kv_status(st.kv) == 0
         del g
+
+
+# ------------------------------------------------------------------ bounded waits
+
+@pytest.mark.parametrize("cta", [0, -2])
+def test_grid_barrier_wait_gives_up_and_the_next_token_runs_clean(vtlib, cta):
+    """The fused kernel's grid-barrier waits are bounded.  One CTA (the first, or the last of the
+    grid) is made to skip its arrival at the token's first barrier and the poll limit is cut to a
+    few thousand: every CTA gives up, the kernel returns (no hang), and the KV status word reports
+    VT_DEV_WAIT_TIMEOUT to the host.  After the status is cleared (which also removes the test
+    settings) the same token, from the same KV length, runs clean and equals the first clean run."""
+    vt = vtlib
+    kw, layers, L0, steps = SHAPES["mha-dh128-3way"]
+    wl = synthetic.small("timeout", kv_len=L0, decode_steps=1, prompt_len=0, **kw)
+    cap = L0 + 4
+    with build(vt, wl, layer_ids=layers, capacity=cap) as st:
+        for i, layer in enumerate(layers):
+            kc, vc = wl.kv_fill(layer, L0, cap)
+            write_cache(vt, st, i, wl, kc, vc, L0, wl.head_ranges)
+        fused, why = vt.vt_decode_token_fused_available(st.part)
+        assert fused, why
+        xin = dev(wl.hidden(1, stream=160).reshape(-1))
+        xout = torch.empty_like(xin)
+
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        vt.vt_decode_token(st.part, st.kv, xin, xout)
+        clean = host(xout).copy()
+        assert vt.vt_kv_status(st.kv) == 0
+
+        # the grid size is the partition's; -2 picks the last CTA through the hook's range check
+        target = cta
+        if cta < 0:
+            target = 0
+            while True:
+                try:
+                    vt.vt_token_test_barrier(st.part, target + 1, 4096)
+                    target += 1
+                except vt.VtError:
+                    break
+        vt.vt_token_test_barrier(st.part, target, 4096)
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        xout.fill_(0)
+        vt.vt_decode_token(st.part, st.kv, xin, xout)
+        torch.cuda.synchronize()
+        flags = vt.vt_kv_status(st.kv, clear=True)
+        assert flags & vt.VT_DEV_WAIT_TIMEOUT, f"status {flags:#x}"
+        assert vt.vt_kv_status(st.kv) == 0
+
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        vt.vt_decode_token(st.part, st.kv, xin, xout)
+        again = host(xout)
+        assert vt.vt_kv_status(st.kv) == 0
+        assert vt.vt_kv_length(st.kv, 0) == L0 + 1
+        d = np.abs(again.astype(np.float64) - clean.astype(np.float64))
+        assert d.max() <= 2e-3, f"clean run after the timeout differs by {d.max():.3e}"
+        with pytest.raises(vt.VtError):
+            vt.vt_token_test_barrier(st.part, -2, 0)
