@@ -46,9 +46,20 @@ WORKLOAD = ("llama2-7b-shaped batch-1 decode: 32 layers, D 4096, 32 heads x 128 
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM bytes (read + write) of one launch of the decode-token kernel, from one ncu capture of
-# that kernel as it is built now (mean of the 12 launches of the 7B launch list); None until
-# captured, and again once the kernel changes.
-K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_504_012_800
+# that kernel (mean of 12 launches of the 7B decode; profiles/k_decode_token_7b.md), and a
+# digest of the sources the captured kernel was built from.  The line reports the bytes only
+# while the sources still hash to that digest: a changed kernel reports null until recaptured.
+K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_504_014_827
+K_TOKEN_SOURCES = ("token_kernel.cuh", "token.cu", "token_v1.cu", "token_v2.cu", "internal.h", "device.cuh")
+K_TOKEN_SOURCES_SHA256 = "998cd22556cd4766"
+
+
+def token_traffic_if_current():
+    import hashlib
+    h = hashlib.sha256()
+    for f in K_TOKEN_SOURCES:
+        h.update((ROOT / "paper_2607_07046_gb300" / "csrc" / f).read_bytes())
+    return K_TOKEN_DRAM_BYTES_PER_LAUNCH if h.hexdigest()[:16] == K_TOKEN_SOURCES_SHA256 else None
 
 
 def measured_peaks():
@@ -500,7 +511,7 @@ def run_decode(args, rank, world):
             "peak_kind": f"{peak_kind} copy bandwidth",
             "bytes_per_launch": int(step_bytes) if fused else None,
             "launch_ms": round(ms_per_step, 5),
-            "traffic": K_TOKEN_DRAM_BYTES_PER_LAUNCH if fused and not args.layers else None,
+            "traffic": token_traffic_if_current() if fused and not args.layers else None,
         },
         "e2e": {"value": round(world / e2e_s, 3), "unit": "tok/s", "h2d_bytes_per_step": 4,
                 "d2h_bytes_per_step": 2 * D, "finite": e2e_finite},
