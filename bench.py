@@ -62,6 +62,22 @@ def token_traffic_if_current():
     return K_TOKEN_DRAM_BYTES_PER_LAUNCH if h.hexdigest()[:16] == K_TOKEN_SOURCES_SHA256 else None
 
 
+def all_ranks_max(torch, x: float, device: str) -> float:
+    """The maximum of x over the ranks of the process group (x itself on one process): the
+    timed region's repeat count and its step time are taken as the slowest rank's."""
+    if not (torch.distributed.is_available() and torch.distributed.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replicas_tok_s(world: int, ms_per_step: float) -> float:
+    """Whole-job decode rate: every rank decodes its own token stream (a replica), so the job
+    makes `world` tokens per step of the slowest rank."""
+    return world * 1000.0 / ms_per_step
+
+
 def measured_peaks():
     p = ROOT / "MEASURED_PEAKS.json"
     if p.exists():
@@ -402,9 +418,7 @@ def run_decode(args, rank, world):
         est_ms = w0.elapsed_time(w1) / max(args.warmup, 1)
         repeats = int(min(64, max(1, np.ceil(args.min_timed_s * 1e3 / max(est_ms * args.steps, 1e-3)))))
         if world > 1:
-            t = torch.tensor([repeats], device="cuda")
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            repeats = int(t.item())
+            repeats = int(all_ranks_max(torch, repeats, "cuda"))
         sch.reset()
         rep_ms = []
         with ClockSampler(torch.cuda.current_device()) as clk:
@@ -423,9 +437,7 @@ def run_decode(args, rank, world):
                 rep_ms.append(e0.elapsed_time(e1))
         ms = float(np.median(rep_ms))
         if world > 1:
-            t = torch.tensor([ms], device="cuda")
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            ms = float(t.item())
+            ms = all_ranks_max(torch, ms, "cuda")
         ms_per_step = ms / args.steps
         kv_status = vt.vt_kv_status(st.kv, clear=True)
         part_status = vt.vt_partition_status(st.part, clear=True)
@@ -454,6 +466,8 @@ def run_decode(args, rank, world):
             for i in range(e2e_steps):
                 e2e_step(i)
         e2e_s = (time.perf_counter() - t0) / e2e_steps
+        if world > 1:
+            e2e_s = all_ranks_max(torch, e2e_s, "cuda")
         e2e_finite = bool(np.isfinite(out_host.numpy().astype(np.float32)).all())
 
         # -------------------------------------------------------------- per-shard kernels, for context
@@ -471,7 +485,7 @@ def run_decode(args, rank, world):
     hbm, _, _, peak_kind = measured_peaks()
     kv_mean = wl.kv_len + (min(args.steps, sched) - 1) / 2.0
     step_bytes = decode_bytes_per_token(wl, kv_mean)
-    value = world * 1000.0 / ms_per_step
+    value = replicas_tok_s(world, ms_per_step)
     achieved = step_bytes / (ms_per_step * 1e-3) / 1e9
     launches_per_token = 1 if fused else kernels_per_token(wl)
     line = {
