@@ -71,6 +71,7 @@ typedef int32_t vt_status;
 #define VT_ERR_ALLOC 9            /* the allocator returned NULL */
 #define VT_ERR_STATE 10           /* object not ready (e.g. a layer's weights never loaded) */
 #define VT_ERR_PLAN_MEMORY 11     /* the devices' memory budgets cannot hold the block */
+#define VT_ERR_PLAN_QOS 12        /* no precision configuration meets the time budget */
 
 #define VT_MAX_DEVICES 16
 
@@ -204,6 +205,33 @@ VT_API vt_status vt_plan_layers(const vt_shapes* shapes, int32_t n_devices, cons
                                 const double* flop_rate, const double* mem_bytes, double link_bytes_per_s,
                                 double link_latency_s, int32_t tokens, int32_t kv_len, vt_block_plan* plans,
                                 double* total_s);
+
+/* vt_plan_precision (host only): importance-aware mixed precision (Voltron Section 4.2.2).  Given
+ * the blocks' plan (plans[2 n_layers], e.g. from vt_plan_layers: each device's heads or columns
+ * of every block, and the block's transfer time comm_s) and an importance score per block
+ * (importance[2 n_layers], ATTN of layer l at 2 l, FFN at 2 l + 1; higher = more important; the
+ * scores are the caller's, the paper's come from offline perplexity profiling), blocks are lowered
+ * one precision step at a time in ascending order of importance (ties: lower block index).
+ * Configuration k (0 <= k <= 4 n_layers) has the min(k, 2 n_layers) least important blocks at
+ * INT8 at least and the first k - 2 n_layers of them at INT4; every block of a configuration is
+ * at one precision on all its devices.  A device's memory (its shards' weights at their
+ * precision: fp16, or codes plus one fp16 scale per 32 weights along the contraction axis, as
+ * vt_partition_set_precision stores them, plus the fp16 K / V cache of its KV heads at max_seq)
+ * and the stack's time (per block the slowest device's streamed bytes / rate[d]: its weights and,
+ * for ATTN, the K / V rows of kv_len + 1 positions; plus the block's comm_s) do not grow with k,
+ * so the smallest k that fits every mem_bytes[d] (nullable: no limit) and qos_s (<= 0 or
+ * infinite: no limit) is found by binary search over k.
+ * bits[2 n_layers] receives 16, 8 or 4 per block; steps (nullable) the chosen k; total_s
+ * (nullable) that configuration's time.  The plan's parallelism is kept: re-planning with the new
+ * precisions is the caller's choice.
+ * Errors: VT_ERR_INVALID_ARG (null pointers, non-finite importance or comm_s, kv_len outside
+ * [0, max_seq), bad rates or budgets), VT_ERR_PARTITION_RANGE / VT_ERR_PARTITION_GQA for a plan
+ * range outside the block or not in whole KV groups; VT_ERR_PLAN_MEMORY or VT_ERR_PLAN_QOS when
+ * even configuration 4 n_layers (every block INT4) misses a budget, with bits, steps and total_s
+ * describing that configuration. */
+VT_API vt_status vt_plan_precision(const vt_shapes* shapes, int32_t n_devices, const vt_block_plan* plans,
+                                   const double* importance, const double* rate, const double* mem_bytes,
+                                   double qos_s, int32_t kv_len, int32_t* bits, int32_t* steps, double* total_s);
 
 /* vt_quantize_rows (host only): block quantization of fp16 weight rows for mixed-precision shards
  * (Voltron Section 3.2.2 and Section 4.2.2, precision heterogeneity; Section 5.1 names k-quant

@@ -508,6 +508,129 @@ extern "C" vt_status vt_plan_layers(const vt_shapes* s, int32_t n, const double*
     return ok();
 }
 
+// Importance-aware mixed precision (Voltron Section 4.2.2): blocks lowered one precision step at a
+// time in ascending order of importance, the number of steps found by binary search.
+namespace {
+// bytes of a rows x k weight matrix at `bits` (16: fp16; 8 / 4: codes + one fp16 scale per block of 32)
+double matrix_bytes(double rows, double k, int bits) {
+    if (bits == 16) return rows * k * 2.0;
+    return rows * std::ceil(k / 32.0) * (32.0 * bits / 8.0 + 2.0);
+}
+struct PrecisionModel {
+    const vt_shapes* s;
+    int n, nb;
+    const vt_block_plan* plans;
+    const double *rate, *mem;
+    double kv_len;
+    std::vector<int> order;  // blocks by ascending importance (ties: lower index)
+    // per device: memory and streamed bytes of block b at `bits`
+    void block_cost(int b, int d, int bits, double* mem_b, double* stream_b) const {
+        const vt_range r = plans[b].ranges[d];
+        const double cnt = r.end - r.begin, D = s->d_model, dh = s->d_head;
+        if (cnt <= 0) {
+            *mem_b = *stream_b = 0.0;
+            return;
+        }
+        if ((b & 1) == 0) {  // ATTN: cnt query heads, cnt / g KV heads
+            const double hk = cnt / (s->n_heads / s->n_kv_heads);
+            const double w = matrix_bytes((cnt + 2.0 * hk) * dh, D, bits) + matrix_bytes(D, cnt * dh, bits);
+            *mem_b = w + 2.0 * 2.0 * hk * s->max_seq * dh;
+            *stream_b = w + 2.0 * 2.0 * hk * dh * (kv_len + 1.0);
+        } else {  // FFN: cnt columns
+            const double w = matrix_bytes(2.0 * cnt, D, bits) + matrix_bytes(D, cnt, bits);
+            *mem_b = *stream_b = w;
+        }
+    }
+    // bits of every block after k steps
+    void bits_at(int k, int32_t* bits) const {
+        for (int b = 0; b < nb; ++b) bits[b] = 16;
+        for (int i = 0; i < nb; ++i) {
+            if (i < k) bits[order[i]] = 8;
+            if (i < k - nb) bits[order[i]] = 4;
+        }
+    }
+    // memory fits every device; total time
+    void eval(const int32_t* bits, bool* mem_ok, double* time_s) const {
+        std::vector<double> used(n, 0.0);
+        double t = 0.0;
+        for (int b = 0; b < nb; ++b) {
+            double slow = 0.0;
+            for (int d = 0; d < n; ++d) {
+                double mb, sb;
+                block_cost(b, d, bits[b], &mb, &sb);
+                used[d] += mb;
+                if (sb > 0.0) slow = std::max(slow, sb / rate[d]);
+            }
+            t += slow + plans[b].comm_s;
+        }
+        *mem_ok = true;
+        if (mem)
+            for (int d = 0; d < n; ++d) *mem_ok = *mem_ok && used[d] <= mem[d];
+        *time_s = t;
+    }
+};
+}  // namespace
+
+extern "C" vt_status vt_plan_precision(const vt_shapes* s, int32_t n, const vt_block_plan* plans,
+                                       const double* importance, const double* rate, const double* mem, double qos_s,
+                                       int32_t kv_len, int32_t* bits, int32_t* steps, double* total_s) {
+    if (!s || !plans || !importance || !rate || !bits)
+        return fail(VT_ERR_INVALID_ARG, "shapes, plans, importance, rate and bits must not be NULL");
+    VT_TRY(vt_shapes_validate(s));
+    if (n < 1 || n > VT_MAX_DEVICES) return fail(VT_ERR_INVALID_ARG, "n_devices must be in [1, %d]", VT_MAX_DEVICES);
+    VT_TRY(check_rates(n, rate, mem));
+    if (std::isnan(qos_s)) return fail(VT_ERR_INVALID_ARG, "qos_s is NaN");
+    if (kv_len < 0 || kv_len >= s->max_seq) return fail(VT_ERR_INVALID_ARG, "kv_len %d outside [0, max_seq)", kv_len);
+    const int nb = 2 * s->n_layers;
+    const int g = s->n_heads / s->n_kv_heads;
+    for (int b = 0; b < nb; ++b) {
+        if (!std::isfinite(importance[b])) return fail(VT_ERR_INVALID_ARG, "importance[%d] is not finite", b);
+        const int total = (b & 1) ? s->d_ffn : s->n_heads;
+        for (int d = 0; d < n; ++d) {
+            const vt_range r = plans[b].ranges[d];
+            if (r.begin < 0 || r.end < r.begin || r.end > total)
+                return fail(VT_ERR_PARTITION_RANGE, "block %d device %d: range [%d, %d)", b, d, r.begin, r.end);
+            if ((b & 1) == 0 && ((r.end - r.begin) % g) != 0)
+                return fail(VT_ERR_PARTITION_GQA, "block %d device %d: %d heads are not whole KV groups", b, d,
+                            r.end - r.begin);
+        }
+        if (!(plans[b].comm_s >= 0.0) || !std::isfinite(plans[b].comm_s))
+            return fail(VT_ERR_INVALID_ARG, "block %d: comm_s must be finite and >= 0", b);
+    }
+    PrecisionModel pm{s, n, nb, plans, rate, mem, (double)kv_len, {}};
+    pm.order.resize(nb);
+    for (int b = 0; b < nb; ++b) pm.order[b] = b;
+    std::stable_sort(pm.order.begin(), pm.order.end(), [&](int a, int b) { return importance[a] < importance[b]; });
+    const bool timed = qos_s > 0.0 && std::isfinite(qos_s);
+    std::vector<int32_t> cand(nb);
+    auto feasible = [&](int k, bool* mem_ok, double* t) {
+        pm.bits_at(k, cand.data());
+        pm.eval(cand.data(), mem_ok, t);
+        return *mem_ok && (!timed || *t <= qos_s);
+    };
+    // memory and time do not grow with k: the smallest feasible k by bisection over [0, 2 nb]
+    bool mem_ok;
+    double t;
+    int lo = 0, hi = 2 * nb;
+    if (!feasible(hi, &mem_ok, &t)) {
+        pm.bits_at(hi, bits);
+        if (steps) *steps = hi;
+        if (total_s) *total_s = t;
+        if (!mem_ok) return fail(VT_ERR_PLAN_MEMORY, "the memory budgets are missed even with every block at INT4");
+        return fail(VT_ERR_PLAN_QOS, "%.6g s with every block at INT4 misses qos_s %.6g s", t, qos_s);
+    }
+    while (lo < hi) {
+        const int mid = lo + (hi - lo) / 2;
+        if (feasible(mid, &mem_ok, &t)) hi = mid;
+        else lo = mid + 1;
+    }
+    feasible(lo, &mem_ok, &t);
+    pm.bits_at(lo, bits);
+    if (steps) *steps = lo;
+    if (total_s) *total_s = t;
+    return ok();
+}
+
 // ================================================================== quantization (host)
 
 // Block quantization of fp16 weight rows (Voltron Sections 3.2.2 / 4.2.2): fp16 scale per block,

@@ -28,6 +28,7 @@ VT_ERR_CUDA = 8
 VT_ERR_ALLOC = 9
 VT_ERR_STATE = 10
 VT_ERR_PLAN_MEMORY = 11
+VT_ERR_PLAN_QOS = 12
 VT_MAX_DEVICES = 16
 VT_DEV_KV_OVERFLOW = 1
 VT_DEV_WAIT_TIMEOUT = 2
@@ -101,6 +102,10 @@ def lib() -> ctypes.CDLL:
                                       ctypes.POINTER(ctypes.c_double), _I32, ctypes.POINTER(vt_range),
                                       ctypes.POINTER(ctypes.c_double)]),
             "vt_quantize_rows": (S, [_P, ctypes.c_int64, ctypes.c_int64, _I32, _I32, _P, _P]),
+            "vt_plan_precision": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(vt_block_plan),
+                                      ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                                      ctypes.POINTER(ctypes.c_double), ctypes.c_double, _I32,
+                                      ctypes.POINTER(_I32), ctypes.POINTER(_I32), ctypes.POINTER(ctypes.c_double)]),
             "vt_plan_layers": (S, [ctypes.POINTER(vt_shapes), _I32, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
                                    ctypes.c_double, ctypes.c_double, _I32, _I32,
@@ -295,6 +300,40 @@ def vt_plan_layers(shapes: vt_shapes, rate, flop_rate=None, mem_bytes=None, link
     plans = [dict(tp=bool(p.tp), device=p.device, ranges=[(p.ranges[d].begin, p.ranges[d].end) for d in range(n)],
                   compute_s=p.compute_s, comm_s=p.comm_s) for p in out]
     return plans, tot.value
+
+
+def vt_plan_precision(shapes: vt_shapes, plans, importance, rate, mem_bytes=None, qos_s: float = 0.0,
+                      kv_len: int = 0):
+    """Importance-aware precision of every block for a given plan (list of per-block dicts as
+    vt_plan_layers returns them): (bits per block, steps, total seconds).  Raises VtError on a
+    failed status (VT_ERR_PLAN_MEMORY / VT_ERR_PLAN_QOS when no configuration fits)."""
+    n = len(rate)
+    nb = 2 * shapes.n_layers
+    if len(plans) != nb or len(importance) != nb:
+        raise ValueError("one plan and one importance score per block")
+    cp = (vt_block_plan * nb)()
+    for i, p in enumerate(plans):
+        cp[i].tp = int(p.get("tp", 0))
+        cp[i].device = int(p.get("device", 0))
+        for d, (a, b) in enumerate(p["ranges"]):
+            cp[i].ranges[d].begin, cp[i].ranges[d].end = int(a), int(b)
+        cp[i].compute_s = float(p.get("compute_s", 0.0))
+        cp[i].comm_s = float(p.get("comm_s", 0.0))
+
+    def arr(v):
+        if v is None:
+            return None
+        if len(v) != n:
+            raise ValueError("one value per device")
+        return (ctypes.c_double * n)(*[float(x) for x in v])
+
+    imp = (ctypes.c_double * nb)(*[float(x) for x in importance])
+    bits = (_I32 * nb)()
+    steps = _I32(0)
+    tot = ctypes.c_double(0.0)
+    _check(lib().vt_plan_precision(ctypes.byref(shapes), n, cp, imp, arr(rate), arr(mem_bytes), float(qos_s),
+                                   int(kv_len), bits, ctypes.byref(steps), ctypes.byref(tot)))
+    return list(bits), steps.value, tot.value
 
 
 # ------------------------------------------------------------------ model

@@ -191,6 +191,57 @@ def test_whole_tokens_mixed_precision_per_layer(vtlib):
         assert vt.vt_kv_status(st.kv) == 0
 
 
+def test_planned_precisions_run_and_match_the_oracle(vtlib):
+    """The precision plan of Section 4.2.2 applied end to end: seeded importance scores per block
+    and a memory budget between the all-fp16 and all-INT4 footprints give vt_plan_precision's bits
+    per block; the stack built with them decodes two tokens that equal the oracle's layers at the
+    same precisions, and the blocks left at fp16 are the most important ones."""
+    vt = vtlib
+    wl = UNEVEN
+    L0, steps, cap = 40, 2, 48
+    sh = shapes_of(vt, wl, max_seq=max(wl.max_seq, cap))
+    plans = [dict(ranges=list(wl.head_ranges), comm_s=0.0) if b % 2 == 0 else dict(ranges=list(wl.ffn_ranges), comm_s=0.0)
+             for b in range(2 * wl.n_layers)]
+    importance = list(np.random.default_rng(5).normal(size=2 * wl.n_layers))
+    rate = [1e9] * len(wl.head_ranges)
+    full, _, _ = vt.vt_plan_precision(sh, plans, importance, rate)
+    assert full == [16] * 4
+    # device 1 holds the most: a budget of 60% of its fp16 footprint forces several steps
+    fp16_mem = []
+    for d in range(len(rate)):
+        h = wl.head_ranges[d][1] - wl.head_ranges[d][0]
+        c = wl.ffn_ranges[d][1] - wl.ffn_ranges[d][0]
+        hk = h // (wl.n_heads // wl.n_kv_heads)
+        attn = 2 * ((h + 2 * hk) * wl.d_head * wl.d_model + wl.d_model * h * wl.d_head) + 4 * hk * sh.max_seq * wl.d_head
+        fp16_mem.append(wl.n_layers * (attn + 2 * 3 * wl.d_model * c))
+    budget = [m * 0.6 for m in fp16_mem]
+    bits, k, _ = vt.vt_plan_precision(sh, plans, importance, rate, mem_bytes=budget)
+    assert 0 < k < 4 * wl.n_layers and any(b != 16 for b in bits)
+    kept = [b for b in range(4) if bits[b] == 16]
+    lowered = [b for b in range(4) if bits[b] != 16]
+    if kept:
+        assert min(importance[b] for b in kept) >= max(importance[b] for b in lowered)
+    ws = [wl.layer_weights(l) for l in range(2)]
+    caches = [wl.kv_fill(l, L0, cap) for l in range(2)]
+    n = len(rate)
+    with stack(vt, wl, cap, precision=lambda l, d, b: bits[2 * l + b]) as st:
+        for l in range(2):
+            for d, hr in enumerate(wl.head_ranges):
+                k0, k1 = kv_range(wl, hr)
+                vt.vt_kv_write_raw(st.kv, l, d, caches[l][0][k0:k1, :L0], caches[l][1][k0:k1, :L0])
+        vt.vt_kv_set_length(st.kv, -1, L0)
+        y = torch.empty(wl.d_model, dtype=torch.float16, device="cuda")
+        for t in range(steps):
+            x = wl.hidden(1, stream=330 + t)
+            vt.vt_decode_token(st.part, st.kv, dev(x.reshape(-1)), y)
+            r = x.reshape(1, -1)
+            for l in range(2):
+                _, r, _, _ = oracle.tp_layer_mixed(wl, ws[l], r, L0 + t, *caches[l], [bits[2 * l]] * n,
+                                                   [bits[2 * l + 1]] * n)
+            assert_close(host(y), r.reshape(-1), f"planned-precision token {t}")
+        assert vt.vt_kv_status(st.kv) == 0
+
+
 def test_precision_api_rules(vtlib):
     vt = vtlib
     wl = dataclasses.replace(UNEVEN, n_layers=1)

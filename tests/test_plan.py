@@ -313,3 +313,146 @@ def test_plans_are_always_valid_partitions(vtlib, seed):
             if not p["tp"]:
                 sizes_ = [b - a for a, b in p["ranges"]]
                 assert sum(1 for x in sizes_ if x) == 1 and sizes_[p["device"]] > 0
+
+
+# ------------------------------------------------------------------ importance-aware precision
+# Voltron Section 4.2.2: blocks are lowered one precision step at a time (fp16 -> INT8 -> INT4) in
+# ascending order of importance, and the number of steps is the smallest that meets the memory
+# budgets and the time budget, found by binary search (memory and time do not grow with steps).
+# Pins: the byte counts restated here from the layer definition and the block format (codes plus
+# one fp16 scale per 32 weights along the contraction axis); the result equals a linear scan over
+# every configuration; the lowered blocks are the least important ones; no budget lowers nothing.
+
+def _q_bytes(rows, k, bits):
+    if bits == 16:
+        return rows * k * 2
+    return rows * math.ceil(k / 32) * (32 * bits // 8 + 2)
+
+
+def _config(nb, order, k):
+    bits = [16] * nb
+    for i, b in enumerate(order):
+        if i < k:
+            bits[b] = 8
+        if i < k - nb:
+            bits[b] = 4
+    return bits
+
+
+def _cost(wl, plans, bits, rate, kv_len, max_seq):
+    """Each device's memory and the stack's time for one configuration, from the definitions."""
+    D, dh, g = wl.d_model, wl.d_head, wl.n_heads // wl.n_kv_heads
+    n = len(rate)
+    used = [0.0] * n
+    t = 0.0
+    for b, p in enumerate(plans):
+        slow = 0.0
+        for d, (lo, hi) in enumerate(p["ranges"]):
+            c = hi - lo
+            if c == 0:
+                continue
+            if b % 2 == 0:
+                hk = c // g
+                w = _q_bytes((c + 2 * hk) * dh, D, bits[b]) + _q_bytes(D, c * dh, bits[b])
+                mem = w + 2 * 2 * hk * max_seq * dh
+                stream = w + 2 * 2 * hk * dh * (kv_len + 1)
+            else:
+                w = _q_bytes(2 * c, D, bits[b]) + _q_bytes(D, c, bits[b])
+                mem = stream = w
+            used[d] += mem
+            slow = max(slow, stream / rate[d])
+        t += slow + p["comm_s"]
+    return used, t
+
+
+def _even_plans(wl, n):
+    """Every block split evenly (whole KV groups for ATTN) over n devices."""
+    g = wl.n_heads // wl.n_kv_heads
+
+    def split(total, unit):
+        units = total // unit
+        cuts = [unit * (units * d // n) for d in range(n + 1)]
+        cuts[-1] = total
+        return [(cuts[d], cuts[d + 1]) for d in range(n)]
+
+    plans = []
+    for _ in range(wl.n_layers):
+        plans.append(dict(tp=1, device=0, ranges=split(wl.n_heads, g), comm_s=1e-5))
+        plans.append(dict(tp=1, device=0, ranges=split(wl.d_ffn, 1), comm_s=1e-5))
+    return plans
+
+
+def _precision_wl():
+    return synthetic.small("prec", n_layers=4, d_model=512, n_heads=8, n_kv_heads=4, d_head=64, d_ffn=1000,
+                           head_ranges=((0, 4), (4, 8)), ffn_ranges=((0, 500), (500, 1000)), kv_len=64)
+
+
+def test_precision_without_budgets_stays_fp16(vtlib):
+    wl = _precision_wl()
+    sh = shapes(vtlib, wl, max_seq=128)
+    plans = _even_plans(wl, 2)
+    bits, steps, t = vtlib.vt_plan_precision(sh, plans, list(range(8)), [1e9, 1e9], kv_len=64)
+    assert bits == [16] * 8 and steps == 0
+    assert t == pytest.approx(_cost(wl, plans, bits, [1e9, 1e9], 64, 128)[1], rel=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_precision_binary_search_equals_a_linear_scan(vtlib, seed):
+    rng = np.random.default_rng(seed)
+    wl = _precision_wl()
+    max_seq, kv_len = 128, int(rng.integers(0, 127))
+    sh = shapes(vtlib, wl, max_seq=max_seq)
+    n = int(rng.integers(1, 4))
+    plans = _even_plans(wl, n)
+    nb = 2 * wl.n_layers
+    importance = list(rng.normal(size=nb))
+    rate = list(rng.uniform(1e9, 4e9, size=n))
+    order = sorted(range(nb), key=lambda b: (importance[b], b))
+    costs = [_cost(wl, plans, _config(nb, order, k), rate, kv_len, max_seq) for k in range(2 * nb + 1)]
+    # memory and time do not grow with k
+    for (m0, t0), (m1, t1) in zip(costs, costs[1:]):
+        assert all(b <= a + 1e-9 for a, b in zip(m0, m1)) and t1 <= t0 + 1e-15
+    # budgets between the fp16 and all-INT4 costs
+    k_mem, k_t = rng.integers(0, 2 * nb + 1, size=2)
+    mem = [costs[k_mem][0][d] for d in range(n)]
+    qos = costs[k_t][1] * (1 + 1e-12)
+    want = next(k for k in range(2 * nb + 1)
+                if all(costs[k][0][d] <= mem[d] for d in range(n)) and costs[k][1] <= qos)
+    bits, steps, t = vtlib.vt_plan_precision(sh, plans, importance, rate, mem_bytes=mem, qos_s=qos, kv_len=kv_len)
+    assert steps == want
+    assert bits == _config(nb, order, want)
+    assert t == pytest.approx(costs[want][1], rel=1e-12)
+    # the lowered blocks are the least important ones
+    lowered = [b for b in range(nb) if bits[b] < 16]
+    kept = [b for b in range(nb) if bits[b] == 16]
+    if lowered and kept:
+        assert max(importance[b] for b in lowered) <= min(importance[b] for b in kept)
+
+
+def test_precision_budgets_that_no_configuration_meets(vtlib):
+    wl = _precision_wl()
+    sh = shapes(vtlib, wl, max_seq=128)
+    plans = _even_plans(wl, 2)
+    imp = [0.0] * 8
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_precision(sh, plans, imp, [1e9, 1e9], mem_bytes=[1.0, 1.0])
+    assert e.value.status == vtlib.VT_ERR_PLAN_MEMORY
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_precision(sh, plans, imp, [1e9, 1e9], qos_s=1e-9)
+    assert e.value.status == vtlib.VT_ERR_PLAN_QOS
+    bad = [dict(p) for p in plans]
+    bad[0] = dict(bad[0], ranges=[(0, 3), (3, 8)])  # 3 heads are not whole KV groups of 2
+    with pytest.raises(vtlib.VtError) as e:
+        vtlib.vt_plan_precision(sh, bad, imp, [1e9, 1e9])
+    assert e.value.status == vtlib.VT_ERR_PARTITION_GQA
+
+
+def test_precision_int8_shard_bytes_match_the_library_format(vtlib):
+    """The planner's INT8 / INT4 bytes are the block format vt_quantize_rows writes: one code per
+    weight (a nibble at INT4) and one fp16 scale per 32 weights of a row."""
+    rows, k = 6, 70
+    w = np.random.default_rng(1).normal(0, 0.02, size=(rows, k)).astype(np.float16)
+    for bits in (8, 4):
+        q, sc = vtlib.vt_quantize_rows(w, bits)
+        assert sc.shape == (rows, math.ceil(k / 32))
+        assert _q_bytes(rows, k, bits) == rows * math.ceil(k / 32) * 32 * bits // 8 + sc.nbytes
