@@ -149,6 +149,17 @@ __device__ __forceinline__ void bulk_reduce_add_f32(float* gdst, const float* ss
         "r"(smem_u32(ssrc)), "r"(bytes)
         : "memory");
 }
+// The same addition, waiting only until the source has been read (the shared memory may then be
+// reused); bulk_wait_all() later waits until every such addition of the thread has completed.
+__device__ __forceinline__ void bulk_reduce_add_f32_issue(float* gdst, const float* ssrc, uint32_t bytes) {
+    asm volatile(
+        "cp.reduce.async.bulk.global.shared::cta.bulk_group.add.f32 [%0], [%1], %2;\n\t"
+        "cp.async.bulk.commit_group;\n\t"
+        "cp.async.bulk.wait_group.read 0;" ::"l"(gdst),
+        "r"(smem_u32(ssrc)), "r"(bytes)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }

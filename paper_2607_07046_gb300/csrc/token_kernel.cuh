@@ -1110,15 +1110,18 @@ __global__ void __launch_bounds__(kTokThreads, 1) k_decode_token(const __grid_co
                 }
                 fence_proxy_async_smem();
                 consumer_bar(1, kTokConsumers);
-                if (tid == 0 && live) {
-                    bulk_reduce_add_f32(a.ffn_part + (size_t)s * D, slots, (uint32_t)D * 4u);
-                    // the reduction's writes (async proxy) before the barrier's release store
-                    asm volatile("fence.proxy.async;" ::: "memory");
-                }
+                // (the additions complete before the phase's grid barrier, below)
+                if (tid == 0 && live) bulk_reduce_add_f32_issue(a.ffn_part + (size_t)s * D, slots, (uint32_t)D * 4u);
                 consumer_bar(1, kTokConsumers);  // the reduction has read the slots
             }
         });
         if (l + 1 < a.n_layers) prefetch_bgain<STEPS>(a.layer[l + 1].attn_norm, mld, gd.L, gf);
+        if (tid == 0) {
+            // this CTA's FFN partial additions (async proxy) complete before the barrier's release
+            // store, which thread 0 makes
+            bulk_wait_all();
+            asm volatile("fence.proxy.async;" ::: "memory");
+        }
         live = grid_sync(a, &s_flag, live, ++epoch, spin, skip_epoch);
     }
 
