@@ -165,6 +165,17 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 }
 
 // ------------------------------------------------------------------ loads
+// 8- and 4-byte loads of read-only data streamed once (weights), no L1 allocation.
+__device__ __forceinline__ uint2 ldg_stream_u2(const void* p) {
+    uint2 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+    return v;
+}
+__device__ __forceinline__ uint32_t ldg_stream_u1(const void* p) {
+    uint32_t v;
+    asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
+    return v;
+}
 // 16-byte load of read-only data that is streamed once (weights): no L1 allocation.
 __device__ __forceinline__ uint4 ldg_stream(const void* p) {
     uint4 v;

@@ -8,13 +8,9 @@
 // 8 bits, 7 for 4 bits) and every weight the code q = round-half-even(w / d) clamped to
 // [-qmax, qmax] (0 when d = 0), both divisions in fp32.  A projection is y = sum_e (q_e d) x_e.
 //
-// The kernel streams the codes with 16-byte loads and rebuilds each code as an fp32 integer with
-// one byte permute (0x4B000000 | u is the float 2^23 + u, u the biased code) and one subtraction,
-// then multiplies with the input in fp32 pairs (packed f32x2 arithmetic, two lanes of the FMA
-// pipe per instruction).  The bias is removed once per chunk: sum_e u_e x_e - bias * sum_e x_e,
-// with the input's chunk sums computed once per CTA.  Decode at batch 1 is bound by HBM, and this
-// keeps the CUDA-core work per byte low enough for 8-bit codes (2 instructions per code) and close
-// enough for 4-bit codes.
+// The kernel keeps the codes as integers and multiplies them on the tensor cores (integer MMA
+// against an exact three-digit int8 split of the input), so the work per code is a small fraction
+// of an instruction and the GEMV streams at the memory rate (details at the kernel).
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -81,90 +77,106 @@ void unpack_qcodes(const uint8_t* codes, int64_t rows, int64_t k, int bits, int8
 
 // ================================================================== device: dequantizing GEMV
 //
-// Geometry.  A warp takes groups of kQRows consecutive rows; the 16-byte chunks of a row (16
-// codes at 8 bits, one block of 32 at 4 bits) are spread over the lanes (chunk 32 i + lane), so
-// every load instruction of the warp reads 512 contiguous bytes of one row, and the input values
-// of a chunk (from shared memory) serve all kQRows rows.  Row partials are reduced across the
-// warp with the multi-row butterfly; a CTA owns a contiguous range of row groups.  The next
-// step's codes and scales are loaded while the current step computes (two register buffers), and
-// the first two steps are issued before griddepcontrol.wait: the weights do not depend on the
-// preceding kernel.
+// Integer tensor-core GEMV.  Decode at batch 1 is bound by HBM only if the work per weight code
+// stays far below one instruction; rebuilding codes as floats costs more than that.  So the codes
+// stay integers and go to `mma.sync m16n8k32` (u8 codes x s8 input, s32 accumulate), one MMA per
+// block of 32 weights of 16 rows:
+//   - the input x^ (fp32) of block b is split into three int8 digits at scales s, s / 254 and
+//     s / 254^2 (s = max|x^| / 127 over the block), which reproduce it to 2^-24 of the block's
+//     largest value; the digits are the MMA's B columns 0, 1, 2, so one MMA gives all three
+//     integer dot products of each row with the block;
+//   - the code bias leaves in integers: sum (u - bias) q = D - bias * Q, Q = sum q over the block;
+//   - a row's block term is s * (D1 - bias Q1) + s / 254 * (D2 - ...) + ..., times the block's
+//     fp16 weight scale, accumulated in fp32.
+// Within a block the k order is permuted the same way for A and B: lane (g, t) of the MMA loads
+// the 8 codes of rows g and g + 8 at positions 8t .. 8t + 7 (one 8-byte load per row at 8 bits;
+// one 4-byte word at 4 bits, whose nibbles unpack to the same positions), which become its
+// fragment's k = 4t .. 4t + 3 and 16 + 4t .. 16 + 4t + 3; the B fragment of lane (n, t) is loaded
+// from the same positions of digit n, stored in the block's natural order.
+// Work split: a CTA takes 64 rows (four MMA row tiles) and one part of the blocks, and computes the
+// input digits of its part only; warp w takes row tile w % 4 and half w / 4 of the part.  The
+// parts of a row tile form a thread-block cluster: after a cluster barrier rank 0 adds the
+// parts' row sums in rank order (distributed shared memory) and runs the epilogue, and a second
+// cluster barrier keeps the other ranks until it has read them.  No global scratch, no flags.
+// The first codes are loaded before griddepcontrol.wait: weights do not depend on the preceding
+// kernel.
 constexpr int kQWarps = 8;
 constexpr int kQThreads = kQWarps * 32;
-constexpr int kQRows = 8;
+constexpr int kQRows = 64;  // rows per CTA
+constexpr int kQUnroll = 4; // blocks in flight per warp and buffer
+constexpr int kQMaxParts = 8;
 
-__device__ __forceinline__ float2 codes_f2(uint32_t u, int b0) {
-    // bytes b0, b0 + 1 of u as the floats 2^23 + byte, then minus 2^23: the byte's value, exactly
-    const float2 f = make_float2(__int_as_float((int)__byte_perm(u, 0x4B000000u, 0x7540u + (unsigned)b0)),
-                                 __int_as_float((int)__byte_perm(u, 0x4B000000u, 0x7541u + (unsigned)b0)));
-    return __fadd2_rn(f, make_float2(-8388608.0f, -8388608.0f));
+__device__ __forceinline__ void mma_u8s8(int (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k32.row.col.s32.u8.s8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+r"(d[0]), "+r"(d[1]), "+r"(d[2]), "+r"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// sum over the chunk's codes of (biased code) * x; x: the chunk's input values in shared memory
-template <int BITS>
-__device__ __forceinline__ float chunk_dot(const uint4& c, const float* x) {
-    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
-    float2 s0 = make_float2(0.f, 0.f), s1 = make_float2(0.f, 0.f);
-    if constexpr (BITS == 8) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float4 xv = *reinterpret_cast<const float4*>(x + 4 * i);
-            s0 = __ffma2_rn(codes_f2(w[i], 0), make_float2(xv.x, xv.y), s0);
-            s1 = __ffma2_rn(codes_f2(w[i], 2), make_float2(xv.z, xv.w), s1);
-        }
-    } else {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint32_t lo = w[i] & 0x0F0F0F0Fu, hi = (w[i] >> 4) & 0x0F0F0F0Fu;
-            const float4 xa = *reinterpret_cast<const float4*>(x + 8 * i);
-            const float4 xb = *reinterpret_cast<const float4*>(x + 8 * i + 4);
-            s0 = __ffma2_rn(codes_f2(lo, 0), make_float2(xa.x, xa.y), s0);
-            s1 = __ffma2_rn(codes_f2(lo, 2), make_float2(xa.z, xa.w), s1);
-            s0 = __ffma2_rn(codes_f2(hi, 0), make_float2(xb.x, xb.y), s0);
-            s1 = __ffma2_rn(codes_f2(hi, 2), make_float2(xb.z, xb.w), s1);
-        }
-    }
-    return (s0.x + s0.y) + (s1.x + s1.y);
+// Blocks of part `part` of `parts` over nb blocks.
+__device__ __forceinline__ void part_blocks(int nb, int part, int parts, int& b0, int& b1) {
+    b0 = (int)(((int64_t)part * nb) / parts);
+    b1 = (int)(((int64_t)(part + 1) * nb) / parts);
 }
+// shared-memory bytes of a CTA whose part has at most `pb` blocks: per block 3 x 32 digits, then
+// 16 bytes of scales (s1, s2, s3) and 16 of bias-scaled digit sums
+static size_t gemv_q_smem(int pb) { return (size_t)pb * (96 + 16 + 16) + 16; }
 
 template <int EPI, int BITS>
 __global__ void __launch_bounds__(kQThreads) k_gemv_q(const __grid_constant__ QGemvArgs a) {
-    constexpr int CPC = BITS == 8 ? 16 : 32;  // codes per 16-byte chunk
-    constexpr float BIAS = BITS == 8 ? 128.f : 8.f;
-    extern __shared__ __align__(16) float qsm[];
+    constexpr int BIAS = BITS == 8 ? 128 : 8;
+    extern __shared__ __align__(16) uint8_t qsm[];
     __shared__ float red[kQWarps + 1];
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    __shared__ float rsum[kQWarps][16];
+    __shared__ float rows_sum[kQRows];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
     const QMatDev& W = a.w;
-    const int kp = W.nb * kQBlock;                 // padded row length of the input
-    const int nch = (int)(W.row_bytes >> 4);       // chunks per row
-    float* xs = qsm;                               // [kp] input (zero past k)
-    float* cs = qsm + kp;                          // [nch] input sum of each chunk
-    const int ngroups = (W.rows + kQRows - 1) / kQRows;
-    const int g0 = (int)(((int64_t)blockIdx.x * ngroups) / gridDim.x);
-    const int g1 = (int)(((int64_t)(blockIdx.x + 1) * ngroups) / gridDim.x);
-    const int nbi = (nch + 31) / 32;               // chunk rounds per row
-    const int my_groups = g1 - g0 > warp ? (g1 - g0 - warp + kQWarps - 1) / kQWarps : 0;
-    const int n_steps = my_groups * nbi;
+    const int nb = W.nb;
+    const int parts = (int)gridDim.x, part = (int)blockIdx.x;  // cluster (parts, 1, 1): rank = part
+    int pb0, pb1;
+    part_blocks(nb, part, parts, pb0, pb1);
+    const int npb = pb1 - pb0;
+    int8_t* xq = reinterpret_cast<int8_t*>(qsm);                           // [npb][3][32]
+    float4* xsc = reinterpret_cast<float4*>(qsm + (size_t)npb * 96);       // [npb] (s1, s2, s3, -)
+    int4* xsum = reinterpret_cast<int4*>(xsc + npb);                       // [npb] bias * digit sums
+    const int tile = warp & 3, half = warp >> 2;
+    const int row0 = (int)blockIdx.y * kQRows + tile * 16;
+    const int ra = row0 + g, rb = row0 + g + 8;
+    const bool oka = ra < W.rows, okb = rb < W.rows;
+    // this warp's blocks: half `half` of the part
+    const int wb0 = pb0 + (half == 0 ? 0 : npb / 2), wb1 = half == 0 ? pb0 + npb / 2 : pb1;
+    const uint8_t* ca = W.codes + (int64_t)(oka ? ra : 0) * W.row_bytes;
+    const uint8_t* cb = W.codes + (int64_t)(okb ? rb : 0) * W.row_bytes;
+    const __half* sa = W.scales + (int64_t)(oka ? ra : 0) * nb;
+    const __half* sb = W.scales + (int64_t)(okb ? rb : 0) * nb;
 
-    auto load = [&](uint4 (&b)[kQRows], __half (&d)[kQRows], int s) {
-        const int gi = s / nbi, bi = s - gi * nbi;
-        const int row0 = (g0 + warp + kQWarps * gi) * kQRows, ch = bi * 32 + lane;
-        const bool on = s < n_steps && ch < nch;
-        const int sidx = BITS == 8 ? ch >> 1 : ch;
+    // codes of rows g, g + 8 (8 bytes each at 8 bits, a word at 4) and, in lane t = 0, the rows'
+    // weight scales, for kQUnroll blocks from block bb
+    auto load = [&](uint2 (&va)[kQUnroll], uint2 (&vb)[kQUnroll], __half2 (&dv)[kQUnroll], int bb) {
 #pragma unroll
-        for (int r = 0; r < kQRows; ++r) {
-            const bool ok = on && row0 + r < W.rows;
-            b[r] = ok ? ldg_stream(W.codes + (int64_t)(row0 + r) * W.row_bytes + (int64_t)ch * 16) : make_uint4(0u, 0u, 0u, 0u);
-            d[r] = ok ? W.scales[(int64_t)(row0 + r) * W.nb + sidx] : __float2half(0.f);
+        for (int u = 0; u < kQUnroll; ++u) {
+            const int b = bb + u;
+            const bool on = b < wb1;
+            if constexpr (BITS == 8) {
+                va[u] = on && oka ? ldg_stream_u2(ca + (int64_t)b * 32 + 8 * t) : make_uint2(0u, 0u);
+                vb[u] = on && okb ? ldg_stream_u2(cb + (int64_t)b * 32 + 8 * t) : make_uint2(0u, 0u);
+            } else {
+                va[u].x = on && oka ? ldg_stream_u1(ca + (int64_t)b * 16 + 4 * t) : 0u;
+                vb[u].x = on && okb ? ldg_stream_u1(cb + (int64_t)b * 16 + 4 * t) : 0u;
+                va[u].y = vb[u].y = 0u;
+            }
+            const __half z = __float2half(0.f);
+            dv[u] = __halves2half2(on && oka && t == 0 ? sa[b] : z, on && okb && t == 0 ? sb[b] : z);
         }
     };
-    uint4 b0[kQRows], b1[kQRows];
-    __half d0[kQRows], d1[kQRows];
-    load(b0, d0, 0);
-    load(b1, d1, 1);
+    uint2 pa[2][kQUnroll], pb[2][kQUnroll];
+    __half2 pd[2][kQUnroll];
+    load(pa[0], pb[0], pd[0], wb0);
+    load(pa[1], pb[1], pd[1], wb0 + kQUnroll);
     pdl_wait();
 
-    // ---------------------------------------------------------------- input into shared memory
+    // ---------------------------------------------------------------- input digits of the part
+    float rinv = 1.f;
     if (a.x != nullptr) {
         float ss = 0.f;
         for (int i = tid; i < W.k; i += kQThreads) {
@@ -175,86 +187,147 @@ __global__ void __launch_bounds__(kQThreads) k_gemv_q(const __grid_constant__ QG
         if (lane == 0) red[warp] = ss;
         __syncthreads();
         if (tid == 0) {
-            float tot = 0.f;
-            for (int w = 0; w < kQWarps; ++w) tot += red[w];
-            red[kQWarps] = 1.0f / sqrtf(tot / (float)W.k + a.eps);
+            float s = 0.f;
+            for (int w = 0; w < kQWarps; ++w) s += red[w];
+            red[kQWarps] = 1.0f / sqrtf(s / (float)W.k + a.eps);
         }
         __syncthreads();
-        const float rinv = red[kQWarps];
-        for (int i = tid; i < kp; i += kQThreads)
-            xs[i] = i < W.k ? __half2float(a.x[i]) * rinv * __half2float(a.gain[i]) : 0.f;
-    } else {
-        for (int i = tid; i < kp; i += kQThreads) xs[i] = i < W.k ? __ldcg(a.vin + i) : 0.f;
+        rinv = red[kQWarps];
     }
-    __syncthreads();
-    for (int c = tid; c < nch; c += kQThreads) {
-        float t = 0.f;
-        for (int e = 0; e < CPC; ++e) t += xs[c * CPC + e];
-        cs[c] = t;
+    for (int j = warp; j < npb; j += kQWarps) {
+        const int i = (pb0 + j) * kQBlock + lane;
+        float v = 0.f;
+        if (i < W.k) v = a.x != nullptr ? __half2float(a.x[i]) * rinv * __half2float(a.gain[i]) : __ldcg(a.vin + i);
+        // the block's largest magnitude (non-negative floats order as their bit patterns)
+        const float amax = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(fabsf(v))));
+        const float s1 = amax / 127.0f, s2 = s1 / 254.0f, s3 = s2 / 254.0f;
+        const float i1 = amax > 0.f ? 127.0f / amax : 0.f, i2 = i1 * 254.0f, i3 = i2 * 254.0f;
+        // three digits: each takes the remainder of the ones before, to within half its step
+        const float sc[3] = {s1, s2, s3}, iv[3] = {i1, i2, i3};
+        int q[3];
+        float r = v;
+#pragma unroll
+        for (int e = 0; e < 3; ++e) {
+            const float f = rintf(r * iv[e]);
+            q[e] = (int)fminf(fmaxf(f, -127.f), 127.f);
+            r = fmaf(-(float)q[e], sc[e], r);
+        }
+        // digits in the codes' own (natural) order: A and B fragments are both loaded by byte
+        // position, so the MMA sees the same permutation of k on both sides
+        int qs[3];
+#pragma unroll
+        for (int e = 0; e < 3; ++e) {
+            xq[j * 96 + e * 32 + lane] = (int8_t)q[e];
+            qs[e] = __reduce_add_sync(0xffffffffu, q[e]);
+        }
+        if (lane == 0) {
+            xsc[j] = make_float4(s1, s2, s3, 0.f);
+            xsum[j] = make_int4(BIAS * qs[0], BIAS * qs[1], BIAS * qs[2], 0);
+        }
     }
     __syncthreads();
     pdl_launch_dependents();
 
-    float acc[kQRows];
-    auto consume = [&](const uint4 (&b)[kQRows], const __half (&d)[kQRows], int s) {
-        const int gi = s / nbi, bi = s - gi * nbi;
-        const int row0 = (g0 + warp + kQWarps * gi) * kQRows, ch = bi * 32 + lane;
-        if (bi == 0)
+    // ---------------------------------------------------------------- this warp's blocks
+    float acc_a = 0.f, acc_b = 0.f;
+    auto consume = [&](const uint2 (&va)[kQUnroll], const uint2 (&vb)[kQUnroll], const __half2 (&dv)[kQUnroll], int bb) {
 #pragma unroll
-            for (int r = 0; r < kQRows; ++r) acc[r] = 0.f;
-        if (ch < nch) {
-            const float* x = xs + ch * CPC;
-            const float bsum = BIAS * cs[ch];
-#pragma unroll
-            for (int r = 0; r < kQRows; ++r) acc[r] = fmaf(__half2float(d[r]), chunk_dot<BITS>(b[r], x) - bsum, acc[r]);
-        }
-        if (bi == nbi - 1) {
-            float v[8];
-#pragma unroll
-            for (int r = 0; r < kQRows; ++r) v[r] = acc[r];
-            const float t = multi_row_sum<kQRows>(v, lane);  // lane 4 r holds row row0 + r
-            const float t_odd = __shfl_down_sync(0xffffffffu, t, 4);  // the next row's total
-            const int r = lane >> 2, row = row0 + r;
-            if ((lane & 3) == 0 && row < W.rows) {
-                if constexpr (EPI == kEpiPlain) {
-                    a.out[row] = t;
-                } else if ((r & 1) == 0 && row + 1 < W.rows) {
-                    if constexpr (EPI == kEpiSwiglu) {
-                        a.out[row >> 1] = silu(t) * t_odd;
-                    } else {  // kEpiQkvRope: rows (row, row + 1) are the RoPE pair (i, i + dh / 2)
-                        const int p = *a.len;
-                        const bool ok = p >= 0 && p < a.cap;
-                        if (!ok && row == 0) set_status(a.status, VT_DEV_KV_OVERFLOW);
-                        const int half = a.dh >> 1;
-                        const int blk = row / a.dh, i = (row - blk * a.dh) >> 1;
-                        if (blk < a.hq + a.hk) {
-                            const float2 cs2 = ok ? a.rope[(int64_t)p * half + i] : make_float2(1.f, 0.f);
-                            const float re = t * cs2.x - t_odd * cs2.y;
-                            const float ro = t * cs2.y + t_odd * cs2.x;
-                            if (blk < a.hq) {
-                                a.out[blk * a.dh + i] = re;
-                                a.out[blk * a.dh + i + half] = ro;
-                            } else if (ok) {
-                                __half* kd = a.kcache + ((int64_t)(blk - a.hq) * a.cap + p) * a.dh;
-                                kd[i] = __float2half_rn(re);
-                                kd[i + half] = __float2half_rn(ro);
-                            }
-                        } else if (ok) {
-                            __half* vd = a.vcache + ((int64_t)(blk - a.hq - a.hk) * a.cap + p) * a.dh;
-                            vd[i] = __float2half_rn(t);
-                            vd[i + half] = __float2half_rn(t_odd);
-                        }
-                    }
-                }
+        for (int u = 0; u < kQUnroll; ++u) {
+            const int b = bb + u;
+            if (b >= wb1) break;
+            const int j = b - pb0;
+            uint32_t af[4];
+            if constexpr (BITS == 8) {
+                af[0] = va[u].x;
+                af[1] = vb[u].x;
+                af[2] = va[u].y;
+                af[3] = vb[u].y;
+            } else {  // byte i of the word: code 8t + i (low nibble), 8t + 4 + i (high nibble)
+                af[0] = va[u].x & 0x0F0F0F0Fu;
+                af[1] = vb[u].x & 0x0F0F0F0Fu;
+                af[2] = (va[u].x >> 4) & 0x0F0F0F0Fu;
+                af[3] = (vb[u].x >> 4) & 0x0F0F0F0Fu;
+            }
+            uint2 bf = make_uint2(0u, 0u);
+            if (g < 3) bf = *reinterpret_cast<const uint2*>(xq + j * 96 + g * 32 + 8 * t);
+            int d[4] = {0, 0, 0, 0};
+            mma_u8s8(d, af, bf.x, bf.y);
+            // lane t = 0 holds the digit-1 and digit-2 products of rows g, g + 8; lane t = 1 digit 3
+            const int d3a = __shfl_down_sync(0xffffffffu, d[0], 1);
+            const int d3b = __shfl_down_sync(0xffffffffu, d[2], 1);
+            if (t == 0) {
+                const float4 sc = xsc[j];
+                const int4 qb = xsum[j];
+                float va_ = sc.z * (float)(d3a - qb.z);
+                va_ = fmaf(sc.y, (float)(d[1] - qb.y), va_);
+                va_ = fmaf(sc.x, (float)(d[0] - qb.x), va_);
+                float vb_ = sc.z * (float)(d3b - qb.z);
+                vb_ = fmaf(sc.y, (float)(d[3] - qb.y), vb_);
+                vb_ = fmaf(sc.x, (float)(d[2] - qb.x), vb_);
+                const float2 ds = __half22float2(dv[u]);
+                acc_a = fmaf(ds.x, va_, acc_a);
+                acc_b = fmaf(ds.y, vb_, acc_b);
             }
         }
     };
-    for (int s = 0; s < n_steps; s += 2) {
-        consume(b0, d0, s);
-        load(b0, d0, s + 2);
-        if (s + 1 < n_steps) {
-            consume(b1, d1, s + 1);
-            load(b1, d1, s + 3);
+    for (int bb = wb0; bb < wb1; bb += 2 * kQUnroll) {
+        consume(pa[0], pb[0], pd[0], bb);
+        load(pa[0], pb[0], pd[0], bb + 2 * kQUnroll);
+        if (bb + kQUnroll < wb1) {
+            consume(pa[1], pb[1], pd[1], bb + kQUnroll);
+            load(pa[1], pb[1], pd[1], bb + 3 * kQUnroll);
+        }
+    }
+    if (t == 0) {
+        rsum[warp][g] = acc_a;
+        rsum[warp][g + 8] = acc_b;
+    }
+    __syncthreads();
+    if (tid < kQRows) rows_sum[tid] = rsum[tid >> 4][tid & 15] + rsum[4 + (tid >> 4)][tid & 15];  // halves in order
+
+    // ---------------------------------------------------------------- parts of the cluster
+    if (parts > 1) cluster_sync();  // every part's row sums are in its shared memory
+    else __syncthreads();
+    float tv = 0.f;
+    const int r = tid, row = (int)blockIdx.y * kQRows + r;
+    if (part == 0 && tid < kQRows) {
+        for (int p = 0; p < parts; ++p) tv += p == 0 ? rows_sum[r] : dsmem_ld(dsmem_addr(&rows_sum[r], (uint32_t)p));
+        rows_sum[r] = tv;
+    }
+    if (parts > 1) cluster_sync();  // rank 0 has read the others' sums (they may leave), and its own are final
+    else __syncthreads();
+    if (part != 0 || tid >= kQRows || row >= W.rows) return;
+
+    // ---------------------------------------------------------------- epilogue (row pairs)
+    if constexpr (EPI == kEpiPlain) {
+        a.out[row] = tv;
+    } else if ((r & 1) == 0 && row + 1 < W.rows) {
+        const float t_odd = rows_sum[r + 1];
+        if constexpr (EPI == kEpiSwiglu) {
+            a.out[row >> 1] = silu(tv) * t_odd;
+        } else {  // kEpiQkvRope: rows (row, row + 1) are the RoPE pair (i, i + dh / 2)
+            const int p = *a.len;
+            const bool ok = p >= 0 && p < a.cap;
+            if (!ok && row == 0) set_status(a.status, VT_DEV_KV_OVERFLOW);
+            const int hd = a.dh >> 1;
+            const int blk = row / a.dh, i = (row - blk * a.dh) >> 1;
+            if (blk < a.hq + a.hk) {
+                const float2 cs2 = ok ? a.rope[(int64_t)p * hd + i] : make_float2(1.f, 0.f);
+                const float re = tv * cs2.x - t_odd * cs2.y;
+                const float ro = tv * cs2.y + t_odd * cs2.x;
+                if (blk < a.hq) {
+                    a.out[blk * a.dh + i] = re;
+                    a.out[blk * a.dh + i + hd] = ro;
+                } else if (ok) {
+                    __half* kd = a.kcache + ((int64_t)(blk - a.hq) * a.cap + p) * a.dh;
+                    kd[i] = __float2half_rn(re);
+                    kd[i + hd] = __float2half_rn(ro);
+                }
+            } else if (ok) {
+                __half* vd = a.vcache + ((int64_t)(blk - a.hq - a.hk) * a.cap + p) * a.dh;
+                vd[i] = __float2half_rn(tv);
+                vd[i + hd] = __float2half_rn(t_odd);
+            }
         }
     }
 }
@@ -323,22 +396,37 @@ cudaError_t launch_quantize_rows(const __half* w, int64_t ld, const QMatDev& m, 
     return cudaGetLastError();
 }
 
+// Parts per row tile: enough CTAs for about 2.5 per SM, each part at least 4 blocks, at most 8
+// (the portable cluster size).
+static int gemv_q_parts(int rows, int nb) {
+    const int tiles = (rows + kQRows - 1) / kQRows;
+    const int want = (int)std::lround(2.5 * (g_num_sms > 0 ? g_num_sms : 148) / std::max(tiles, 1));
+    return std::max(1, std::min({kQMaxParts, want, std::max(1, nb / 4)}));
+}
+
 template <int EPI>
 static cudaError_t launch_q_epi(const QGemvArgs& a, cudaStream_t st) {
-    const int ngroups = (a.w.rows + kQRows - 1) / kQRows;
-    int grid = (g_num_sms > 0 ? g_num_sms : 148) * 2;
-    grid = std::min(grid, std::max(ngroups, 1));
-    const size_t smem = ((size_t)a.w.nb * kQBlock + (size_t)(a.w.row_bytes >> 4)) * sizeof(float);
+    const int parts = gemv_q_parts(a.w.rows, a.w.nb);
+    const int pb = (a.w.nb + parts - 1) / parts;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid);
+    cfg.gridDim = dim3((unsigned)parts, (unsigned)((a.w.rows + kQRows - 1) / kQRows));
     cfg.blockDim = dim3(kQThreads);
-    cfg.dynamicSmemBytes = smem;
+    cfg.dynamicSmemBytes = gemv_q_smem(pb);
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = (unsigned)parts;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+    if (g_use_pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = g_use_pdl ? 1 : 0;
+    cfg.numAttrs = (unsigned)na;
     if (a.w.bits == 8) return cudaLaunchKernelEx(&cfg, k_gemv_q<EPI, 8>, a);
     if (a.w.bits == 4) return cudaLaunchKernelEx(&cfg, k_gemv_q<EPI, 4>, a);
     return cudaErrorInvalidValue;
@@ -346,8 +434,8 @@ static cudaError_t launch_q_epi(const QGemvArgs& a, cudaStream_t st) {
 
 cudaError_t launch_gemv_q(int epi, const QGemvArgs& a, cudaStream_t st) {
     if (a.w.rows <= 0) return cudaSuccess;
-    const size_t smem = ((size_t)a.w.nb * kQBlock + (size_t)(a.w.row_bytes >> 4)) * sizeof(float);
-    if (smem > 200 * 1024) return cudaErrorInvalidValue;
+    const int parts = gemv_q_parts(a.w.rows, a.w.nb);
+    if (gemv_q_smem((a.w.nb + parts - 1) / parts) > 200 * 1024) return cudaErrorInvalidValue;
     switch (epi) {
         case kEpiPlain: return launch_q_epi<kEpiPlain>(a, st);
         case kEpiSwiglu: return launch_q_epi<kEpiSwiglu>(a, st);
