@@ -49,9 +49,9 @@ FALLBACK_HBM_GBS = 6800.0
 # that kernel (mean of 12 launches of the 7B decode; profiles/k_decode_token_7b.md), and a
 # digest of the sources the captured kernel was built from.  The line reports the bytes only
 # while the sources still hash to that digest: a changed kernel reports null until recaptured.
-K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_504_014_827
+K_TOKEN_DRAM_BYTES_PER_LAUNCH = 13_504_082_645
 K_TOKEN_SOURCES = ("token_kernel.cuh", "token.cu", "token_v1.cu", "token_v2.cu", "internal.h", "device.cuh")
-K_TOKEN_SOURCES_SHA256 = "998cd22556cd4766"
+K_TOKEN_SOURCES_SHA256 = "1fcbc27eaa724733"
 
 
 def token_traffic_if_current():
@@ -545,16 +545,21 @@ def run_decode(args, rank, world):
     return line, clk.summary()
 
 
-def run_decode_workload(cid, steps, warmup, bits=16):
+def run_decode_workload(cid, steps, warmup, bits=16, layers=0):
     """Decode tok/s of one more workload (the 13B uneven 3-way and the 8B GQA 4-way shapes), timed
     like the headline one: vt_decode_token replayed as a CUDA graph over the workload's KV schedule
-    (kv_len -> kv_len + decode_steps - 1, then rewound), inputs resident on the device."""
+    (kv_len -> kv_len + decode_steps - 1, then rewound), inputs resident on the device.  layers > 0:
+    only the first `layers` layers (a small case for profiling)."""
+    import dataclasses
+
     import torch
 
     from paper_2607_07046_gb300 import vt
     from paper_2607_07046_gb300.stack import Stack
 
     wl = synthetic.WORKLOADS[cid]
+    if layers:
+        wl = dataclasses.replace(wl, n_layers=layers)
     sched = wl.decode_steps
     cap = wl.kv_len + sched + 8
     stream = torch.cuda.Stream()
@@ -730,10 +735,17 @@ def main():
                     help="repeat the K-step timed region until it covers this many seconds in total")
     ap.add_argument("--other-steps", type=int, default=64,
                     help="timed tokens of the 13B and 8B decode workloads, 1 GPU only (0: skip)")
+    ap.add_argument("--quantized", type=int, default=0, choices=[0, 4, 8],
+                    help="only the 7B decode with every shard block-quantized to this many bits "
+                         "(--other-steps timed tokens; --layers for a small case)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.sweep:
         print(json.dumps(run_sweep(args)), flush=True)
+        return
+    if args.quantized:
+        print(json.dumps(run_decode_workload(2, max(args.other_steps, 1), args.warmup, args.quantized, args.layers)),
+              flush=True)
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
