@@ -999,7 +999,7 @@ struct PrefillAttnKArgs {
     __half* out;  // [n][hq * dh]
 };
 
-// The shards of one ATTN block in one launch: blockIdx.y runs over every shard's query heads
+// The shards of one ATTN block in one launch: blockIdx.x runs over every shard's query heads
 // (shard g owns [head_end[g - 1], head_end[g])).
 struct PrefillAttnGroup {
     int n_groups;
@@ -1046,8 +1046,11 @@ constexpr size_t prefill_attn_smem() {
 // loads hit distinct banks).
 template <int DH>
 __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ PrefillAttnGroup G) {
+    // blockIdx.x: the query head over every shard, the fastest index, so that the heaviest row
+    // tiles of every head are dispatched first; blockIdx.y: the row tile from the end
+    const int hg = (int)blockIdx.x;
     int gi = 0;
-    while (gi + 1 < G.n_groups && (int)blockIdx.y >= G.head_end[gi]) ++gi;
+    while (gi + 1 < G.n_groups && hg >= G.head_end[gi]) ++gi;
     const PrefillAttnKArgs& a = G.a[gi];
     constexpr int LDS = DH + 8, KC = DH / 16, DT = DH / 8;
     extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -1055,8 +1058,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ Pr
     __half* Vs = Ks + 2 * kAttnKeys * LDS;              // [2][64][LDS]
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
     // the last row tiles see the most positions: they are scheduled first
-    const int h = (int)blockIdx.y - (gi > 0 ? G.head_end[gi - 1] : 0), j = h / a.group;
-    const int r0 = ((int)gridDim.x - 1 - (int)blockIdx.x) * kAttnRows;
+    const int h = hg - (gi > 0 ? G.head_end[gi - 1] : 0), j = h / a.group;
+    const int r0 = ((int)gridDim.y - 1 - (int)blockIdx.y) * kAttnRows;
 
     pdl_wait();
     const int P0 = *a.len + a.row_offset;
@@ -1595,7 +1598,7 @@ static vt_status prefill_attention(const PrefillAttnArgs* as, int n, cudaStream_
     }
     G.n_groups = n;
     if (n < 1 || heads < 1) return VT_OK;
-    const dim3 grid((as[0].n + kAttnRows - 1) / kAttnRows, heads);
+    const dim3 grid(heads, (as[0].n + kAttnRows - 1) / kAttnRows);
     if (as[0].dh == 128) k_prefill_attn<128><<<grid, 128, prefill_attn_smem<128>(), st>>>(G);
     else k_prefill_attn<64><<<grid, 128, prefill_attn_smem<64>(), st>>>(G);
     cudaError_t e = cudaGetLastError();
