@@ -663,8 +663,9 @@ __device__ __forceinline__ Ring attn_slice(const TokArgs& a, const TokShardPtrs*
 }
 
 // The attention output of shard s (K = its query heads x dh), merged from the slice states with
-// log-sum-exp weights: each thread takes 4 consecutive elements of one query head and issues all
-// its loads together; the result goes to xh / xl as fp16 hi / lo halves.
+// log-sum-exp weights: each thread takes 4 consecutive elements of one query head and issues the
+// loads of 8 slices together (heads cut into more slices take further batches of 8); the result
+// goes to xh / xl as fp16 hi / lo halves.
 __device__ __forceinline__ void merge_heads(const TokArgs& a, int s, int K, const int* mtab, int mstride, int dsh, int gsh,
                                          __half* xh, __half* xl, int tid) {
     const int dh = a.dh, G = a.group;
@@ -689,8 +690,6 @@ __device__ __forceinline__ void merge_heads(const TokArgs& a, int s, int K, cons
         float M = -INFINITY;
 #pragma unroll
         for (int k = 0; k < 8; ++k) M = fmaxf(M, ml[k].x);
-        for (int k = 8; k < mstride; ++k)  // heads split over more than 8 CTAs
-            if (tb[k] >= 0) M = fmaxf(M, __ldcg(a.states + tb[k] + g * (dh + 4)));
         float L = 0.f, y0 = 0.f, y1 = 0.f, y2 = 0.f, y3 = 0.f;
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
@@ -701,17 +700,42 @@ __device__ __forceinline__ void merge_heads(const TokArgs& a, int s, int K, cons
             y2 = fmaf(ov[k].z, w, y2);
             y3 = fmaf(ov[k].w, w, y3);
         }
-        for (int k = 8; k < mstride; ++k) {
-            if (tb[k] < 0) continue;
-            const float* st = a.states + tb[k] + g * (dh + 4);
-            const float2 m2 = __ldcg(reinterpret_cast<const float2*>(st));
-            const float4 o4 = __ldcg(reinterpret_cast<const float4*>(st + 4 + d));
-            const float w = exp2f(m2.x - M);
-            L = fmaf(m2.y, w, L);
-            y0 = fmaf(o4.x, w, y0);
-            y1 = fmaf(o4.y, w, y1);
-            y2 = fmaf(o4.z, w, y2);
-            y3 = fmaf(o4.w, w, y3);
+        // heads split over more than 8 CTAs (long caches): further slices 8 at a time, each
+        // batch's loads issued together, the running sums rescaled when a batch raises the maximum
+        for (int k0 = 8; k0 < mstride; k0 += 8) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int b = k0 + k < mstride ? tb[k0 + k] : -1;
+                if (b >= 0) {
+                    const float* st = a.states + b + g * (dh + 4);
+                    ml[k] = __ldcg(reinterpret_cast<const float2*>(st));
+                    ov[k] = __ldcg(reinterpret_cast<const float4*>(st + 4 + d));
+                } else {
+                    ml[k] = make_float2(-INFINITY, 0.f);
+                    ov[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            }
+            float nm = M;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) nm = fmaxf(nm, ml[k].x);
+            if (M != -INFINITY && nm != M) {
+                const float r = exp2f(M - nm);
+                L *= r;
+                y0 *= r;
+                y1 *= r;
+                y2 *= r;
+                y3 *= r;
+            }
+            M = nm;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const float w = ml[k].x == -INFINITY ? 0.f : exp2f(ml[k].x - M);
+                L = fmaf(ml[k].y, w, L);
+                y0 = fmaf(ov[k].x, w, y0);
+                y1 = fmaf(ov[k].y, w, y1);
+                y2 = fmaf(ov[k].z, w, y2);
+                y3 = fmaf(ov[k].w, w, y3);
+            }
         }
         const float linv = L > 0.f ? 1.0f / L : 0.f;
         const float yv[4] = {y0 * linv, y1 * linv, y2 * linv, y3 * linv};
