@@ -544,7 +544,8 @@ VT_API vt_status vt_token_test_barrier(vt_partition* part, int32_t cta, uint32_t
  * 3.2.1): n prompt rows through every layer (same order as vt_decode_token), then every layer's
  * KV length advances by n.  x_in, x_out: device fp16 [n, D], may be the same.  The shards of a
  * block run together: one tensor-core GEMM launch per projection covers every shard (each with
- * its own partial), then the combine adds them in shard order. */
+ * its own partial), then the combine adds them in shard order.  Prompts longer than 1024 rows run
+ * in chunks of 1024.  Every shard must be fp16: VT_ERR_STATE when one is block-quantized. */
 VT_API vt_status vt_prefill_tokens(const vt_partition* part, vt_kv* kv, const void* x_in, int32_t n,
                             void* x_out, vt_stream stream);
 

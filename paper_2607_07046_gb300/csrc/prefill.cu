@@ -9,10 +9,16 @@
 // in tensor memory, operands staged by TMA); X^, Q, the attention output and U are fp16 operands,
 // accumulation and partials are fp32.
 //
-//   k_rmsnorm_rows   one CTA per row
-//   k_gemm           C = A . B^T, A [M][K] and B [N][K] fp16 (K contiguous), one 128 x 256 output
-//                    tile per CTA; epilogues: fp32 store, RoPE + q store + KV append, SwiGLU
-//   k_prefill_attn   causal flash attention, 64 query rows of one head per CTA (mma.sync)
+//   k_rmsnorm_rows   one CTA per row (also the fp16 hi / lo split of the ATTN input)
+//   k_combine_norm   residual + shard partials in shard order, then the next block's RMSNorm
+//   k_gemm_p         C = A . B^T, A [M][K] and B [N][K] fp16 (K contiguous), persistent over the
+//                    output tiles of every shard's GEMM of a block: CTA pairs (tcgen05 cta_group::2,
+//                    256 x BN tiles) or single CTAs (128 x 256); epilogues: fp32 store, RoPE + q
+//                    store + KV append, SwiGLU
+//   k_gemm           the same MMA and copies, one 128 x 256 tile per CTA with an optional
+//                    cluster split-K, for groups too small to fill the GPU
+//   k_prefill_attn   causal flash attention, 64 query rows of one head per CTA (mma.sync), one
+//                    launch over every shard's heads
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
