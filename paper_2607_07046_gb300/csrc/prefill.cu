@@ -17,8 +17,8 @@
 //                    store + KV append, SwiGLU
 //   k_gemm           the same MMA and copies, one 128 x 256 tile per CTA with an optional
 //                    cluster split-K, for groups too small to fill the GPU
-//   k_prefill_attn   causal flash attention, 64 query rows of one head per CTA (mma.sync), one
-//                    launch over every shard's heads
+//   k_prefill_attn_tc causal flash attention on tcgen05 (S and O in tensor memory, K / V by TMA),
+//                    128 query rows of one head per CTA, one launch over every shard's heads
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
@@ -26,6 +26,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <climits>
 #include <cstdlib>
 #include <string>
 
@@ -74,6 +75,14 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* m
         "[%4];" ::"r"(smem_u32(dst)),
         "l"(map), "r"(x), "r"(y), "r"(bar)
         : "memory");
+}
+
+// 2-D tiled TMA store of a shared-memory box to (x, y) of the map's tensor (rows past the
+// tensor's end are not written); completion is tracked by the bulk async-group of this thread.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int y, const void* src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(map), "r"(x),
+                 "r"(y), "r"(smem_u32(src))
+                 : "memory");
 }
 
 // 16-byte store into the shared memory of a CTA of the cluster (address from mapa).
@@ -160,6 +169,30 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
         : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// The wait with the loaded registers as operands, so that no use of them is scheduled before it.
+__device__ __forceinline__ void tmem_ld_wait_on(uint32_t (&r)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                   "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                   "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+                 :
+                 : "memory");
+}
+// The store counterpart: thread t writes 32 consecutive columns of lane (base + t).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+        "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+        "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 // Shared-memory matrix descriptor of a K-major operand tile written by TMA with the 128-byte
 // swizzle: rows of 64 fp16 (128 bytes), 8-row groups 1024 bytes apart.  The tile base is 1024-byte
@@ -174,10 +207,26 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
     return d;
 }
 
+// Descriptor of an MN-major operand (the N index contiguous) written by TMA with the 128-byte
+// swizzle: each K index is one 128-byte row of 64 consecutive N elements, 8-row groups are 1024
+// bytes apart, and the next 64 N elements sit `lbo` bytes further (the next TMA box).  Stepping K
+// by 16 advances the start address by 16 rows (2048 bytes).
+__device__ __forceinline__ uint64_t desc_sw128_mn(uint32_t saddr, uint32_t lbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+    d |= (uint64_t)(lbo >> 4) << 16;           // offset between 64-element groups of N
+    d |= (uint64_t)(1024 >> 4) << 32;          // stride between 8-row groups of K
+    d |= (uint64_t)1 << 46;                    // descriptor version
+    d |= (uint64_t)2 << 61;                    // 128-byte swizzle
+    return d;
+}
+
 // Instruction descriptor: fp16 A and B (both K-major), fp32 accumulator, M x N.
 __host__ __device__ constexpr uint32_t idesc_f16(int m, int n) {
     return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
+// The same with B MN-major (transposed B).
+__host__ __device__ constexpr uint32_t idesc_f16_bmn(int m, int n) { return idesc_f16(m, n) | (1u << 16); }
 
 }  // namespace tc
 
@@ -992,224 +1041,445 @@ static int pgemm_stages(int bn_cta, int kts) {
     return s > kPStages ? kPStages : s;
 }
 
-// ================================================================== causal attention
-
-struct PrefillAttnKArgs {
-    const __half* q;  // [n][hq][dh]
-    const __half* kcache;
-    const __half* vcache;
-    const int32_t* len;
-    int row_offset, n, hq, group, cap;
-    int window;  // > 0: row at position p sees positions [p - window + 1, p]
-    float scale_log2;
-    __half* out;  // [n][hq * dh]
-};
-
-// The shards of one ATTN block in one launch: blockIdx.x runs over every shard's query heads
-// (shard g owns [head_end[g - 1], head_end[g])).
-struct PrefillAttnGroup {
-    int n_groups;
-    int head_end[VT_MAX_DEVICES];
-    PrefillAttnKArgs a[VT_MAX_DEVICES];
-};
-
-__device__ __forceinline__ void cp_async16(void* s, const void* g) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(s)), "l"(g) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
 __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
     const __half2 h = __floats2half2_rn(lo, hi);
     return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-constexpr int kAttnRows = 64;  // query rows per CTA (16 per warp)
-constexpr int kAttnKeys = 64;  // cached positions per tile
+// ================================================================== causal attention on tcgen05
+//
+// One CTA per (query head, 128-row tile); the launch covers every shard's heads (up to kFaGroups
+// shards).  The attended positions [kbeg, kend) of the tile are walked in blocks of 128 keys:
+//   S_j = Q . K_j^T           (tcgen05, M 128, N 128, K dh; fp32 in tensor memory)
+//   P_j = 2^(S_j log2(e)/sqrt(dh) - m), masked (causal, window), fp16 into shared memory
+//   O  += P_j . V_j           (tcgen05, M 128, N dh, K 128, one accumulator in tensor memory; V
+//                              read MN-major as it lies in the cache, so it needs no transpose)
+//   warp 0      TMA: one thread loads Q, then serves the K and V rings (two slots each), filling
+//               each slot as soon as the MMA that read it has completed;
+//   warp 1      tensor memory (S of even / odd blocks, O) and the MMA thread: S_0, S_1, then per
+//               block O += P_j V_j and S_{j+2} (S_{j+2} first when its operands are already there);
+//   warps 2-9   softmax: warp (g, q) holds query rows 32q .. 32q + 31 (its quarter of the tensor
+//               memory lanes) and key columns 64g .. 64g + 63 of every block; the two warps of a
+//               quarter exchange row maxima through shared memory.  m is a reference maximum: O
+//               (in tensor memory) and l are rescaled only when a row's block maximum exceeds it
+//               by more than 8 (log2 units), so P stays below 2^8.
+// Keys past the window or the causal bound, and rows past n (zero Q from TMA's fill), take no
+// part in any stored result; V rows outside [kbeg, kend) meet zero weights (the cache holds finite
+// values: zeroed at creation, written by the QKV epilogues).  Every wait is bounded; on a timeout
+// the CTA sets VT_DEV_WAIT_TIMEOUT and stops issuing, waits for what it issued and frees tensor
+// memory; the softmax warps still pass every named barrier, so no partner waits on them.
+constexpr int kFaRows = 128, kFaKeys = 128;
+constexpr int kFaThreads = 320;
+constexpr int kFaGroups = 6;  // four tensor maps a shard: 6 keep the parameters under 4 KB
 
+struct FaShard {
+    int n, hq, group, cap, row_offset, window;
+    const int32_t* len;  // rows sit at positions *len + row_offset + i
+    float scale_log2;
+    __half* out;         // [n][hq * dh]
+    uint32_t* status;
+};
+struct FaGroup {
+    int n_groups;
+    int head_end[kFaGroups];
+    CUtensorMap tq[kFaGroups], tk[kFaGroups], tv[kFaGroups];  // q [n][hq dh], K / V [hk cap][dh]
+    CUtensorMap to[kFaGroups];                                 // the output [n][hq dh]
+    FaShard a[kFaGroups];
+};
+
+// Q, two K and two V slots, two P slots, the max exchange (2 x 128 floats), barriers
 template <int DH>
-constexpr size_t prefill_attn_smem() {
-    return (size_t)4 * kAttnKeys * (DH + 8) * 2;  // K and V, two buffers each, padded rows
+constexpr size_t fa_smem() {
+    return 1024 + (size_t)kFaRows * DH * 2 + 4 * (size_t)kFaKeys * DH * 2 + 2 * (size_t)kFaRows * kFaKeys * 2 +
+           2 * kFaRows * 4 + 256;
 }
 
-// Flash attention (online softmax) over the causal set.  Warp w owns query rows r0 + 16 w ..
-// + 15; S = Q K^T and O += P V use m16n8k16 tensor-core MMAs with fp32 accumulation; K/V tiles of
-// 64 positions are double-buffered in shared memory (rows padded by 16 bytes so the fragment
-// loads hit distinct banks).
+// bounded wait polled by lane 0, result broadcast to the warp
+__device__ __forceinline__ bool fa_wait_warp(uint64_t* bar, uint32_t parity) {
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity) ? 1 : 0;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+// one non-blocking test of a phase
+__device__ __forceinline__ bool fa_test(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ void fa_pair_sync(uint32_t id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
+
+// 2^x on the special-function unit (inputs far below -126 and -inf give 0)
+__device__ __forceinline__ float fa_ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float fa_max3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// bits [b, e) of a 32-bit word, b and e clamped to [0, 32]
+__device__ __forceinline__ uint32_t fa_range_bits(int b, int e) {
+    b = max(0, min(32, b));
+    e = max(0, min(32, e));
+    if (e <= b) return 0u;
+    const uint32_t below_e = e == 32 ? 0xffffffffu : ((1u << e) - 1u);
+    return below_e & ~((1u << b) - 1u);
+}
+
 template <int DH>
-__global__ void __launch_bounds__(128) k_prefill_attn(const __grid_constant__ PrefillAttnGroup G) {
-    // blockIdx.x: the query head over every shard, the fastest index, so that the heaviest row
-    // tiles of every head are dispatched first; blockIdx.y: the row tile from the end
+__global__ void __launch_bounds__(kFaThreads, 1) k_prefill_attn_tc(const __grid_constant__ FaGroup G) {
+    constexpr uint32_t kQBytes = kFaRows * DH * 2, kKVBytes = kFaKeys * DH * 2, kPBytes = kFaRows * kFaKeys * 2;
+    constexpr uint32_t kAtom = kFaRows * 128;  // one 64-column box of 128 rows
+    constexpr uint32_t kOCol = 2 * kFaKeys;    // O's first tensor-memory column (after the two S)
     const int hg = (int)blockIdx.x;
     int gi = 0;
     while (gi + 1 < G.n_groups && hg >= G.head_end[gi]) ++gi;
-    const PrefillAttnKArgs& a = G.a[gi];
-    constexpr int LDS = DH + 8, KC = DH / 16, DT = DH / 8;
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    __half* Ks = reinterpret_cast<__half*>(smem_raw);  // [2][64][LDS]
-    __half* Vs = Ks + 2 * kAttnKeys * LDS;              // [2][64][LDS]
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
-    // the last row tiles see the most positions: they are scheduled first
-    const int h = hg - (gi > 0 ? G.head_end[gi - 1] : 0), j = h / a.group;
-    const int r0 = ((int)gridDim.y - 1 - (int)blockIdx.y) * kAttnRows;
+    const FaShard& a = G.a[gi];
+    const int h = hg - (gi > 0 ? G.head_end[gi - 1] : 0), kvh = h / a.group;
+    const int r0 = ((int)gridDim.y - 1 - (int)blockIdx.y) * kFaRows;  // heaviest tiles first
 
-    pdl_wait();
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint8_t* Qs = smem;
+    uint8_t* Ks = Qs + kQBytes;       // [2][kKVBytes]
+    uint8_t* Vs = Ks + 2 * kKVBytes;  // [2][kKVBytes]
+    uint8_t* Ps = Vs + 2 * kKVBytes;  // [2][kPBytes]
+    float* red = reinterpret_cast<float*>(Ps + 2 * kPBytes);  // [2 column halves][128 rows]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(red + 2 * kFaRows);
+    uint64_t* q_full = bars;
+    uint64_t* k_full = bars + 1;   // [2]
+    uint64_t* v_full = bars + 3;   // [2]
+    uint64_t* k_empty = bars + 5;  // [2]
+    uint64_t* v_empty = bars + 7;  // [2]
+    uint64_t* s_full = bars + 9;   // [2]
+    uint64_t* s_free = bars + 11;  // [2]
+    uint64_t* p_full = bars + 13;  // [2]
+    uint64_t* o_full = bars + 15;  // [2]: O += P_j V_j has completed, j even / odd
+    uint64_t* done = bars + 17;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+    volatile int* s_err = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        mbar_init(q_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_empty[s], 1);
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_free[s], 8);  // one arrival per softmax warp
+            mbar_init(&p_full[s], 8);
+            mbar_init(&o_full[s], 1);
+        }
+        mbar_init(done, 1);
+        *s_err = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(tmem_slot, 512);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    pdl_wait();  // q and the cache rows were written by the preceding kernel
+    // Q does not depend on the KV length: its load goes out first
+    if (warp == 0 && lane == 0 && r0 < a.n) {
+        mbar_arrive_expect_tx(q_full, kQBytes);
+        for (int c = 0; c < DH / 64; ++c) tc::tma_load_2d(Qs + c * kAtom, &G.tq[gi], h * DH + 64 * c, r0, q_full);
+    }
     const int P0 = *a.len + a.row_offset;
-    const int rlast = min(r0 + kAttnRows - 1, a.n - 1);
-    const int kend = min(P0 + rlast + 1, a.cap);  // positions [kbeg, kend) are needed
-    const int nkb = (kend + kAttnKeys - 1) / kAttnKeys;
-    // with a sliding window the first row of the CTA sees nothing before P0 + r0 - window + 1
+    const int rlast = min(r0 + kFaRows - 1, a.n - 1);
+    const int kend = min(P0 + rlast + 1, a.cap);
     const int kbeg = a.window > 0 ? max(0, P0 + r0 - a.window + 1) : 0;
-    const int kb0 = kbeg / kAttnKeys;
-    const __half* kbase = a.kcache + (size_t)j * a.cap * DH;
-    const __half* vbase = a.vcache + (size_t)j * a.cap * DH;
+    const int nb = kend > kbeg ? (kend - kbeg + kFaKeys - 1) / kFaKeys : 0;
 
-    auto load_tile = [&](int kb, int buf) {
-        for (int c = tid; c < kAttnKeys * DH / 8; c += 128) {
-            const int r = c / (DH / 8), col = (c % (DH / 8)) * 8;
-            const int pos = kb * kAttnKeys + r;
-            __half* dk = Ks + (buf * kAttnKeys + r) * LDS + col;
-            __half* dv = Vs + (buf * kAttnKeys + r) * LDS + col;
-            if (pos < kend) {
-                cp_async16(dk, kbase + (size_t)pos * DH + col);
-                cp_async16(dv, vbase + (size_t)pos * DH + col);
-            } else {
-                *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
-                *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
-            }
-        }
-        cp_async_commit();
-    };
-
-    const int qr0 = r0 + warp * 16;
-    uint32_t qa[KC][4];
-#pragma unroll
-    for (int kc = 0; kc < KC; ++kc)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const int row = qr0 + g + (e & 1) * 8, col = kc * 16 + 2 * t + (e >> 1) * 8;
-            qa[kc][e] = row < a.n ? *reinterpret_cast<const uint32_t*>(a.q + ((size_t)row * a.hq + h) * DH + col) : 0u;
-        }
-    float o[DT][4];
-#pragma unroll
-    for (int d = 0; d < DT; ++d) o[d][0] = o[d][1] = o[d][2] = o[d][3] = 0.f;
-    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
-    const int qpos[2] = {P0 + qr0 + g, P0 + qr0 + g + 8};
-    const int warp_last = P0 + qr0 + 15;
-    // first position any row of this warp sees (sliding window), and the window's lower bound
-    // of each of the lane's two rows
-    const int warp_first = a.window > 0 ? P0 + qr0 - a.window + 1 : 0;
-    const int qlo[2] = {a.window > 0 ? qpos[0] - a.window + 1 : 0, a.window > 0 ? qpos[1] - a.window + 1 : 0};
-
-    if (kb0 < nkb) load_tile(kb0, kb0 & 1);
-    for (int kb = kb0; kb < nkb; ++kb) {
-        const int buf = kb & 1;
-        if (kb + 1 < nkb) {
-            load_tile(kb + 1, buf ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-        __syncthreads();
-        if (kb * kAttnKeys <= warp_last && (kb + 1) * kAttnKeys - 1 >= warp_first) {
-            const __half* kt = Ks + buf * kAttnKeys * LDS;
-            float s[8][4];
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-                const __half* kr = kt + (nt * 8 + g) * LDS + 2 * t;
-#pragma unroll
-                for (int kc = 0; kc < KC; ++kc) {
-                    const uint32_t b0 = *reinterpret_cast<const uint32_t*>(kr + kc * 16);
-                    const uint32_t b1 = *reinterpret_cast<const uint32_t*>(kr + kc * 16 + 8);
-                    mma16816(s[nt], qa[kc], b0, b1);
+    if (warp == 0) {
+        if (lane == 0 && nb == 0) mbar_wait(q_full, 0);  // no copy may be in flight when the CTA ends
+        if (lane == 0 && nb > 0) {
+            // one thread serves both rings, each load as soon as its slot is free (a blocked wait on
+            // one ring would hold up the other); V_j goes out after K_{j+1}, so that the copies the
+            // first MMAs need (Q, K_0, K_1) are ahead of V in the copy engine
+            const int krow0 = kvh * a.cap + kbeg;
+            auto load = [&](bool is_v, int j) {
+                const int s = j & 1;
+                uint64_t* full = is_v ? &v_full[s] : &k_full[s];
+                mbar_arrive_expect_tx(full, kKVBytes);
+                for (int c = 0; c < DH / 64; ++c)
+                    tc::tma_load_2d((is_v ? Vs : Ks) + s * kKVBytes + c * kAtom, is_v ? &G.tv[gi] : &G.tk[gi], 64 * c,
+                                    krow0 + j * kFaKeys, full);
+            };
+            int jk = 0, jv = 0;
+            uint32_t idle = 0;
+            bool ok = true;
+            while (jk < nb || jv < nb) {
+                bool moved = false;
+                if (jk < nb && (jk < 2 || fa_test(&k_empty[jk & 1], ((jk - 2) >> 1) & 1))) {
+                    load(false, jk++);
+                    moved = true;
+                }
+                if (jv < nb && (jk > jv + 1 || jk == nb) && (jv < 2 || fa_test(&v_empty[jv & 1], ((jv - 2) >> 1) & 1))) {
+                    load(true, jv++);
+                    moved = true;
+                }
+                if (moved) {
+                    idle = 0;
+                } else if (++idle > (kSpinLimit << 2) || *s_err) {
+                    ok = false;
+                    break;
                 }
             }
-            float mx[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int pos = kb * kAttnKeys + nt * 8 + 2 * t + (e & 1);
-                    const float v = (pos <= qpos[e >> 1] && pos >= qlo[e >> 1]) ? s[nt][e] * a.scale_log2 : -INFINITY;
-                    s[nt][e] = v;
-                    mx[e >> 1] = fmaxf(mx[e >> 1], v);
-                }
-            float corr[2];
-#pragma unroll
-            for (int r = 0; r < 2; ++r) {
-                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
-                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
-                const float mn = fmaxf(mrow[r], mx[r]);
-                corr[r] = mn == -INFINITY ? 1.f : exp2f(mrow[r] - mn);
-                mrow[r] = mn;
-            }
-            float ls[2] = {0.f, 0.f};
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float m = mrow[e >> 1];
-                    const float p = m == -INFINITY ? 0.f : exp2f(s[nt][e] - m);
-                    s[nt][e] = p;
-                    ls[e >> 1] += p;
-                }
-#pragma unroll
-            for (int r = 0; r < 2; ++r) lrow[r] = lrow[r] * corr[r] + ls[r];
-#pragma unroll
-            for (int d = 0; d < DT; ++d) {
-                o[d][0] *= corr[0];
-                o[d][1] *= corr[0];
-                o[d][2] *= corr[1];
-                o[d][3] *= corr[1];
-            }
-            const uint32_t vt_base = smem_u32(Vs + buf * kAttnKeys * LDS);
-#pragma unroll
-            for (int kk = 0; kk < kAttnKeys / 16; ++kk) {
-                const uint32_t pa[4] = {pack_h2(s[2 * kk][0], s[2 * kk][1]), pack_h2(s[2 * kk][2], s[2 * kk][3]),
-                                        pack_h2(s[2 * kk + 1][0], s[2 * kk + 1][1]),
-                                        pack_h2(s[2 * kk + 1][2], s[2 * kk + 1][3])};
-                const int vrow = kk * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
-#pragma unroll
-                for (int d = 0; d < DT; d += 2) {
-                    const int vcol = (d + (lane >> 4)) * 8;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_trans(vt_base + (uint32_t)(vrow * LDS + vcol) * 2, b0, b1, b2, b3);
-                    mma16816(o[d], pa, b0, b1);
-                    mma16816(o[d + 1], pa, b2, b3);
-                }
+            if (!ok) {
+                *s_err = 1;
+                set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+                // no copy may still be in flight when the CTA ends
+                mbar_wait(q_full, 0);
+                for (int j = jk > 2 ? jk - 2 : 0; j < jk; ++j) mbar_wait(&k_full[j & 1], (j >> 1) & 1);
+                for (int j = jv > 2 ? jv - 2 : 0; j < jv; ++j) mbar_wait(&v_full[j & 1], (j >> 1) & 1);
             }
         }
-        __syncthreads();
+    } else if (warp == 1) {
+        if (lane == 0 && nb > 0) {
+            constexpr uint32_t idesc_s = tc::idesc_f16(kFaRows, kFaKeys);
+            constexpr uint32_t idesc_o = tc::idesc_f16_bmn(kFaRows, DH);
+            const uint32_t qa = smem_u32(Qs), ka = smem_u32(Ks), va = smem_u32(Vs), pa = smem_u32(Ps);
+            auto qk = [&](int j) -> bool {
+                const int s = j & 1;
+                if (!mbar_wait(&k_full[s], (j >> 1) & 1)) return false;
+                if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1)) return false;
+                if (*s_err) return false;
+                tc::fence_after();
+#pragma unroll
+                for (int kk = 0; kk < DH / 16; ++kk) {
+                    const uint32_t off = (uint32_t)(kk >> 2) * kAtom + (uint32_t)(kk & 3) * 32;
+                    tc::mma_f16(tmem + (uint32_t)(s * kFaKeys), tc::desc_sw128(qa + off),
+                                tc::desc_sw128(ka + s * kKVBytes + off), idesc_s, kk > 0);
+                }
+                tc::mma_commit(&k_empty[s]);
+                tc::mma_commit(&s_full[s]);
+                return true;
+            };
+            auto qk_ready = [&](int j) -> bool {
+                return fa_test(&k_full[j & 1], (j >> 1) & 1) && (j < 2 || fa_test(&s_free[j & 1], ((j - 2) >> 1) & 1));
+            };
+            auto pv = [&](int j) -> bool {
+                const int s = j & 1;
+                if (!mbar_wait(&v_full[s], (j >> 1) & 1)) return false;
+                if (!mbar_wait(&p_full[s], (j >> 1) & 1)) return false;
+                if (*s_err) return false;
+                tc::fence_after();
+#pragma unroll
+                for (int kk = 0; kk < kFaKeys / 16; ++kk)
+                    tc::mma_f16(tmem + kOCol,
+                                tc::desc_sw128(pa + s * kPBytes + (uint32_t)(kk >> 2) * kAtom + (uint32_t)(kk & 3) * 32),
+                                tc::desc_sw128_mn(va + s * kKVBytes + (uint32_t)kk * 2048, kAtom), idesc_o,
+                                (j > 0 || kk > 0) ? 1u : 0u);
+                tc::mma_commit(&v_empty[s]);
+                tc::mma_commit(&o_full[s]);
+                return true;
+            };
+            bool ok = mbar_wait(q_full, 0);
+            ok = ok && qk(0);
+            if (ok && nb > 1) ok = qk(1);
+            for (int j = 0; ok && j < nb; ++j) {
+                bool issued = false;
+                if (j + 2 < nb && qk_ready(j + 2)) {
+                    ok = qk(j + 2);
+                    issued = true;
+                }
+                ok = ok && pv(j);
+                if (ok && j + 2 < nb && !issued) ok = qk(j + 2);
+            }
+            if (!ok) {
+                *s_err = 1;
+                set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+            }
+            // tensor memory is freed only after every MMA issued has completed
+            tc::mma_commit(done);
+            if (!mbar_wait(done, 0)) set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+        }
+    } else {
+        const int g = (warp - 2) >> 2, quad = warp & 3, row = quad * 32 + lane;
+        const uint32_t lane_off = (uint32_t)(quad * 32) << 16, pair = 1u + (uint32_t)quad;
+        const int qp = P0 + r0 + row;
+        const int lo = a.window > 0 ? qp - a.window + 1 : INT_MIN;
+        const float sl2 = a.scale_log2;
+        float m_use = -INFINITY, l = 0.f;
+        bool ok = true;
+        for (int j = 0; j < nb; ++j) {
+            const int s = j & 1;
+            if (ok && *s_err) ok = false;
+            if (ok) ok = fa_wait_warp(&s_full[s], (j >> 1) & 1);
+            // this warp's 64 columns of S_j and their attended range [cb, ce)
+            const int kp0 = kbeg + j * kFaKeys + 64 * g;
+            const int cb = a.window > 0 ? max(0, min(64, lo - kp0)) : 0;
+            const int ce = max(0, min(64, qp - kp0 + 1));
+            uint32_t sv[2][32];
+            float pm = -INFINITY;
+            if (ok) {
+                tc::fence_after();
+                const uint32_t at = tmem + lane_off + (uint32_t)(s * kFaKeys + 64 * g);
+                tc::tmem_ld32(at, sv[0]);
+                tc::tmem_ld32(at + 32, sv[1]);
+                tc::tmem_ld_wait_on(sv[0]);
+                tc::tmem_ld_wait_on(sv[1]);
+                tc::fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s_free[s]);  // S is in registers: the slot may take S_{j+2}
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    const uint32_t mw = fa_range_bits(cb - 32 * c, ce - 32 * c);
+                    if (__all_sync(0xffffffffu, mw == 0xffffffffu)) {
+#pragma unroll
+                        for (int e = 0; e < 32; e += 2)
+                            pm = fa_max3(pm, __uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1]));
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            if ((mw >> e) & 1u) pm = fmaxf(pm, __uint_as_float(sv[c][e]));
+                    }
+                }
+            }
+            // the row maximum over both column halves (every warp passes both barriers)
+            red[g * kFaRows + row] = pm;
+            fa_pair_sync(pair);
+            const float bms = fmaxf(pm, red[(1 - g) * kFaRows + row]) * sl2;
+            fa_pair_sync(pair);
+            // O += P_{j-2} V_{j-2} has completed: P_j's slot is free
+            if (ok && j >= 2) ok = fa_wait_warp(&o_full[s], ((j - 2) >> 1) & 1);
+            if (!ok) continue;
+            float alpha = 1.f;
+            bool resc = false;
+            if (bms > m_use + 8.f) {
+                if (m_use != -INFINITY) {
+                    alpha = fa_ex2(m_use - bms);
+                    resc = true;
+                }
+                m_use = bms;
+            }
+            if (__any_sync(0xffffffffu, resc)) {
+                // O holds every earlier block once O += P_{j-1} V_{j-1} has completed
+                if (j >= 1 && !fa_wait_warp(&o_full[(j - 1) & 1], ((j - 1) >> 1) & 1)) {
+                    ok = false;
+                    continue;
+                }
+                tc::fence_after();
+#pragma unroll
+                for (int c = 0; c < DH / 64; ++c) {
+                    const uint32_t at = tmem + lane_off + kOCol + (uint32_t)(g * (DH / 2) + 32 * c);
+                    uint32_t o[32];
+                    tc::tmem_ld32(at, o);
+                    tc::tmem_ld_wait_on(o);
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                    tc::tmem_st32(at, o);
+                }
+                tc::tmem_st_wait();
+            }
+            l *= alpha;
+            // P_j: this warp's 64 keys are box g of the slot (row `row`, 128-byte swizzle)
+            uint8_t* prow = Ps + s * kPBytes + g * kAtom + row * 128;
+            const float nm = -m_use;
+            float ls0 = 0.f, ls1 = 0.f;
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const uint32_t mw = fa_range_bits(cb - 32 * c, ce - 32 * c);
+                uint32_t w[16];
+                if (__all_sync(0xffffffffu, mw == 0xffffffffu)) {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const float p0 = fa_ex2(fmaf(__uint_as_float(sv[c][2 * e]), sl2, nm));
+                        const float p1 = fa_ex2(fmaf(__uint_as_float(sv[c][2 * e + 1]), sl2, nm));
+                        ls0 += p0;
+                        ls1 += p1;
+                        w[e] = pack_h2(p0, p1);
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const float x0 = ((mw >> (2 * e)) & 1u) ? fmaf(__uint_as_float(sv[c][2 * e]), sl2, nm) : -INFINITY;
+                        const float x1 =
+                            ((mw >> (2 * e + 1)) & 1u) ? fmaf(__uint_as_float(sv[c][2 * e + 1]), sl2, nm) : -INFINITY;
+                        const float p0 = fa_ex2(x0), p1 = fa_ex2(x1);
+                        ls0 += p0;
+                        ls1 += p1;
+                        w[e] = pack_h2(p0, p1);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int chunk = c * 4 + u;
+                    *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) =
+                        make_uint4(w[4 * u], w[4 * u + 1], w[4 * u + 2], w[4 * u + 3]);
+                }
+            }
+            l += ls0 + ls1;
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[s]);
+        }
+        if (ok && nb > 0) ok = fa_wait_warp(done, 0);  // every MMA has completed
+        if (!ok && lane == 0) {
+            *s_err = 1;
+            set_status(a.status, VT_DEV_WAIT_TIMEOUT);
+        }
+        tc::fence_after();
+        // l over both column halves (the same reference maximum)
+        red[g * kFaRows + row] = l;
+        fa_pair_sync(pair);
+        const float lt = l + red[(1 - g) * kFaRows + row];
+        const float inv = lt > 0.f ? 1.f / lt : 0.f;
+        if (ok) {
+            // this warp's half of the row, O columns [g dh/2, (g + 1) dh/2), as fp16 into Q's slot
+            // (free once every MMA is done) in the output's 64-column boxes, 128-byte swizzle
+            uint32_t o[DH / 64][32];
+#pragma unroll
+            for (int c = 0; c < DH / 64; ++c) {
+                if (nb > 0) tc::tmem_ld32(tmem + lane_off + kOCol + (uint32_t)(g * (DH / 2) + 32 * c), o[c]);
+                else
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) o[c][e] = 0u;
+            }
+#pragma unroll
+            for (int c = 0; c < DH / 64; ++c) tc::tmem_ld_wait_on(o[c]);
+#pragma unroll
+            for (int c = 0; c < DH / 64; ++c)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        w[e] = pack_h2(__uint_as_float(o[c][8 * u + 2 * e]) * inv, __uint_as_float(o[c][8 * u + 2 * e + 1]) * inv);
+                    const int col = g * (DH / 2) + 32 * c + 8 * u, box = col >> 6, chunk = (col & 63) >> 3;
+                    *reinterpret_cast<uint4*>(Qs + box * kAtom + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                        make_uint4(w[0], w[1], w[2], w[3]);
+                }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        }
+        // every softmax warp has staged its part (or has given up): one thread stores the boxes
+        asm volatile("bar.sync 5, %0;" ::"n"(kFaThreads - 64) : "memory");
+        if (warp == 2 && lane == 0 && !*s_err) {
+            for (int c = 0; c < DH / 64; ++c) tc::tma_store_2d(&G.to[gi], h * DH + 64 * c, r0, Qs + c * kAtom);
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");  // the slot has been read
+        }
     }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
-        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
-    }
-    const float inv[2] = {lrow[0] > 0.f ? 1.f / lrow[0] : 0.f, lrow[1] > 0.f ? 1.f / lrow[1] : 0.f};
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const int row = qr0 + g + r * 8;
-        if (row >= a.n) continue;
-        __half* dst = a.out + (size_t)row * a.hq * DH + (size_t)h * DH + 2 * t;
-#pragma unroll
-        for (int d = 0; d < DT; ++d)
-            *reinterpret_cast<uint32_t*>(dst + d * 8) = pack_h2(o[d][2 * r] * inv[r], o[d][2 * r + 1] * inv[r]);
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_dealloc(tmem, 512);
     }
 }
 
@@ -1284,11 +1554,11 @@ cudaError_t init_prefill_kernels() {
             g_pgemm_pairs = nc;
         }
     }
-    if ((e = cudaFuncSetAttribute(k_prefill_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)prefill_attn_smem<128>())) != cudaSuccess)
+    if ((e = cudaFuncSetAttribute(k_prefill_attn_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)fa_smem<128>())) != cudaSuccess)
         return e;
-    if ((e = cudaFuncSetAttribute(k_prefill_attn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)prefill_attn_smem<64>())) != cudaSuccess)
+    if ((e = cudaFuncSetAttribute(k_prefill_attn_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)fa_smem<64>())) != cudaSuccess)
         return e;
     return cudaSuccess;
 }
@@ -1580,39 +1850,50 @@ static GemmSpec o_spec(const PrefillAttnArgs& a) {
     return GemmSpec{a.attn, K, a.wo, K, a.d, K, o};
 }
 
-// Causal attention of every shard of an ATTN block in one launch (all with the same rows).
-static vt_status prefill_attention(const PrefillAttnArgs* as, int n, cudaStream_t st, std::string* err) {
-    PrefillAttnGroup G{};
-    int heads = 0;
-    for (int i = 0; i < n; ++i) {
-        const PrefillAttnArgs& a = as[i];
-        PrefillAttnKArgs& t = G.a[i];
-        t.q = a.q;
-        t.kcache = a.kcache;
-        t.vcache = a.vcache;
-        t.len = a.len;
-        t.row_offset = a.row_offset;
-        t.n = a.n;
-        t.hq = a.hq;
-        t.group = a.hq / a.hk;
-        t.cap = a.cap;
-        t.window = a.window;
-        t.scale_log2 = a.scale_log2;
-        t.out = a.attn;
-        heads += a.hq;
-        G.head_end[i] = heads;
-    }
-    G.n_groups = n;
-    if (n < 1 || heads < 1) return VT_OK;
-    const dim3 grid(heads, (as[0].n + kAttnRows - 1) / kAttnRows);
-    if (as[0].dh == 128) k_prefill_attn<128><<<grid, 128, prefill_attn_smem<128>(), st>>>(G);
-    else k_prefill_attn<64><<<grid, 128, prefill_attn_smem<64>(), st>>>(G);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) {
-        *err = std::string("prefill attention launch failed: ") + cudaGetErrorString(e);
-        return VT_ERR_CUDA;
+// Causal attention of every shard of an ATTN block on tcgen05: one launch per kFaGroups shards.
+static vt_status prefill_attention_tc(const PrefillAttnArgs* as, int n, cudaStream_t st, std::string* err) {
+    for (int g0 = 0; g0 < n; g0 += kFaGroups) {
+        const int ng = std::min(kFaGroups, n - g0);
+        FaGroup G{};
+        int heads = 0;
+        for (int i = 0; i < ng; ++i) {
+            const PrefillAttnArgs& a = as[g0 + i];
+            FaShard& t = G.a[i];
+            t.n = a.n;
+            t.hq = a.hq;
+            t.group = a.hq / a.hk;
+            t.cap = a.cap;
+            t.row_offset = a.row_offset;
+            t.window = a.window;
+            t.len = a.len;
+            t.scale_log2 = a.scale_log2;
+            t.out = a.attn;
+            t.status = a.status;
+            if (!make_map(&G.tq[i], a.q, (int64_t)a.hq * a.dh, a.n, (int64_t)a.hq * a.dh, kFaRows, err) ||
+                !make_map(&G.tk[i], a.kcache, a.dh, (int64_t)a.hk * a.cap, a.dh, kFaKeys, err) ||
+                !make_map(&G.tv[i], a.vcache, a.dh, (int64_t)a.hk * a.cap, a.dh, kFaKeys, err) ||
+                !make_map(&G.to[i], a.attn, (int64_t)a.hq * a.dh, a.n, (int64_t)a.hq * a.dh, kFaRows, err))
+                return VT_ERR_CUDA;
+            heads += a.hq;
+            G.head_end[i] = heads;
+        }
+        G.n_groups = ng;
+        if (heads < 1 || as[0].n < 1) continue;
+        const dim3 grid(heads, (as[0].n + kFaRows - 1) / kFaRows);
+        if (as[0].dh == 128) k_prefill_attn_tc<128><<<grid, kFaThreads, fa_smem<128>(), st>>>(G);
+        else k_prefill_attn_tc<64><<<grid, kFaThreads, fa_smem<64>(), st>>>(G);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) {
+            *err = std::string("prefill attention launch failed: ") + cudaGetErrorString(e);
+            return VT_ERR_CUDA;
+        }
     }
     return VT_OK;
+}
+
+// Causal attention of every shard of an ATTN block (all with the same rows).
+static vt_status prefill_attention(const PrefillAttnArgs* as, int n, cudaStream_t st, std::string* err) {
+    return prefill_attention_tc(as, n, st, err);
 }
 
 vt_status prefill_attn_shard(const PrefillAttnArgs& a, cudaStream_t st, std::string* err) {

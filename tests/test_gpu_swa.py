@@ -178,6 +178,33 @@ def test_prefill_shard_window(vtlib, pos0, n, W):
         assert vt.vt_kv_status(st.kv) == 0
 
 
+@pytest.mark.parametrize("cid,pos0,n,W", [(1, 1000, 300, 0), (1, 1000, 300, 700), (5, 900, 260, 0), (5, 900, 260, 300)])
+def test_prefill_long_history(vtlib, cid, pos0, n, W):
+    """Prompt rows after a long cached history: up to 11 blocks of 128 keys per row tile, so the
+    two-slot K/V rings are refilled many times and every row's running maximum meets new blocks;
+    with and without a window, at dh 64 (config 1) and dh 128 with 4 query heads per KV head
+    (config 5).  Per-shard attention partials on sampled rows against the oracle."""
+    vt = vtlib
+    wl = dataclasses.replace(synthetic.WORKLOADS[cid], n_layers=1)
+    w = wl.layer_weights(0)
+    cap = pos0 + n + 8
+    kc, vc = wl.kv_fill(0, pos0, cap)
+    X = wl.hidden(n, stream=260 + cid + W)
+    rows = np.array([0, 1, 127, 128, 200, 255, 256, n - 1])
+    D = wl.d_model
+    with stack(vt, wl, cap, W) as st:
+        fill(vt, st, 0, wl, kc, vc, pos0)
+        parts = [torch.empty((n, D), dtype=torch.float32, device="cuda") for _ in wl.head_ranges]
+        for d in range(len(wl.head_ranges)):
+            vt.vt_prefill(st.part, (0, d, ATTN), dev(X), n, st.kv, parts[d])
+        for hr in wl.head_ranges:
+            oracle.kv_append(wl, w, oracle.kv_heads_of(wl, hr), X, pos0, kc, vc)
+        for d, hr in enumerate(wl.head_ranges):
+            ap = oracle.attn_partial(wl, w, hr, X[rows], pos0 + rows, kc, vc, W)
+            assert_close(host(parts[d])[rows], ap, f"cid {cid} pos0 {pos0} W {W} partial dev {d}")
+        assert vt.vt_kv_status(st.kv) == 0
+
+
 def test_prefill_tokens_windows_two_layers(vtlib):
     """The whole-stack prefill with windows 64 and 0 on two layers, and then a decode token on the
     cache it wrote, against the oracle chained layer by layer."""
