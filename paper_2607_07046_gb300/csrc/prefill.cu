@@ -405,6 +405,7 @@ struct GemmGroup {
     CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
     GemmArgs a[kGemmGroups];
 };
+static_assert(sizeof(GemmGroup) <= 4096, "the GEMM launch's parameters must fit in 4 KB");
 
 // 16-byte slot of the split-K receive buffer that holds floats [4e, 4e + 4) of 32-column chunk
 // `chunk` of local row `lr`.  128-bit shared accesses are served 8 threads at a time; the slot
@@ -701,6 +702,8 @@ struct PGemmGroup {
     CUtensorMap ta[kGemmGroups], tb[kGemmGroups];
     GemmArgs a[kGemmGroups];
 };
+
+static_assert(sizeof(PGemmGroup) <= 4096, "the GEMM launch's parameters must fit in 4 KB");
 
 // Tile t of the group: the row tile (tm rows: 128, or 256 for a CTA pair) is the fastest index.
 __device__ __forceinline__ void ptile(const PGemmGroup& G, int t, int& g, int& m0, int& n0) {
@@ -1086,6 +1089,8 @@ struct FaGroup {
     CUtensorMap to[kFaGroups];                                 // the output [n][hq dh]
     FaShard a[kFaGroups];
 };
+
+static_assert(sizeof(FaGroup) <= 4096, "the attention launch's parameters must fit in 4 KB");
 
 // Q, two K and two V slots, two P slots, the max exchange (2 x 128 floats), barriers
 template <int DH>

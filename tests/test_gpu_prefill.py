@@ -152,6 +152,9 @@ UNEVEN = [
     (8, 4, ((0, 2), (2, 8)), ((0, 9), (9, 1408))),
     (8, 2, ((0, 4), (4, 8)), ((0, 704), (704, 1408))),
     (8, 1, ((0, 8),), ((0, 1408),)),
+    # nine shards (one head each and an empty one): more than one launch per block for the
+    # attention (six shards a launch) and the GEMMs (eight)
+    (8, 8, tuple((h, h + 1) for h in range(8)) + ((8, 8),), tuple((i * 1408 // 9, (i + 1) * 1408 // 9) for i in range(9))),
 ]
 
 
