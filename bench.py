@@ -536,9 +536,20 @@ def run_decode(args, rank, world):
         "setup_s": round(setup_s, 1),
     }
     if sharded_ms is not None:
+        # the same token through the per-shard entry points: the same bytes at its own schedule's
+        # mean KV length
+        sh_bytes = decode_bytes_per_token(wl, wl.kv_len + (min(args.sharded_steps, sched) - 1) / 2.0)
+        sh_achieved = sh_bytes / (sharded_ms * 1e-3) / 1e9
         line["sharded_token"] = {"ms_per_step": round(sharded_ms, 5), "value": round(1000.0 / sharded_ms, 3),
                                  "unit": "tok/s", "steps": args.sharded_steps,
-                                 "note": "vt_decode_token_sharded: per-shard kernels with PDL, for context"}
+                                 "note": "vt_decode_token_sharded: per-shard kernels with PDL, for context",
+                                 "roofline": {"bound": "hbm",
+                                              "kernel": "the whole token step (k_gemv, k_attn_decode, k_ffn and "
+                                                        "k_combine for every shard and block)",
+                                              "achieved": round(sh_achieved, 1), "peak": hbm, "unit": "GB/s",
+                                              "frac": round(sh_achieved / hbm, 4),
+                                              "peak_kind": f"{peak_kind} copy bandwidth",
+                                              "bytes_per_step": int(sh_bytes)}}
     if prefill is not None:
         line["prefill"] = prefill
         line["gpu_launches"] += prefill["gpu_launches"]
