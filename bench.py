@@ -165,7 +165,8 @@ def decode_bytes_per_token(wl, kv_mean):
 def quant_bytes_per_token(wl, bits, kv_mean):
     """Algorithmic HBM bytes of one decode token with every shard block-quantized at `bits`: the
     codes (one byte per weight at 8 bits, half a byte at 4; rows padded to whole blocks of 32) and
-    one fp16 scale per block of every projection, the RMSNorm gains, the cache at the mean length."""
+    one fp16 scale per block of every projection, the layer's two RMSNorm gains (one buffer each,
+    as in decode_bytes_per_token), the cache at the mean length."""
     D, H, Hk, dh, F, L = wl.d_model, wl.n_heads, wl.n_kv_heads, wl.d_head, wl.d_ffn, wl.n_layers
     cb = 1.0 if bits == 8 else 0.5
 
@@ -173,14 +174,14 @@ def quant_bytes_per_token(wl, bits, kv_mean):
         nb = (k + 31) // 32
         return rows * (nb * 32 * cb + nb * 2)
 
-    w = 0.0
+    w = 2.0 * 2 * D
     for (h0, h1), (c0, c1) in zip(wl.head_ranges, wl.ffn_ranges):
         hq, c = h1 - h0, c1 - c0
         hk = hq * Hk // H
         if hq:
-            w += mat((hq + 2 * hk) * dh, D) + mat(D, hq * dh) + 2 * D
+            w += mat((hq + 2 * hk) * dh, D) + mat(D, hq * dh)
         if c:
-            w += mat(2 * c, D) + mat(D, c) + 2 * D
+            w += mat(2 * c, D) + mat(D, c)
     kv = 2 * 2 * Hk * dh * (kv_mean + 1)
     return int(L * (w + kv))
 
