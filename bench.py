@@ -270,8 +270,9 @@ def prefill_attn_flops(wl, n):
 
 
 def run_prefill(vt, st, wl, stream, steps, warmup):
-    """The 512-token prompt of the 7B prefill workload through every layer (vt_prefill_tokens,
-    shards one after another), captured with the embedding and a KV rewind as one CUDA graph."""
+    """The 512-token prompt of the 7B prefill workload through every layer (vt_prefill_tokens: the
+    shards of a block together, one launch per projection and one for the attention), captured
+    with the embedding and a KV rewind as one CUDA graph."""
     import torch
     wp = synthetic.WORKLOADS[4]
     n, D = wp.prompt_len, wl.d_model
@@ -299,10 +300,10 @@ def run_prefill(vt, st, wl, stream, steps, warmup):
     gemm = prefill_gemm_flops(wl, n)
     tflops = gemm / (ms * 1e-3) / 1e12
     n_dev = len(wl.head_ranges)
-    # kernels per prompt: embedding, the first RMSNorm, per layer (per ATTN shard: QKV GEMM,
-    # attention, O GEMM; combine + RMSNorm; per FFN shard: gate/up GEMM, down GEMM; combine +
+    # kernels per prompt: embedding, the first RMSNorm, per layer (QKV, O, gate/up and down GEMMs,
+    # one launch each per 8 shards; the attention, one launch per 6 shards; two combines +
     # RMSNorm), KV advance and rewind
-    launches = 2 + wl.n_layers * (3 * n_dev + 1 + 2 * n_dev + 1) + 2
+    launches = 2 + wl.n_layers * (4 * -(-n_dev // 8) + -(-n_dev // 6) + 2) + 2
     return {
         "workload": f"llama2-7b-shaped prefill: {n}-token prompt (seeded ids, embedding gather), "
                     f"{wl.n_layers} layers, even {n_dev}-way TP on 1 GPU (one grouped GEMM launch per "
